@@ -1,0 +1,465 @@
+"""Benchmark: the Qwen3-shaped decode-step weight pass (W3G128 by default) on GB300.
+
+One step = one replay of a CUDA graph holding every quantized projection of the model once
+(36 layers x q, k, v, o, gate, up, down = 252 ``laq_gemm_wxg128`` launches, M = 1), i.e. the
+weight streaming of one batch-1 decode step.  Quantization and packing (``laq_quantize_rtn``,
+``laq_pack``) are the offline model-preparation steps and run once before timing; their time is
+reported as ``prep_ms``.  Synthetic weights ~ N(0, 0.02^2) and activations ~ N(0, 1) stand in
+for the paper's Qwen3 checkpoints.
+
+Prints one JSON line.  ``value`` is the achieved HBM bandwidth of the pass (algorithmic bytes =
+packed codes + s + z + X + Y, per step, all ranks) over the device time of the timed replays.
+
+    python bench.py [--steps K] [--warmup W] [--model qwen3-4b|qwen3-8b] [--bits 3|4] [--M 1]
+    python bench.py --impl reference      # the CPU oracle, timed on the host cores
+    torchrun --nproc-per-node N bench.py --gpus N   # N independent replicas (no data exchange)
+"""
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "W3G128 dequant-GEMV HBM GB/s (% of peak); µs per Qwen3-4B-shaped decode step"
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=4000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", default="laq", choices=["laq", "reference"])
+    ap.add_argument("--model", default="qwen3-4b", choices=["qwen3-4b", "qwen3-8b"])
+    ap.add_argument("--bits", type=int, default=3, choices=[3, 4])
+    ap.add_argument("--M", type=int, default=1)
+    ap.add_argument("--layers", type=int, default=36)
+    ap.add_argument("--no-fp16", action="store_true", help="skip the fp16 torch.matmul context")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0,
+                    help="CPU work budget of the oracle baseline sample")
+    return ap.parse_args()
+
+
+def workload_name(a):
+    return (f"{a.model} decode-step weight pass, {a.layers} layers x 7 projections, "
+            f"W{a.bits}G128, M={a.M}, one CUDA graph")
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    return 6800.0, "fallback"
+
+
+# ------------------------------------------------------------------ distributed plumbing
+
+
+def dist_setup(a):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        backend = "nccl" if a.impl == "laq" else "gloo"
+        if backend == "nccl":
+            import torch
+            torch.cuda.set_device(local)
+        dist.init_process_group(backend=backend)
+    return world, rank, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(world, value, device=None):
+    if world == 1:
+        return value
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def sum_over_ranks(world, value, device=None):
+    if world == 1:
+        return value
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.SUM)
+    return float(t.item())
+
+
+# ------------------------------------------------------------------ clocks
+
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons while the timed region runs."""
+
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.out = None
+
+    def __enter__(self):
+        try:
+            self.out = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.Q}", "--format=csv,noheader,nounits",
+                 "-i", str(self.gpu), "-lms", "100"], stdout=self.out,
+                stderr=subprocess.DEVNULL)
+        except (OSError, ValueError):
+            self.proc = None
+        time.sleep(0.3)
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        if self.proc is None or self.out is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.out.flush()
+        rows = []
+        with open(self.out.name) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    rows.append((float(parts[1]), float(parts[2]), float(parts[3]), parts[4:]))
+                except ValueError:
+                    continue
+        os.unlink(self.out.name)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = set()
+        for *_, flags in rows:
+            for n, v in zip(names, flags[1:]):
+                if v.strip().lower() == "active":
+                    reasons.add(n)
+        loaded = [r for r in rows if r[2] > 0] or rows
+        return {"sm_mhz": statistics.median(r[0] for r in loaded),
+                "sm_max_mhz": max(r[1] for r in rows), "reasons": sorted(reasons),
+                "samples": len(rows), "power_w_max": max(r[2] for r in rows)}
+
+
+# ------------------------------------------------------------------ CPU oracle baseline
+
+
+class OracleSample:
+    """A bounded sample of the same workload for the C oracle: the projections of layer 0 (same
+    shapes, distributions and seeds recipe), quantized once by the oracle (untimed).  ``run``
+    times the oracle's fp64 dequantize-and-multiply over whole projections (or a leading
+    column slice of one, when a short step is asked for)."""
+
+    def __init__(self, model, bits, M, seed=0):
+        from oracle import c_oracle
+        from paper_2605_08755_gb300 import inputs
+        from paper_2605_08755_gb300.weight_pass import shapes
+        self.co = c_oracle
+        self.bits, self.M = bits, M
+        self.items = []
+        for pi, (name, K, N) in enumerate(shapes(model)):
+            sd = inputs.proj_seed(seed, 0, pi)
+            W = inputs.weights(K, N, sd, outliers=(model == "qwen3-8b"))
+            codes, s, z = c_oracle.quantize_rtn(W, bits)
+            self.items.append((f"L0.{name}", codes, s, z, inputs.activations(M, K, sd)))
+        self.next = 0
+
+    def nbytes(self, K, N):
+        return K * N * self.bits // 8 + (K // 128) * N * 3 + 2 * self.M * K + 2 * self.M * N
+
+    def run(self, seconds, max_cols=None):
+        """Oracle work for about ``seconds``; returns (bytes, seconds spent, items done)."""
+        done = 0
+        spent = 0.0
+        names = []
+        while True:   # at least one item
+            name, codes, s, z, X = self.items[self.next % len(self.items)]
+            self.next += 1
+            K, N = codes.shape
+            if max_cols is not None and max_cols < N:
+                codes, s, z = (codes[:, :max_cols].copy(), s[:, :max_cols].copy(),
+                               z[:, :max_cols].copy())
+                N = max_cols
+                name += f"[:, :{N}]"
+            t0 = time.perf_counter()
+            self.co.gemm(X, codes, s, z)
+            spent += time.perf_counter() - t0
+            done += self.nbytes(K, N)
+            names.append(name)
+            if spent >= seconds:
+                break
+        return done, spent, names
+
+
+# ------------------------------------------------------------------ reference arm
+
+
+def run_reference(a, world, rank):
+    """The oracle, as it stands, on the host cores: each step is a bounded sample of the pass
+    (a column slice of one projection, sized so the whole run stays within a few minutes)."""
+    if rank != 0:
+        return
+    smp = OracleSample(a.model, a.bits, a.M)
+    per_step_s = min(0.25, max(0.002, 90.0 / max(1, a.steps + a.warmup)))
+    # calibrate columns per step on the first projection
+    name, codes, *_ = smp.items[0]
+    K, N = codes.shape
+    b, sp, _ = smp.run(0.0, max_cols=64)
+    cols = int(max(16, min(N, 64 * per_step_s / max(sp, 1e-6))) // 16 * 16)
+    smp.next = 0
+    for _ in range(a.warmup):
+        smp.run(0.0, max_cols=cols)
+    tot_b, tot_s, names = 0, 0.0, []
+    step_s = []
+    for _ in range(a.steps):
+        b, sp, nm = smp.run(0.0, max_cols=cols)
+        tot_b += b
+        tot_s += sp
+        step_s.append(sp)
+        names += nm
+    value = tot_b / tot_s / 1e9
+    sample = (f"C oracle (fp64, one thread) dequantize-and-multiply; each step = the first "
+              f"{cols} columns of one layer-0 projection, round-robin over q,k,v,o,gate,up,down; "
+              f"{tot_s:.1f} s of CPU work over {a.steps} steps; quantization not timed")
+    line = {"metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": a.gpus,
+            "steps": a.steps, "warmup": a.warmup,
+            "ms_per_step": 1e3 * statistics.median(step_s), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "impl": "reference", "config": {"workload": workload_name(a), "model": a.model},
+            "cpu_baseline": {"value": value, "unit": "GB/s", "cores": 1, "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": value, "unit": "GB/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# ------------------------------------------------------------------ GPU arm
+
+
+def fp16_context(a, dev, steps=50):
+    """Time torch.matmul in fp16 over the same 252 shapes in one CUDA graph (context ratio)."""
+    import torch
+
+    from paper_2605_08755_gb300 import inputs
+    from paper_2605_08755_gb300.weight_pass import shapes
+    Ws, Xs, Ys = [], [], []
+    for layer in range(a.layers):
+        for pi, (_, K, N) in enumerate(shapes(a.model)):
+            sd = inputs.proj_seed(0, layer, pi)
+            Ws.append(inputs.weights_torch(K, N, sd, dev))
+            Xs.append(inputs.activations_torch(a.M, K, sd, dev))
+            Ys.append(torch.empty((a.M, N), dtype=torch.float16, device=dev))
+
+    def run():
+        for W, X, Y in zip(Ws, Xs, Ys):
+            torch.matmul(X, W, out=Y)
+
+    run()
+    torch.cuda.synchronize(dev)
+    g = torch.cuda.CUDAGraph()
+    s = torch.cuda.Stream(dev)
+    with torch.cuda.graph(g, stream=s):
+        run()
+    for _ in range(5):
+        g.replay()
+    torch.cuda.synchronize(dev)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(steps):
+        g.replay()
+    e1.record()
+    torch.cuda.synchronize(dev)
+    us = e0.elapsed_time(e1) * 1e3 / steps
+    nbytes = sum(W.numel() * 2 for W in Ws) + sum(X.numel() * 2 for X in Xs) + \
+        sum(Y.numel() * 2 for Y in Ys)
+    del Ws, Xs, Ys, g
+    torch.cuda.empty_cache()
+    return us, nbytes
+
+
+def run_laq(a, world, rank, local):
+    import torch
+
+    import __graft_entry__
+    from paper_2605_08755_gb300.weight_pass import WeightPass
+
+    __graft_entry__.build()
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    peak, peak_kind = load_peaks()
+
+    t0 = time.perf_counter()
+    wp = WeightPass(model=a.model, bits=a.bits, M=a.M, layers=a.layers,
+                    outliers=(a.model == "qwen3-8b"), device=dev)
+    prep_ms = (time.perf_counter() - t0) * 1e3
+    bytes_step = wp.bytes_per_pass()
+
+    # Plain graph for the timed region; a second capture of the same launches carries an
+    # external timing event before every launch and after the last, so each launch's device
+    # time is measured on the stream it runs on, in replays right after the timed region.
+    stream = torch.cuda.Stream(dev)
+    graph = wp.capture(stream=stream)
+    try:
+        events = [torch.cuda.Event(enable_timing=True, external=True)
+                  for _ in range(wp.launches + 1)]
+        igraph = wp.capture(stream=stream, events=events)
+    except TypeError:
+        events, igraph = None, None
+
+    with torch.cuda.stream(stream):
+        for _ in range(a.warmup):
+            graph.replay()
+    torch.cuda.synchronize(dev)
+
+    step_ms = []
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(a.steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(a.steps)]
+    with ClockSampler(local) as clk:
+        barrier(world)
+        torch.cuda.synchronize(dev)
+        with torch.cuda.stream(stream):
+            for i in range(a.steps):
+                starts[i].record(stream)
+                graph.replay()
+                ends[i].record(stream)
+        torch.cuda.synchronize(dev)
+        barrier(world)
+    clocks = clk.summary()
+    for i in range(a.steps):
+        step_ms.append(starts[i].elapsed_time(ends[i]))
+    total_ms = starts[0].elapsed_time(ends[-1])
+    total_ms = max_over_ranks(world, total_ms, dev)
+    ms_per_step = total_ms / a.steps
+    value = sum_over_ranks(world, bytes_step * a.steps, dev) / (total_ms * 1e-3) / 1e9
+
+    per_launch = [0.0] * wp.launches
+    reps = 20
+    if igraph is not None:
+        with torch.cuda.stream(stream):
+            for _ in range(reps):
+                igraph.replay()
+                torch.cuda.synchronize(dev)
+                for j in range(wp.launches):
+                    per_launch[j] += events[j].elapsed_time(events[j + 1]) / reps
+        kernel_ms = sum(per_launch)
+        ievent_ms = events[0].elapsed_time(events[-1])
+    else:
+        kernel_ms, ievent_ms = ms_per_step, None
+    kernel_gbs = bytes_step / (kernel_ms * 1e-3) / 1e9
+    by_name = {}
+    for (layer, pi, name, q), t in zip(wp.linears, per_launch):
+        d = by_name.setdefault(name, [0.0, 0])
+        d[0] += t * 1e3
+        d[1] += q.bytes_per_call(a.M)
+    per_proj = {k: {"us_per_launch": v[0] / a.layers,
+                    "gbs": v[1] / (v[0] * 1e-6) / 1e9 if v[0] else None}
+                for k, v in by_name.items()}
+
+    # end to end through the public API with host buffers
+    xh = torch.empty_like(wp.Xbuf, device="cpu").pin_memory()
+    xh.copy_(wp.Xbuf)
+    yh = torch.empty_like(wp.Ybuf, device="cpu").pin_memory()
+    e2e_steps = max(10, min(a.steps, 400))
+    torch.cuda.synchronize(dev)
+    e_a, e_b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        e_a.record(stream)
+        for _ in range(e2e_steps):
+            wp.Xbuf.copy_(xh, non_blocking=True)
+            graph.replay()
+            yh.copy_(wp.Ybuf, non_blocking=True)
+        e_b.record(stream)
+    torch.cuda.synchronize(dev)
+    e2e_ms = max_over_ranks(world, e_a.elapsed_time(e_b), dev) / e2e_steps
+    e2e_gbs = sum_over_ranks(world, bytes_step, dev) / (e2e_ms * 1e-3) / 1e9
+
+    fp16_us = None
+    if not a.no_fp16 and rank == 0:
+        fp16_us, _ = fp16_context(a, dev)
+
+    cpu = None
+    if rank == 0:
+        smp = OracleSample(a.model, a.bits, a.M)
+        b, spent, names = smp.run(a.cpu_seconds)
+        cpu = {"value": b / spent / 1e9, "unit": "GB/s", "cores": 1, "kind": "oracle",
+               "sample": f"C oracle (fp64, one thread) dequantize-and-multiply of "
+                         f"{len(names)} whole projections of layer 0, round-robin over "
+                         f"q,k,v,o,gate,up,down, {spent:.1f} s of CPU work; quantization not "
+                         f"timed"}
+
+    if rank != 0:
+        return
+    line = {
+        "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": world, "steps": a.steps,
+        "warmup": a.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "u3+f16 (fp32 accumulate)"
+        if a.bits == 3 else "u4+f16 (fp32 accumulate)", "data": "synthetic",
+        "config": {"workload": workload_name(a), "model": a.model, "bits": a.bits, "M": a.M,
+                   "launches_per_step": wp.launches, "bytes_per_step": bytes_step,
+                   "us_per_step": ms_per_step * 1e3,
+                   "pct_of_peak": 100.0 * value / world / peak,
+                   "peak_gbs": peak, "peak_kind": peak_kind,
+                   "l2": "inputs larger than L2 (packed weights per step >> 129 MB)",
+                   "step_ms_p10_p50_p90": [sorted(step_ms)[int(0.1 * (len(step_ms) - 1))],
+                                           statistics.median(step_ms),
+                                           sorted(step_ms)[int(0.9 * (len(step_ms) - 1))]],
+                   "prep_ms": prep_ms,
+                   "fp16_torch_matmul_us_per_step": fp16_us,
+                   "speedup_vs_fp16_torch": (fp16_us / (ms_per_step * 1e3)) if fp16_us else None,
+                   "parallelism": f"replicas x{world}"},
+        "roofline": {"bound": "hbm", "achieved": kernel_gbs, "peak": peak, "unit": "GB/s",
+                     "frac": kernel_gbs / peak, "traffic": None,
+                     "kernel": "gemm_kernel, all launches of one step: algorithmic bytes / "
+                               "sum of per-launch event times",
+                     "peak_kind": peak_kind, "kernel_us_per_step": kernel_ms * 1e3,
+                     "instrumented_step_us": None if ievent_ms is None else ievent_ms * 1e3,
+                     "per_projection": per_proj},
+        "cpu_baseline": cpu,
+        "e2e": {"value": e2e_gbs, "unit": "GB/s", "h2d_bytes_per_step": wp.Xbuf.numel() * 2,
+                "d2h_bytes_per_step": wp.Ybuf.numel() * 2, "us_per_step": e2e_ms * 1e3},
+        "gpu_launches": wp.launches * a.steps,
+        "clocks": clocks,
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    a = parse()
+    world, rank, local = dist_setup(a)
+    if a.impl == "reference":
+        run_reference(a, world, rank)
+    else:
+        run_laq(a, world, rank, local)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

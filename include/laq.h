@@ -1,0 +1,168 @@
+/*
+ * laq.h -- C ABI of the weight-only WbG128 (b = 3 or 4) quantized linear layer for NVIDIA GB300
+ * (sm_103a): RTN group quantizer, bit packing, and the dequantize-fused GEMV / skinny GEMM
+ * Y[M,N] = X[M,K] * W_hat[K,N] for M = 1..16 (LAQuant, arXiv 2605.08755).
+ *
+ * Quantization format (Eq. (1) and Sec. 2 "Grouped quantization"): every weight w is a b-bit
+ * code q in [0, 2^b - 1] with a scale s and a zero z shared by a group of g = 128 consecutive
+ * elements of a weight row, and w_hat = s * (q - z).  With the weight stored as W[K][N]
+ * (K = in_features, N = out_features) a group is 128 consecutive k of one column n, and the
+ * scales and zeros form (num_groups, out_features) tensors as in App. H ("Group-wise
+ * quantization").  No online transform is applied to X (Sec. 3, "Runtime-overhead-free
+ * quantization").
+ *
+ * Conventions shared by every entry point:
+ *   - Pointers are caller-owned DEVICE memory unless stated otherwise.  The library never
+ *     allocates, frees or synchronizes, and never reads device memory on the host.
+ *   - `stream` is a cudaStream_t (NULL = the legacy default stream).  Work is enqueued
+ *     asynchronously on it; results are ready when the stream says so.
+ *   - Arguments are validated on the host first.  An invalid call returns its status and
+ *     enqueues nothing.  A launch failure returns LAQ_ERR_CUDA.
+ *   - Matrices are dense row-major with no padding: X[M][K] and Y[M][N] fp16, W[K][N] fp16,
+ *     codes[K][N] uint8, s[K/128][N] fp16, z[K/128][N] uint8.
+ *   - Empty shapes are legal: a call with M, K or N equal to 0 writes only the (possibly
+ *     empty) outputs it defines (a GEMM with K = 0 sets Y to zero).
+ *   - Every entry point that takes a stream may be captured into a CUDA graph, provided the
+ *     first call for each (bits, M-class) variant happens before capture begins (that first
+ *     call sets the kernel's shared-memory limit and caches the device's SM count).
+ */
+#ifndef LAQ_H
+#define LAQ_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    LAQ_OK = 0,
+    LAQ_ERR_NULL = 1,     /* a required pointer is NULL                                  */
+    LAQ_ERR_BITS = 2,     /* bits is not 3 or 4                                          */
+    LAQ_ERR_GROUP = 3,    /* group size is not 128                                       */
+    LAQ_ERR_SHAPE = 4,    /* negative size, K % 128 != 0, N % 16 != 0, or a size too big */
+    LAQ_ERR_ALIGN = 5,    /* a pointer breaks its alignment requirement                  */
+    LAQ_ERR_M_RANGE = 6,  /* M outside 0..16                                             */
+    LAQ_ERR_CUDA = 7,     /* the CUDA runtime reported an error for the launch           */
+    LAQ_ERR_TIMEOUT = 8,  /* reserved: a bounded device-side wait gave up                */
+    LAQ_ERR_CONFIG = 9    /* an explicit launch configuration is not supported           */
+} laq_status;
+
+/* Human-readable name of a status code (static storage, never NULL). */
+const char *laq_status_str(int status);
+
+/* ABI version of this header: 1. */
+int laq_version(void);
+
+/* Bytes of packed codes for a K x N weight at `bits` per code: K * N * bits / 8 exactly (no
+ * padding).  Returns 0 for invalid arguments. */
+size_t laq_packed_bytes(int64_t K, int64_t N, int bits);
+
+/*
+ * laq_quantize_rtn -- min-max round-to-nearest group quantizer of Eq. (1).
+ *
+ *   W      [K][N] fp16, finite values.                                  (in,  2-byte aligned)
+ *   codes  [K][N] uint8, q = clip(rint(w / s) + z, 0, 2^b - 1).          (out)
+ *   s      [K/128][N] fp16 group scales.                                 (out, 2-byte aligned)
+ *   z      [K/128][N] uint8 group zeros in [0, 2^b - 1].                 (out)
+ *   bits   3 or 4;  group must be 128;  K % 128 == 0.
+ *
+ * Eq. (1) fixes q and w_hat given s and z; the paper learns s and z by QAT.  This initializer
+ * fixes them per (group, column) from lo = min w, hi = max w, in fp64:
+ *   - constant group (lo == hi == c): s = |c| (1.0 if c == 0), z = 1 if c < 0 else 0, so
+ *     w_hat == c exactly;
+ *   - otherwise lo' = min(lo, 0), hi' = max(hi, 0), s = the smallest fp16 >= (hi' - lo') /
+ *     (2^b - 1), raised to 2^-14 if below it, and z = rint(-lo' / s);
+ *   - rint is round-half-to-even and is applied to w / s before z is added, as Eq. (1) reads.
+ * Consequences: 0 <= z <= 2^b - 1 and |w - w_hat| <= s / 2 for every element.  Results are
+ * deterministic and bit-identical to a plain fp64 implementation of the rule above.
+ * Non-finite inputs give unspecified codes.
+ */
+laq_status laq_quantize_rtn(const void *W, int64_t K, int64_t N, int bits, int group,
+                            uint8_t *codes, void *s, uint8_t *z, void *stream);
+
+/*
+ * laq_pack -- codes[K][N] (values < 2^bits) -> packed words, the layout laq_gemm_wxg128 reads.
+ * App. H keeps the INT3 kernel's "32 weights in three 32-bit words" packing; this library uses
+ * its own layout with the same density (K * N * bits / 8 bytes), built around the tensor-core
+ * fragment that consumes it.  Requires K % 128 == 0, N % 16 == 0, packed 16-byte aligned.
+ *
+ * Layout.  Codes are grouped into records of 16 columns x 128 rows: record (t, g) covers
+ * columns n = 16t..16t+15 and rows k = 128g..128g+127 and is stored at record index
+ * t * (K/128) + g (tile-major).  A record is 32 * bits 32-bit words (1024 bytes at b = 4, 768
+ * at b = 3) and is split among 32 lanes; lane l (c = l % 4, r = l / 4) owns the 64 codes at
+ * columns r and r + 8 of the tile and rows k = 16j + 8h + 2c + e (j = 0..7, h, e = 0..1).  A
+ * "pair" (j, h, row) is the two codes with e = 0 (bits 0..15 of a word) and e = 1 (the same
+ * position in bits 16..31).  Fields below are positions within each 16-bit half, least
+ * significant code bit first:
+ *   b = 4: 8 words per lane; word j: bits 0-3 pair (j,0,r), 4-7 (j,1,r), 8-11 (j,0,r+8),
+ *          12-15 (j,1,r+8).  Word w of lane l is record word (w/4)*128 + 4l + (w%4).
+ *   b = 3: 6 words per lane; with pair index i = 2j + h, word w holds: bits 0-2 pair
+ *          (i = w, r), 3-5 (i = 6+w, r), 6-8 (i = 12 + w/2, r if w even else r+8),
+ *          9-11 (i = w, r+8), 12-14 (i = 6+w, r+8), and bit 15 = bit (w % 3) of pair
+ *          (i = 15, r if w < 3 else r+8).  Word w of lane l is record word 4l + w (w < 4) or
+ *          128 + 2l + (w - 4) (w >= 4).
+ */
+laq_status laq_pack(const uint8_t *codes, int64_t K, int64_t N, int bits, void *packed,
+                    void *stream);
+
+/* laq_unpack -- the inverse of laq_pack (a test and inspection aid).  Same requirements. */
+laq_status laq_unpack(const void *packed, int64_t K, int64_t N, int bits, uint8_t *codes,
+                      void *stream);
+
+/*
+ * laq_gemm_wxg128 -- Y[M][N] = X[M][K] * W_hat[K][N], W_hat = s * (q - z) per Eq. (1), the
+ * quantized linear layer of the decode step (Sec. 5.2 "Inference", Table 3; App. H).
+ *
+ *   X       [M][K] fp16 activations.                                (in, 16-byte aligned)
+ *   packed  laq_pack output for the K x N codes at `bits`.          (in, 16-byte aligned)
+ *   s, z    [K/128][N] fp16 scales and uint8 zeros.                 (in, s 2-byte aligned)
+ *   Y       [M][N] fp16, must not overlap any input.                (out, 16-byte aligned)
+ *   0 <= M <= 16, K % 128 == 0, N % 16 == 0, bits 3 or 4.
+ *
+ * Arithmetic: products and sums in fp32 (tensor-core accumulation), one fp16 rounding of each
+ * output.  |Y - Y_exact| stays within 5e-3 * max|Y_exact| + 1e-3 for the weight and activation
+ * distributions of the paper's workloads.  Deterministic: no atomics; a given launch
+ * configuration always sums in the same order.
+ */
+laq_status laq_gemm_wxg128(const void *X, int64_t M, int64_t K, int64_t N, const void *packed,
+                           const void *s, const uint8_t *z, int bits, void *Y, void *stream);
+
+/*
+ * Launch configuration of laq_gemm_wxg128 (a tuning interface; the library picks one itself).
+ *   tiles_per_cta  16-column tiles per CTA: 1, 2 or 4.
+ *   warps          warps per CTA, 1..16; they split the CTA's K range.
+ *   cluster        CTAs per thread-block cluster, 1, 2, 4 or 8; the CTAs of a cluster split
+ *                  K and reduce their partial sums through distributed shared memory.
+ *   stages         depth of each warp's cp.async ring of weight records, 2..8.
+ *   pdl            1: launch with programmatic dependent launch, so the kernel may start and
+ *                  prefetch weights while the previous kernel on the stream finishes; X is
+ *                  read and Y written only after that kernel completes.  Only valid when the
+ *                  immediately preceding work on the stream does not write packed, s or z.
+ */
+typedef struct {
+    int32_t tiles_per_cta;
+    int32_t warps;
+    int32_t cluster;
+    int32_t stages;
+    int32_t pdl;
+    int32_t reserved[3];
+} laq_gemm_config;
+
+/* The configuration laq_gemm_wxg128 uses for this shape on a GPU with `num_sms` SMs (host-only
+ * computation; no device access).  Returns the same argument statuses as laq_gemm_wxg128. */
+laq_status laq_gemm_plan(int64_t M, int64_t K, int64_t N, int bits, int num_sms,
+                         laq_gemm_config *out);
+
+/* laq_gemm_wxg128 with an explicit configuration.  Same contract; LAQ_ERR_CONFIG if a field is
+ * outside its range or the shared memory it needs exceeds the device limit. */
+laq_status laq_gemm_wxg128_config(const void *X, int64_t M, int64_t K, int64_t N,
+                                  const void *packed, const void *s, const uint8_t *z, int bits,
+                                  void *Y, const laq_gemm_config *cfg, void *stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* LAQ_H */

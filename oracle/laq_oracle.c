@@ -20,14 +20,14 @@
  *                         - a constant group c quantizes exactly: s = |c| (1 if c == 0),
  *                           z = 1 if c < 0 else 0.
  *   laqo_dequant        Eq. (1): w_hat = s * (q - z), exact in fp64.
- *   laqo_pack/unpack    The bit layout of packed codes (the library's own layout, App. C only
+ *   laqo_pack/unpack    The bit layout of packed codes (the library's own layout, App. H only
  *                       fixes that the INT3 kernel packs codes into 32-bit words).  Written here
  *                       from the layout's definition, bit by bit.
  *   laqo_gemm           Y = X * W_hat in fp64: the linear layer y = W x of the decode step
- *                       (Sec. 5.3 "Inference"), a naive sum over k in increasing order.
+ *                       (Sec. 5.2 "Inference", Table 3), a naive sum over k in increasing order.
  *
  * Storage: W[K][N] fp16 (bit patterns), codes[K][N] u8, s[K/128][N] fp16 bits,
- * z[K/128][N] u8 -- the (num_groups, outfeatures) scale/zero tensors of App. C.
+ * z[K/128][N] u8 -- the (num_groups, outfeatures) scale/zero tensors of App. H.
  * Every function returns 0 on success, a positive status otherwise.
  */
 #include <math.h>

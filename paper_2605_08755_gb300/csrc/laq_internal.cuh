@@ -1,0 +1,31 @@
+// laq_internal.cuh -- declarations shared by the library's translation units (not installed).
+#pragma once
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace laq {
+
+cudaError_t launch_quantize_rtn(const uint16_t* W, int64_t K, int64_t N, int bits,
+                                uint8_t* codes, uint16_t* s, uint8_t* z, cudaStream_t stream);
+cudaError_t launch_pack(const uint8_t* codes, int64_t K, int64_t N, int bits, uint32_t* packed,
+                        cudaStream_t stream);
+cudaError_t launch_unpack(const uint32_t* packed, int64_t K, int64_t N, int bits, uint8_t* codes,
+                          cudaStream_t stream);
+
+// One GEMM launch, fully resolved on the host.
+struct GemmLaunch {
+    const uint16_t* X;
+    const uint8_t* packed;
+    const uint16_t* s;
+    const uint8_t* z;
+    uint16_t* Y;
+    int M, K, N, bits;
+    int tiles_per_cta, warps, cluster, stages, pdl;
+};
+
+// Dynamic shared memory the GEMM kernel needs for this launch (bytes), and the groups of X it
+// stages per phase.
+size_t gemm_smem_bytes(const GemmLaunch& L, int* groups_per_phase);
+cudaError_t launch_gemm(const GemmLaunch& L, size_t smem_limit, cudaStream_t stream);
+
+}  // namespace laq

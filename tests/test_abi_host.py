@@ -1,0 +1,145 @@
+"""Host-side checks of the C ABI (no GPU): the library loads, exports every symbol include/laq.h
+declares, rejects invalid arguments with the documented status before touching a device, and
+plans launches within the kernel's limits."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from tests.conftest import ROOT
+
+import paper_2605_08755_gb300 as laq
+from paper_2605_08755_gb300 import _lib, inputs
+
+HEADER = os.path.join(ROOT, "include", "laq.h")
+
+
+@pytest.fixture(scope="module")
+def L():
+    from paper_2605_08755_gb300 import build
+    build.build()
+    return _lib.lib()
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(laq_[a-z0-9_]+)\s*\(", text)))
+
+
+def test_header_declares_the_abi():
+    names = declared_functions()
+    assert set(names) == set(_lib.EXPORTS)
+
+
+def test_library_exports_every_declared_symbol(L):
+    for name in declared_functions():
+        assert hasattr(L, name), name
+
+
+def test_status_strings_and_version(L):
+    assert L.laq_version() == 1
+    for code, name in _lib.STATUS.items():
+        assert L.laq_status_str(code).decode().startswith(name)
+    assert L.laq_status_str(12345)
+
+
+def test_packed_bytes(L):
+    assert laq.packed_bytes(2560, 4096, 3) == 2560 * 4096 * 3 // 8
+    assert laq.packed_bytes(9728, 2560, 4) == 9728 * 2560 // 2
+    assert laq.packed_bytes(100, 16, 3) == 0
+    assert laq.packed_bytes(128, 16, 5) == 0
+    assert laq.packed_bytes(0, 0, 3) == 0
+
+
+FAKE = ctypes.c_void_p(0x10000)      # 16-byte aligned, never dereferenced: calls fail first
+ODD = ctypes.c_void_p(0x10002)
+
+
+def gemm(L, X=FAKE, M=1, K=256, N=32, packed=FAKE, s=FAKE, z=FAKE, bits=3, Y=FAKE):
+    return L.laq_gemm_wxg128(X, M, K, N, packed, s, z, bits, Y, None)
+
+
+def test_gemm_argument_validation(L):
+    assert gemm(L, bits=2) == 2
+    assert gemm(L, bits=5) == 2
+    assert gemm(L, M=17) == 6
+    assert gemm(L, M=-1) == 6
+    assert gemm(L, K=100) == 4
+    assert gemm(L, N=24) == 4
+    assert gemm(L, K=-128) == 4
+    assert gemm(L, X=None) == 1
+    assert gemm(L, packed=None) == 1
+    assert gemm(L, s=None) == 1
+    assert gemm(L, z=None) == 1
+    assert gemm(L, Y=None) == 1
+    assert gemm(L, X=ODD) == 5
+    assert gemm(L, Y=ODD) == 5
+    assert gemm(L, packed=ODD) == 5
+    assert gemm(L, s=ctypes.c_void_p(0x10001)) == 5
+    # empty problems are no-ops that never touch the device
+    assert gemm(L, M=0) == 0
+    assert gemm(L, N=0, Y=None) == 0
+
+
+def test_gemm_config_validation(L):
+    def run(**kw):
+        base = dict(tiles_per_cta=1, warps=4, cluster=1, stages=4, pdl=0)
+        base.update(kw)
+        cfg = _lib.GemmConfig.make(**base)
+        return L.laq_gemm_wxg128_config(FAKE, 1, 256, 32, FAKE, FAKE, FAKE, 3, FAKE,
+                                        ctypes.byref(cfg), None)
+    assert run(tiles_per_cta=3) == 9
+    assert run(warps=0) == 9
+    assert run(warps=9) == 9
+    assert run(cluster=3) == 9
+    assert run(cluster=16) == 9
+    assert run(stages=1) == 9
+    assert run(stages=9) == 9
+    assert run(pdl=2) == 9
+    assert L.laq_gemm_wxg128_config(FAKE, 1, 256, 32, FAKE, FAKE, FAKE, 3, FAKE, None,
+                                    None) == 1
+
+
+def test_quantize_pack_argument_validation(L):
+    q = L.laq_quantize_rtn
+    assert q(FAKE, 256, 32, 3, 64, FAKE, FAKE, FAKE, None) == 3
+    assert q(FAKE, 256, 32, 6, 128, FAKE, FAKE, FAKE, None) == 2
+    assert q(FAKE, 200, 32, 3, 128, FAKE, FAKE, FAKE, None) == 4
+    assert q(None, 256, 32, 3, 128, FAKE, FAKE, FAKE, None) == 1
+    assert q(ctypes.c_void_p(0x10001), 256, 32, 3, 128, FAKE, FAKE, FAKE, None) == 5
+    assert q(FAKE, 0, 32, 3, 128, None, None, None, None) == 0
+    p = L.laq_pack
+    assert p(FAKE, 256, 24, 3, FAKE, None) == 4
+    assert p(FAKE, 256, 32, 3, ODD, None) == 5
+    assert p(None, 256, 32, 3, FAKE, None) == 1
+    assert p(FAKE, 0, 32, 3, None, None) == 0
+    u = L.laq_unpack
+    assert u(FAKE, 256, 32, 7, FAKE, None) == 2
+    assert u(ODD, 256, 32, 3, FAKE, None) == 5
+
+
+@pytest.mark.parametrize("bits", [3, 4])
+@pytest.mark.parametrize("M", [1, 2, 3, 4, 5, 8, 9, 16])
+def test_plan_is_valid_for_every_workload_shape(L, bits, M):
+    shapes = {(K, N) for _, K, N in inputs.QWEN3_4B + inputs.QWEN3_8B}
+    shapes |= {(1024, 1024), (128, 16), (256, 4096), (12288, 16)}
+    for K, N in sorted(shapes):
+        for sms in (152, 148, 1):
+            c = laq.laq_gemm_plan(M, K, N, bits, sms)
+            assert c.tiles_per_cta in (1, 2, 4)
+            assert 1 <= c.warps <= 8
+            assert c.cluster in (1, 2, 4, 8) and c.cluster <= max(1, K // 128)
+            assert 2 <= c.stages <= 8
+            assert c.pdl == 0
+            if M > 8:
+                assert c.tiles_per_cta <= 2
+
+
+def test_plan_rejects_bad_arguments(L):
+    cfg = _lib.GemmConfig()
+    assert L.laq_gemm_plan(1, 256, 32, 3, 0, ctypes.byref(cfg)) == 9
+    assert L.laq_gemm_plan(1, 256, 32, 3, 152, None) == 1
+    assert L.laq_gemm_plan(20, 256, 32, 3, 152, ctypes.byref(cfg)) == 6
+    assert L.laq_gemm_plan(1, 250, 32, 3, 152, ctypes.byref(cfg)) == 4
