@@ -303,6 +303,48 @@ def fp16_context(a, dev, steps=50):
     return us, nbytes
 
 
+def time_graph(graph, stream, reps, dev):
+    """Device time (ms) of ``reps`` back-to-back replays, CUDA events on ``stream``."""
+    import torch
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        graph.replay()
+        e0.record(stream)
+        for _ in range(reps):
+            graph.replay()
+        e1.record(stream)
+    torch.cuda.synchronize(dev)
+    return e0.elapsed_time(e1) / reps
+
+
+def kernel_breakdown(wp, stream, dev, reps=200):
+    """Per GEMM kernel instance (bits, M class, tiles per CTA): a CUDA graph of all of its
+    launches of one step, in pass order, timed on the stream they run on; returns rows of
+    (instance, launches, algorithmic bytes per step, us per step)."""
+    import torch
+    from paper_2605_08755_gb300 import _lib
+    mp = 1 if wp.M <= 1 else 2 if wp.M <= 2 else 4 if wp.M <= 4 else 8 if wp.M <= 8 else 16
+    groups = {}
+    for i, (*_, q) in enumerate(wp.linears):
+        key = f"gemm_kernel<{q.bits}, {mp}, {wp.configs[i].tiles_per_cta}>"
+        groups.setdefault(key, []).append(i)
+    rows = []
+    for key, idxs in groups.items():
+        def run(s=None):
+            for i in idxs:
+                q = wp.linears[i][3]
+                _lib.laq_gemm_wxg128(wp.X[i], q.packed, q.s, q.z, q.bits, Y=wp.Y[i],
+                                     config=wp.configs[i], stream=s)
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            run(stream)
+        ms = time_graph(g, stream, reps, dev)
+        nbytes = sum(wp.linears[i][3].bytes_per_call(wp.M) for i in idxs)
+        rows.append((key, len(idxs), nbytes, ms * 1e3))
+        del g
+    return rows
+
+
 def run_laq(a, world, rank, local):
     import torch
 
@@ -313,31 +355,22 @@ def run_laq(a, world, rank, local):
     dev = torch.device("cuda", local)
     torch.cuda.set_device(dev)
     peak, peak_kind = load_peaks()
+    outliers = a.model == "qwen3-8b"
 
     t0 = time.perf_counter()
-    wp = WeightPass(model=a.model, bits=a.bits, M=a.M, layers=a.layers,
-                    outliers=(a.model == "qwen3-8b"), device=dev)
+    wp = WeightPass(model=a.model, bits=a.bits, M=a.M, layers=a.layers, outliers=outliers,
+                    device=dev)
+    torch.cuda.synchronize(dev)
     prep_ms = (time.perf_counter() - t0) * 1e3
     bytes_step = wp.bytes_per_pass()
 
-    # Plain graph for the timed region; a second capture of the same launches carries an
-    # external timing event before every launch and after the last, so each launch's device
-    # time is measured on the stream it runs on, in replays right after the timed region.
     stream = torch.cuda.Stream(dev)
     graph = wp.capture(stream=stream)
-    try:
-        events = [torch.cuda.Event(enable_timing=True, external=True)
-                  for _ in range(wp.launches + 1)]
-        igraph = wp.capture(stream=stream, events=events)
-    except TypeError:
-        events, igraph = None, None
-
     with torch.cuda.stream(stream):
         for _ in range(a.warmup):
             graph.replay()
     torch.cuda.synchronize(dev)
 
-    step_ms = []
     starts = [torch.cuda.Event(enable_timing=True) for _ in range(a.steps)]
     ends = [torch.cuda.Event(enable_timing=True) for _ in range(a.steps)]
     with ClockSampler(local) as clk:
@@ -351,40 +384,21 @@ def run_laq(a, world, rank, local):
         torch.cuda.synchronize(dev)
         barrier(world)
     clocks = clk.summary()
-    for i in range(a.steps):
-        step_ms.append(starts[i].elapsed_time(ends[i]))
-    total_ms = starts[0].elapsed_time(ends[-1])
-    total_ms = max_over_ranks(world, total_ms, dev)
+    step_ms = sorted(starts[i].elapsed_time(ends[i]) for i in range(a.steps))
+    total_ms = max_over_ranks(world, starts[0].elapsed_time(ends[-1]), dev)
     ms_per_step = total_ms / a.steps
     value = sum_over_ranks(world, bytes_step * a.steps, dev) / (total_ms * 1e-3) / 1e9
 
-    per_launch = [0.0] * wp.launches
-    reps = 20
-    if igraph is not None:
-        with torch.cuda.stream(stream):
-            for _ in range(reps):
-                igraph.replay()
-                torch.cuda.synchronize(dev)
-                for j in range(wp.launches):
-                    per_launch[j] += events[j].elapsed_time(events[j + 1]) / reps
-        kernel_ms = sum(per_launch)
-        ievent_ms = events[0].elapsed_time(events[-1])
-    else:
-        kernel_ms, ievent_ms = ms_per_step, None
-    kernel_gbs = bytes_step / (kernel_ms * 1e-3) / 1e9
-    by_name = {}
-    for (layer, pi, name, q), t in zip(wp.linears, per_launch):
-        d = by_name.setdefault(name, [0.0, 0])
-        d[0] += t * 1e3
-        d[1] += q.bytes_per_call(a.M)
-    per_proj = {k: {"us_per_launch": v[0] / a.layers,
-                    "gbs": v[1] / (v[0] * 1e-6) / 1e9 if v[0] else None}
-                for k, v in by_name.items()}
+    # Per-instance launch times (the roofline of the dominant kernel).
+    rows = kernel_breakdown(wp, stream, dev)
+    dom = max(rows, key=lambda r: r[3])
+    kernel_gbs = dom[2] / (dom[3] * 1e-6) / 1e9
 
-    # end to end through the public API with host buffers
-    xh = torch.empty_like(wp.Xbuf, device="cpu").pin_memory()
+    # End to end through the public API with host buffers: every step copies all X from
+    # pinned host memory, replays the 252 calls and copies all Y back.
+    xh = torch.empty(wp.Xbuf.shape, dtype=wp.Xbuf.dtype, pin_memory=True)
     xh.copy_(wp.Xbuf)
-    yh = torch.empty_like(wp.Ybuf, device="cpu").pin_memory()
+    yh = torch.empty(wp.Ybuf.shape, dtype=wp.Ybuf.dtype, pin_memory=True)
     e2e_steps = max(10, min(a.steps, 400))
     torch.cuda.synchronize(dev)
     e_a, e_b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -398,6 +412,20 @@ def run_laq(a, world, rank, local):
     torch.cuda.synchronize(dev)
     e2e_ms = max_over_ranks(world, e_a.elapsed_time(e_b), dev) / e2e_steps
     e2e_gbs = sum_over_ranks(world, bytes_step, dev) / (e2e_ms * 1e-3) / 1e9
+    h2d, d2h = wp.Xbuf.numel() * 2, wp.Ybuf.numel() * 2
+    launches = wp.launches
+    del graph, wp
+    torch.cuda.empty_cache()
+
+    # The same pass with q|k|v and gate|up fused (4 launches per layer), reported beside it.
+    wpf = WeightPass(model=a.model, bits=a.bits, M=a.M, layers=a.layers, outliers=outliers,
+                     device=dev, fuse=True)
+    gf = wpf.capture(stream=stream)
+    fused_ms = time_graph(gf, stream, max(20, min(a.steps, 500)), dev)
+    fused_bytes = wpf.bytes_per_pass()
+    fused_launches = wpf.launches
+    del gf, wpf
+    torch.cuda.empty_cache()
 
     fp16_us = None
     if not a.no_fp16 and rank == 0:
@@ -415,35 +443,36 @@ def run_laq(a, world, rank, local):
 
     if rank != 0:
         return
+    pct = lambda q: step_ms[min(len(step_ms) - 1, int(q * (len(step_ms) - 1)))]
     line = {
         "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": world, "steps": a.steps,
         "warmup": a.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None, "dtype": "u3+f16 (fp32 accumulate)"
-        if a.bits == 3 else "u4+f16 (fp32 accumulate)", "data": "synthetic",
+        "scaling": "weak", "vs_baseline": None,
+        "dtype": f"u{a.bits} codes + fp16 (fp32 accumulate)", "data": "synthetic",
         "config": {"workload": workload_name(a), "model": a.model, "bits": a.bits, "M": a.M,
-                   "launches_per_step": wp.launches, "bytes_per_step": bytes_step,
+                   "launches_per_step": launches, "bytes_per_step": bytes_step,
                    "us_per_step": ms_per_step * 1e3,
                    "pct_of_peak": 100.0 * value / world / peak,
                    "peak_gbs": peak, "peak_kind": peak_kind,
                    "l2": "inputs larger than L2 (packed weights per step >> 129 MB)",
-                   "step_ms_p10_p50_p90": [sorted(step_ms)[int(0.1 * (len(step_ms) - 1))],
-                                           statistics.median(step_ms),
-                                           sorted(step_ms)[int(0.9 * (len(step_ms) - 1))]],
+                   "step_ms_p10_p50_p90": [pct(0.1), pct(0.5), pct(0.9)],
                    "prep_ms": prep_ms,
+                   "fused_qkv_gateup": {"launches_per_step": fused_launches,
+                                        "us_per_step": fused_ms * 1e3,
+                                        "gbs": fused_bytes / (fused_ms * 1e-3) / 1e9},
                    "fp16_torch_matmul_us_per_step": fp16_us,
                    "speedup_vs_fp16_torch": (fp16_us / (ms_per_step * 1e3)) if fp16_us else None,
                    "parallelism": f"replicas x{world}"},
         "roofline": {"bound": "hbm", "achieved": kernel_gbs, "peak": peak, "unit": "GB/s",
-                     "frac": kernel_gbs / peak, "traffic": None,
-                     "kernel": "gemm_kernel, all launches of one step: algorithmic bytes / "
-                               "sum of per-launch event times",
-                     "peak_kind": peak_kind, "kernel_us_per_step": kernel_ms * 1e3,
-                     "instrumented_step_us": None if ievent_ms is None else ievent_ms * 1e3,
-                     "per_projection": per_proj},
+                     "frac": kernel_gbs / peak, "traffic": None, "kernel": dom[0],
+                     "launches_per_step": dom[1], "us_per_launch": dom[3] / dom[1],
+                     "bytes_per_launch": dom[2] / dom[1], "peak_kind": peak_kind,
+                     "instances": [{"kernel": k, "launches": n, "us_per_step": us,
+                                    "gbs": nb / (us * 1e-6) / 1e9} for k, n, nb, us in rows]},
         "cpu_baseline": cpu,
-        "e2e": {"value": e2e_gbs, "unit": "GB/s", "h2d_bytes_per_step": wp.Xbuf.numel() * 2,
-                "d2h_bytes_per_step": wp.Ybuf.numel() * 2, "us_per_step": e2e_ms * 1e3},
-        "gpu_launches": wp.launches * a.steps,
+        "e2e": {"value": e2e_gbs, "unit": "GB/s", "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h, "us_per_step": e2e_ms * 1e3},
+        "gpu_launches": launches * a.steps,
         "clocks": clocks,
     }
     print(json.dumps(line), flush=True)

@@ -92,17 +92,17 @@ laq_status laq_quantize_rtn(const void *W, int64_t K, int64_t N, int bits, int g
  * columns n = 16t..16t+15 and rows k = 128g..128g+127 and is stored at record index
  * t * (K/128) + g (tile-major).  A record is 32 * bits 32-bit words (1024 bytes at b = 4, 768
  * at b = 3) and is split among 32 lanes; lane l (c = l % 4, r = l / 4) owns the 64 codes at
- * columns r and r + 8 of the tile and rows k = 16j + 8h + 2c + e (j = 0..7, h, e = 0..1).  A
- * "pair" (j, h, row) is the two codes with e = 0 (bits 0..15 of a word) and e = 1 (the same
- * position in bits 16..31).  Fields below are positions within each 16-bit half, least
- * significant code bit first:
+ * columns r and r + 8 of the tile and rows k = 128g + 32c + 4j + 2h + e (j = 0..7,
+ * h, e = 0..1), so a lane's rows are 32 consecutive rows of the group.  A "pair" (j, h, row) is
+ * the two codes with e = 0 (bits 0..15 of a word) and e = 1 (the same position in bits
+ * 16..31).  Fields below are positions within each 16-bit half, least significant code bit
+ * first:
  *   b = 4: 8 words per lane; word j: bits 0-3 pair (j,0,r), 4-7 (j,1,r), 8-11 (j,0,r+8),
  *          12-15 (j,1,r+8).  Word w of lane l is record word (w/4)*128 + 4l + (w%4).
- *   b = 3: 6 words per lane; with pair index i = 2j + h, word w holds: bits 0-2 pair
- *          (i = w, r), 3-5 (i = 6+w, r), 6-8 (i = 12 + w/2, r if w even else r+8),
- *          9-11 (i = w, r+8), 12-14 (i = 6+w, r+8), and bit 15 = bit (w % 3) of pair
- *          (i = 15, r if w < 3 else r+8).  Word w of lane l is record word 4l + w (w < 4) or
- *          128 + 2l + (w - 4) (w >= 4).
+ *   b = 3: 6 words per lane; with pair index i = 2j + h, word w holds: bit 0 = bit (w % 3)
+ *          of pair (i = 15, r if w < 3 else r+8), bits 1-3 pair (i = w, r), 4-6 (i = 6+w, r),
+ *          7-9 (i = 12 + w/2, r if w even else r+8), 10-12 (i = w, r+8), 13-15 (i = 6+w, r+8).
+ *          Word w of lane l is record word 4l + w (w < 4) or 128 + 2l + (w - 4) (w >= 4).
  */
 laq_status laq_pack(const uint8_t *codes, int64_t K, int64_t N, int bits, void *packed,
                     void *stream);
@@ -117,7 +117,7 @@ laq_status laq_unpack(const void *packed, int64_t K, int64_t N, int bits, uint8_
  *
  *   X       [M][K] fp16 activations.                                (in, 16-byte aligned)
  *   packed  laq_pack output for the K x N codes at `bits`.          (in, 16-byte aligned)
- *   s, z    [K/128][N] fp16 scales and uint8 zeros.                 (in, s 2-byte aligned)
+ *   s, z    [K/128][N] fp16 scales and uint8 zeros.                 (in, 16-byte aligned)
  *   Y       [M][N] fp16, must not overlap any input.                (out, 16-byte aligned)
  *   0 <= M <= 16, K % 128 == 0, N % 16 == 0, bits 3 or 4.
  *
@@ -132,10 +132,12 @@ laq_status laq_gemm_wxg128(const void *X, int64_t M, int64_t K, int64_t N, const
 /*
  * Launch configuration of laq_gemm_wxg128 (a tuning interface; the library picks one itself).
  *   tiles_per_cta  16-column tiles per CTA: 1, 2 or 4.
- *   warps          warps per CTA, 1..16; they split the CTA's K range.
+ *   warps          warps per CTA, 1..8, a multiple of tiles_per_cta; each tile gets
+ *                  warps / tiles_per_cta warps, which split the CTA's K range.
  *   cluster        CTAs per thread-block cluster, 1, 2, 4 or 8; the CTAs of a cluster split
  *                  K and reduce their partial sums through distributed shared memory.
- *   stages         depth of each warp's cp.async ring of weight records, 2..8.
+ *   stages         depth of each warp's cp.async ring of weight records, 2..16; with
+ *                  stages > the warp's record count the whole slice is copied up front.
  *   pdl            1: launch with programmatic dependent launch, so the kernel may start and
  *                  prefetch weights while the previous kernel on the stream finishes; X is
  *                  read and Y written only after that kernel completes.  Only valid when the

@@ -181,7 +181,7 @@ int laqo_gemm_columns(const uint16_t *X, int64_t M, int64_t K, int64_t N, const 
  * tile).  Record (t, g) covers columns n = 16t .. 16t+15 and rows k = 128g .. 128g+127; records
  * are stored tile-major: record index t * (K/128) + g.  A record holds 32 lanes; lane l has
  * c = l % 4 and r = l / 4 and owns the 64 codes at columns r and r + 8 of the tile and rows
- *     k = 16j + 8h + 2c + e    (j = 0..7, h = 0..1, e = 0..1).
+ *     k = 32c + 4j + 2h + e    (j = 0..7, h = 0..1, e = 0..1) of the group.
  * A "pair" (j, h, row) is the two codes e = 0 (bits 0..15 of a word) and e = 1 (bits 16..31,
  * same position + 16).  Within each 16-bit half:
  *
@@ -189,10 +189,10 @@ int laqo_gemm_columns(const uint16_t *X, int64_t M, int64_t K, int64_t N, const 
  *        row r), 8-11: (j, h=0, row r+8), 12-15: (j, h=1, row r+8).  Word w of lane l sits at
  *        word offset (w / 4) * 128 + 4 l + (w % 4) of the 256-word record.
  * b = 3: 6 words per lane.  Let pair index i = 2j + h (0..15).  In word w, half-bits
- *        0-2: pair i = w, row r;      3-5: pair i = 6 + w, row r;
- *        6-8: pair i = 12 + w/2, row r if w is even else r + 8;
- *        9-11: pair i = w, row r+8;   12-14: pair i = 6 + w, row r+8;
- *        15: bit (w % 3) of pair i = 15, row r for w < 3 else r + 8.
+ *        0: bit (w % 3) of pair i = 15, row r for w < 3 else r + 8;
+ *        1-3: pair i = w, row r;      4-6: pair i = 6 + w, row r;
+ *        7-9: pair i = 12 + w/2, row r if w is even else r + 8;
+ *        10-12: pair i = w, row r+8;  13-15: pair i = 6 + w, row r+8.
  *        Word w of lane l sits at word offset 4 l + w (w < 4) or 128 + 2 l + (w - 4) (w >= 4)
  *        of the 192-word record.
  * Bit 0 of a field is the code's least significant bit.  Words are little-endian uint32.
@@ -213,16 +213,16 @@ static void layout_bit(int bits, int l, int w, int b, int *kk, int *nn, int *cb)
         row = f / 2;
     } else {
         int i;
-        if (hb < 3)       { i = w;          row = 0;       *cb = hb; }
-        else if (hb < 6)  { i = 6 + w;      row = 0;       *cb = hb - 3; }
-        else if (hb < 9)  { i = 12 + w / 2; row = w % 2;   *cb = hb - 6; }
-        else if (hb < 12) { i = w;          row = 1;       *cb = hb - 9; }
-        else if (hb < 15) { i = 6 + w;      row = 1;       *cb = hb - 12; }
-        else              { i = 15;         row = w >= 3;  *cb = w % 3; }
+        if (hb == 0)      { i = 15;         row = w >= 3;  *cb = w % 3; }
+        else if (hb < 4)  { i = w;          row = 0;       *cb = hb - 1; }
+        else if (hb < 7)  { i = 6 + w;      row = 0;       *cb = hb - 4; }
+        else if (hb < 10) { i = 12 + w / 2; row = w % 2;   *cb = hb - 7; }
+        else if (hb < 13) { i = w;          row = 1;       *cb = hb - 10; }
+        else              { i = 6 + w;      row = 1;       *cb = hb - 13; }
         j = i / 2;
         h = i % 2;
     }
-    *kk = 16 * j + 8 * h + 2 * c + e;
+    *kk = 32 * c + 4 * j + 2 * h + e;
     *nn = r + 8 * row;
 }
 

@@ -65,12 +65,12 @@ def _field_table(bits):
     """Arrays over (lane, word, bit) of the row-in-group kk, column-in-tile nn and code bit cb,
     and the word offset of (lane, word) in the record.
 
-    Lane l: c = l % 4, r = l / 4.  Pair (j, h, row) = codes at rows 16j + 8h + 2c + e (e = 0 in
-    bits 0..15, e = 1 in bits 16..31) of column r (row 0) or r + 8 (row 1).
+    Lane l: c = l % 4, r = l / 4.  Pair (j, h, row) = codes at rows 32c + 4j + 2h + e of the group
+    (e = 0 in bits 0..15, e = 1 in bits 16..31) of column r (row 0) or r + 8 (row 1).
       b = 4: word j; half-bit fields of 4 bits: (h=0,row0), (h=1,row0), (h=0,row1), (h=1,row1).
-      b = 3: pair i = 2j + h; fields of 3 bits at half-bits 0, 3, 6, 9, 12 carry pairs
-             (w,row0), (6+w,row0), (12+w//2,row w%2), (w,row1), (6+w,row1); half-bit 15 carries
-             bit w%3 of pair (15, row 0 if w < 3 else row 1).
+      b = 3: pair i = 2j + h; half-bit 0 carries bit w%3 of pair (15, row 0 if w < 3 else
+             row 1); fields of 3 bits at half-bits 1, 4, 7, 10, 13 carry pairs (w,row0),
+             (6+w,row0), (12+w//2,row w%2), (w,row1), (6+w,row1).
     """
     wpl = 8 if bits == 4 else 6
     L, Wd, B = np.meshgrid(np.arange(32), np.arange(wpl), np.arange(32), indexing="ij")
@@ -81,14 +81,15 @@ def _field_table(bits):
         cb = hb % 4
         j, h, row = Wd, f % 2, f // 2
     else:
-        field = np.minimum(hb // 3, 5)
-        i = np.select([field == 0, field == 1, field == 2, field == 3, field == 4],
-                      [Wd, 6 + Wd, 12 + Wd // 2, Wd, 6 + Wd], 15)
-        row = np.select([field == 0, field == 1, field == 2, field == 3, field == 4],
-                        [0 * Wd, 0 * Wd, Wd % 2, 0 * Wd + 1, 0 * Wd + 1], (Wd >= 3).astype(int))
-        cb = np.where(field < 5, hb - 3 * field, Wd % 3)
+        spare = hb == 0
+        field = np.where(spare, 0, (hb - 1) // 3)          # 0..4 for half-bits 1..15
+        i = np.select([spare, field == 0, field == 1, field == 2, field == 3],
+                      [15 + 0 * Wd, Wd, 6 + Wd, 12 + Wd // 2, Wd], 6 + Wd)
+        row = np.select([spare, field == 0, field == 1, field == 2, field == 3],
+                        [(Wd >= 3).astype(int), 0 * Wd, 0 * Wd, Wd % 2, 0 * Wd + 1], 0 * Wd + 1)
+        cb = np.where(spare, Wd % 3, hb - 1 - 3 * field)
         j, h = i // 2, i % 2
-    kk = 16 * j + 8 * h + 2 * c + e
+    kk = 32 * c + 4 * j + 2 * h + e
     nn = r + 8 * row
     lw_l, lw_w = np.meshgrid(np.arange(32), np.arange(wpl), indexing="ij")
     if bits == 4:

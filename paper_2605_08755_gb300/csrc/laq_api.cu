@@ -75,7 +75,8 @@ laq_status check_gemm_args(const void* X, int64_t M, int64_t K, int64_t N, const
     if (!aligned(Y, 16)) return LAQ_ERR_ALIGN;
     if (K == 0) return LAQ_OK;
     if (!X || !packed || !s || !z) return LAQ_ERR_NULL;
-    if (!aligned(X, 16) || !aligned(packed, 16) || !aligned(s, 2)) return LAQ_ERR_ALIGN;
+    if (!aligned(X, 16) || !aligned(packed, 16) || !aligned(s, 16) || !aligned(z, 16))
+        return LAQ_ERR_ALIGN;
     return LAQ_OK;
 }
 
@@ -84,68 +85,63 @@ laq_status check_config(const laq_gemm_config* c) {
     if (c->tiles_per_cta != 1 && c->tiles_per_cta != 2 && c->tiles_per_cta != 4)
         return LAQ_ERR_CONFIG;
     if (c->warps < 1 || c->warps > 8) return LAQ_ERR_CONFIG;
+    if (c->warps % c->tiles_per_cta) return LAQ_ERR_CONFIG;  // whole warps per tile
     if (c->cluster != 1 && c->cluster != 2 && c->cluster != 4 && c->cluster != 8)
         return LAQ_ERR_CONFIG;
-    if (c->stages < 2 || c->stages > 8) return LAQ_ERR_CONFIG;
+    if (c->stages < 2 || c->stages > 16) return LAQ_ERR_CONFIG;
     if (c->pdl != 0 && c->pdl != 1) return LAQ_ERR_CONFIG;
     return LAQ_OK;
 }
 
 int ceil_div(int64_t a, int64_t b) { return (int)((a + b - 1) / b); }
 
-// Launch-shape heuristic.  The kernel is HBM-bound; the plan aims for one wave of CTAs that
-// splits the records (16 columns x 128 rows of K) evenly over the SMs with enough copies in
-// flight per SM.  Estimated time in units of "records streamed by one SM":
-//   max(perfect balance, busiest SM's load at ~2.5x its fair-share rate) + per-wave latency,
-// plus a small cost for cluster reductions.
+// Launch-shape plan.  The kernel streams each 16-column x 128-row record once, so the plan is
+// about keeping HBM busy: (1) enough CTAs to occupy every SM -- the largest tiles-per-CTA and
+// the smallest cluster (K split) that still give at least one CTA per SM; (2) eight warps
+// (fewer when a CTA owns fewer than eight groups); (3) a cp.async ring deep enough that each
+// warp keeps all but one of its groups in flight (up to 7 records per tile), capped so the ring
+// stays within 96 KB and two CTAs can share an SM.
 void plan(int64_t M, int64_t K, int64_t N, int bits, int sms, laq_gemm_config* out) {
     const int64_t T = N / 16, G = K / kGroup;
     const int mp = M <= 1 ? 1 : M <= 2 ? 2 : M <= 4 ? 4 : M <= 8 ? 8 : 16;
-    double best = 1e300;
-    laq_gemm_config bestc = {1, 8, 1, 4, 0, {0, 0, 0}};
-    const int nts[3] = {1, 2, 4};
+    const int64_t rec = bits == 4 ? 1024 : 768;
+    const int nts[3] = {4, 2, 1};
     const int cls[4] = {1, 2, 4, 8};
-    const int wps[2] = {4, 8};
-    for (int a = 0; a < 3; ++a) {
-        const int nt = nts[a];
-        if (mp == 16 && nt == 4) continue;  // register pressure: two MMA column halves
-        for (int b = 0; b < 4; ++b) {
-            const int cl = cls[b];
-            if (cl > 1 && cl > G) continue;
-            for (int d = 0; d < 2; ++d) {
-                const int w = wps[d];
-                const int64_t ctas = (int64_t)ceil_div(T, nt) * cl;
-                const int64_t gc = (G + cl - 1) / cl;
-                const int64_t iters = (gc + w - 1) / w;
-                const double cta_rec = (double)nt * iters * w;
-                laq::GemmLaunch L = {};
-                L.M = (int)M; L.K = (int)K; L.N = (int)N; L.bits = bits;
-                L.tiles_per_cta = nt; L.warps = w; L.cluster = cl; L.stages = 4;
-                const size_t smem = laq::gemm_smem_bytes(L, nullptr);
-                int occ = (int)((228 * 1024) / (smem + 1024));
-                const int occ_thr = 16 / w;  // 2 CTAs of 8 warps per SM (launch bounds)
-                if (occ > occ_thr) occ = occ_thr;
-                if (occ < 1) continue;
-                const int64_t slots = (int64_t)sms * occ;
-                const int64_t busiest = (ctas + sms - 1) / sms;
-                const int64_t waves = (ctas + slots - 1) / slots;
-                const double t_bw = (double)T * G / sms;
-                const double t_sm = (double)busiest * cta_rec / 2.5;
-                double est = (t_bw > t_sm ? t_bw : t_sm) + 12.0 * waves;
-                if (cl > 1) est += 2.0;
-                if (ctas < sms) est += 0.5 * (double)(sms - ctas) / sms * t_bw;
-                if (est < best - 1e-9) {
-                    best = est;
-                    bestc.tiles_per_cta = nt;
-                    bestc.warps = w;
-                    bestc.cluster = cl;
-                    bestc.stages = 4;
-                    bestc.pdl = 0;
-                }
+    int best_nt = 1, best_cl = 1;
+    int64_t best_ctas = -1;
+    bool found = false;
+    for (int b = 0; b < 4 && !found; ++b) {
+        const int cl = cls[b];
+        if (cl > 1 && cl > G) break;
+        for (int a = 0; a < 3; ++a) {
+            const int nt = nts[a];
+            const int64_t ctas = (int64_t)ceil_div(T, nt) * cl;
+            if (ctas >= sms) {
+                best_nt = nt;
+                best_cl = cl;
+                found = true;
+                break;
+            }
+            if (ctas > best_ctas) {
+                best_ctas = ctas;
+                best_nt = nt;
+                best_cl = cl;
             }
         }
     }
-    *out = bestc;
+    const int64_t gc = (G + best_cl - 1) / best_cl;
+    const int64_t wt_max = 8 / best_nt;                        // warps per tile
+    const int64_t wt = gc < wt_max ? (gc < 1 ? 1 : gc) : wt_max;
+    const int w = (int)(wt * best_nt);
+    const int64_t iters = (gc + wt - 1) / wt;
+    int st = (int)(iters + 1 > 16 ? 16 : (iters + 1 < 2 ? 2 : iters + 1));
+    while (st > 2 && (int64_t)w * st * rec > 100 * 1024) --st;
+    out->tiles_per_cta = best_nt;
+    out->warps = w;
+    out->cluster = best_cl;
+    out->stages = st;
+    out->pdl = 0;
+    out->reserved[0] = out->reserved[1] = out->reserved[2] = 0;
 }
 
 laq_status run_gemm(const void* X, int64_t M, int64_t K, int64_t N, const void* packed,

@@ -8,14 +8,19 @@
 //    each of its NT tiles (768 B at b = 3, 1024 B at b = 4).  Every lane copies and later
 //    reads only its own 16 + 8 (b = 3) or 16 + 16 (b = 4) bytes, so the ring needs no barrier.
 //
-//  * Dequantization is folded into a tensor-core contraction.  A code q at bit position p of
-//    an fp16 mantissa becomes the exact fp16 value 1024 + q * 2^p with one LOP3 (two codes per
-//    32-bit register).  X is pre-scaled per row of K by 2^-p, so the m16n8k16 MMA (fp16 in, fp32
-//    accumulate) of these registers against x' = x * 2^-p yields, per group g and column n,
-//        D = sum_k (1024 + q 2^p) x 2^-p = 1024 * S'_g + sum_k q x,     S'_g = sum_k x'.
-//    The group epilogue applies Eq. (1):  y_n += s_gn * (D - 1024 S'_g - z_gn * S_g),
-//    S_g = sum_k x_k, which equals sum_k x_k * s_gn * (q - z_gn).  No per-weight subtract or
-//    multiply is needed; the unpack is ~0.7 integer ops per weight.
+//  * Dequantization is folded into a tensor-core contraction.  A code q at mantissa bit p of
+//    an fp16 whose exponent field is 25 - p has the exact value 2^(10-p) + q, so one LOP3
+//    (mask | exponent) turns two codes of a 32-bit word into A-fragment values c + q with a
+//    per-field offset c = 2^(10-p).  The m16n8k16 MMA (fp16 in, fp32 accumulate) of these
+//    against raw x gives, per group g and MMA column, D = sum_k c_k x_k + sum_k q_k x_k.  A
+//    second MMA per k16 step, whose A rows 0-7 hold c_k and rows 8-15 hold 1, gives
+//    P_g = sum_k c_k x_k and S_g = sum_k x_k in the same registers, so the group epilogue
+//    applies Eq. (1) directly:  y_n += s_gn * (D - P_g - z_gn * S_g)  (= sum_k x_k s (q - z)).
+//    The unpack costs about 0.7 integer ops per weight; nothing else touches a weight.
+//
+//  * Inside a record, lane c's rows are k = 32c + 4j + 2h + e, so its B fragments for the 8 k16
+//    steps are the 32 consecutive x values x[32c .. 32c+31] of the group: four 16-byte shared
+//    loads from a plain cp.async copy of X, with no pre-scaling or permutation pass.
 //
 //  * The MMA's 8 output columns are shared between batch rows and groups: with MP = M rounded
 //    up to a power of two (<= 8), column col = b * (8/MP) + (group index mod 8/MP).  At M = 1
@@ -38,11 +43,23 @@
 
 namespace cg = cooperative_groups;
 
+// Compile-time trace points (start, PDL wait done, X staged, K loop done, reduction done, end).
+// Empty in the library build; a tracing build defines LAQ_TRACE to timestamp them.
+#ifndef LAQ_TRACE
+#define LAQ_TRACE(point) \
+    do {                 \
+    } while (0)
+#endif
+#ifndef LAQ_TRACE_LOOP
+#define LAQ_TRACE_LOOP(point, iter) \
+    do {                            \
+    } while (0)
+#endif
+
 namespace laq {
 
 namespace {
 
-constexpr uint32_t kMagic = 0x64006400u;  // fp16 1024.0 in both halves
 constexpr int kMaxWarps = 8;
 
 template <int BITS>
@@ -58,16 +75,6 @@ struct RecordFmt<3> {
     static constexpr int kChunk1 = 8;
 };
 
-struct Params {
-    const uint16_t* X;
-    const uint8_t* packed;
-    const uint16_t* s;
-    const uint8_t* z;
-    uint16_t* Y;
-    int M, K, N, G, T;
-    int stages;  // cp.async ring depth per warp
-    int gpp;     // groups of X staged in shared memory per phase
-};
 
 __device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
     asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(dst), "l"(src) : "memory");
@@ -78,7 +85,7 @@ __device__ __forceinline__ void cp_async8(uint32_t dst, const void* src) {
 __device__ __forceinline__ void cp_async_commit() {
     asm volatile("cp.async.commit_group;\n" ::: "memory");
 }
-// Wait until at most n of this thread's committed cp.async groups are pending (n = 0..7).
+// Wait until at most n of this thread's committed cp.async groups are pending (n = 0..15).
 __device__ __forceinline__ void cp_async_wait(int n) {
     switch (n) {
         case 0: asm volatile("cp.async.wait_group 0;\n" ::: "memory"); break;
@@ -88,7 +95,15 @@ __device__ __forceinline__ void cp_async_wait(int n) {
         case 4: asm volatile("cp.async.wait_group 4;\n" ::: "memory"); break;
         case 5: asm volatile("cp.async.wait_group 5;\n" ::: "memory"); break;
         case 6: asm volatile("cp.async.wait_group 6;\n" ::: "memory"); break;
-        default: asm volatile("cp.async.wait_group 7;\n" ::: "memory"); break;
+        case 7: asm volatile("cp.async.wait_group 7;\n" ::: "memory"); break;
+        case 8: asm volatile("cp.async.wait_group 8;\n" ::: "memory"); break;
+        case 9: asm volatile("cp.async.wait_group 9;\n" ::: "memory"); break;
+        case 10: asm volatile("cp.async.wait_group 10;\n" ::: "memory"); break;
+        case 11: asm volatile("cp.async.wait_group 11;\n" ::: "memory"); break;
+        case 12: asm volatile("cp.async.wait_group 12;\n" ::: "memory"); break;
+        case 13: asm volatile("cp.async.wait_group 13;\n" ::: "memory"); break;
+        case 14: asm volatile("cp.async.wait_group 14;\n" ::: "memory"); break;
+        default: asm volatile("cp.async.wait_group 15;\n" ::: "memory"); break;
     }
 }
 
@@ -109,51 +124,81 @@ __device__ __forceinline__ void mma16816(float (&d)[4], uint32_t a0, uint32_t a1
         : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
 }
 
-// Pre-scale exponent p of pair index i = 2j + h (the bit position its codes occupy inside the
-// fp16 mantissa after extraction).  b = 4: h = 0 -> 0, h = 1 -> 4.  b = 3: fields at bits 0 / 3 /
-// 6 for i < 6 / < 12 / < 15, and the assembled spare-bit code at bit 4 for i = 15.
-template <int BITS>
-__device__ __forceinline__ int pair_shift(int i) {
-    if (BITS == 4) return (i & 1) ? 4 : 0;
-    return i < 6 ? 0 : (i < 12 ? 3 : (i < 15 ? 6 : 4));
+// Exponent fields that turn a code at mantissa bit p into the exact fp16 value 2^(10-p) + q:
+// exponent 25 - p, in both halves of a 32-bit register.
+constexpr uint32_t kExpP0 = 0x64006400u;  // p = 0: 1024 + q
+constexpr uint32_t kExpP1 = 0x60006000u;  // p = 1:  512 + q
+constexpr uint32_t kExpP4 = 0x54005400u;  // p = 4:   64 + q
+constexpr uint32_t kExpP7 = 0x48004800u;  // p = 7:    8 + q
+
+// The exponent fields a kernel instance ORs into its A fragments: b = 3 uses p = 1, 4, 7;
+// b = 4 uses p = 0, 4.  They arrive as kernel parameters so that they stay in registers and
+// each extraction is a single mask-and-or.
+struct Exps {
+    uint32_t e[3];
+};
+inline Exps exps_for(int bits) {
+    Exps x;
+    if (bits == 4) {
+        x.e[0] = kExpP0; x.e[1] = kExpP4; x.e[2] = 0u;
+    } else {
+        x.e[0] = kExpP1; x.e[1] = kExpP4; x.e[2] = kExpP7;
+    }
+    return x;
 }
 
+struct Params {
+    const uint16_t* X;
+    const uint8_t* packed;
+    const uint16_t* s;
+    const uint8_t* z;
+    uint16_t* Y;
+    int M, K, N, G, T;
+    int stages;  // cp.async ring depth per warp
+    int gpp;     // groups of X staged in shared memory per phase
+    int gc;      // most groups a CTA owns: ceil(G / cluster)
+    Exps exps;   // exponent fields of the A-fragment extraction
+};
+
 // Extract the A fragments of one record (one lane's words) into a[j][0..3] for the 8 k16 steps:
-// a0 = (row r, k 2c..2c+1), a1 = (row r+8, same k), a2 = (row r, k 2c+8..), a3 = (row r+8, ...).
+// a0 = (row r, pair (j,0)), a1 = (row r+8, pair (j,0)), a2 = (row r, pair (j,1)),
+// a3 = (row r+8, pair (j,1)); each register holds 2^(10-p) + q for its two codes.  Right shifts
+// are multiplications by powers of two (high word), left shifts plain multiplications, so they
+// run on the FMA pipe beside the mask-and-or operations.
 template <int BITS>
 __device__ __forceinline__ void extract(const uint32_t (&wd)[BITS == 4 ? 8 : 6],
-                                        uint32_t (&a)[8][4]) {
+                                        const Exps& x, uint32_t (&a)[8][4]) {
     if constexpr (BITS == 4) {
+        const uint32_t e0 = x.e[0], e4 = x.e[1];
 #pragma unroll
         for (int j = 0; j < 8; ++j) {
-            const uint32_t w = wd[j], t = w >> 8;
-            a[j][0] = (w & 0x000f000fu) | kMagic;  // pair (j, 0, r)      p = 0
-            a[j][2] = (w & 0x00f000f0u) | kMagic;  // pair (j, 1, r)      p = 4
-            a[j][1] = (t & 0x000f000fu) | kMagic;  // pair (j, 0, r + 8)  p = 0
-            a[j][3] = (t & 0x00f000f0u) | kMagic;  // pair (j, 1, r + 8)  p = 4
+            const uint32_t w = wd[j], t = __umulhi(w, 1u << 24);  // w >> 8
+            a[j][0] = (w & 0x000f000fu) | e0;  // pair (j, 0, r)      p = 0
+            a[j][2] = (w & 0x00f000f0u) | e4;  // pair (j, 1, r)      p = 4
+            a[j][1] = (t & 0x000f000fu) | e0;  // pair (j, 0, r + 8)  p = 0
+            a[j][3] = (t & 0x00f000f0u) | e4;  // pair (j, 1, r + 8)  p = 4
         }
     } else {
-        uint32_t u[6];
-#pragma unroll
-        for (int w = 0; w < 6; ++w) u[w] = wd[w] >> 9;
+        const uint32_t e1 = x.e[0], e4 = x.e[1], e7 = x.e[2];
         uint32_t rp[16][2];
 #pragma unroll
         for (int w = 0; w < 6; ++w) {
-            rp[w][0] = (wd[w] & 0x00070007u) | kMagic;      // bits 0-2    p = 0
-            rp[w][1] = (u[w] & 0x00070007u) | kMagic;       // bits 9-11   p = 0
-            rp[6 + w][0] = (wd[w] & 0x00380038u) | kMagic;  // bits 3-5    p = 3
-            rp[6 + w][1] = (u[w] & 0x00380038u) | kMagic;   // bits 12-14  p = 3
+            const uint32_t u = __umulhi(wd[w], 1u << 23);       // w >> 9
+            rp[w][0] = (wd[w] & 0x000e000eu) | e1;              // bits 1-3    p = 1
+            rp[6 + w][0] = (wd[w] & 0x00700070u) | e4;          // bits 4-6    p = 4
+            rp[w][1] = (u & 0x000e000eu) | e1;                  // bits 10-12  p = 1
+            rp[6 + w][1] = (u & 0x00700070u) | e4;              // bits 13-15  p = 4
         }
 #pragma unroll
         for (int q = 0; q < 3; ++q) {
-            rp[12 + q][0] = (wd[2 * q] & 0x01c001c0u) | kMagic;      // bits 6-8  p = 6
-            rp[12 + q][1] = (wd[2 * q + 1] & 0x01c001c0u) | kMagic;
+            rp[12 + q][0] = (wd[2 * q] & 0x03800380u) | e7;      // bits 7-9   p = 7
+            rp[12 + q][1] = (wd[2 * q + 1] & 0x03800380u) | e7;
         }
-        // pair 15: bit 15 of words 0,1,2 (row r) / 3,4,5 (row r+8) -> code bits 0,1,2 at p = 4
-        rp[15][0] = kMagic | ((u[0] >> 2) & 0x00100010u) | ((u[1] >> 1) & 0x00200020u) |
-                    (u[2] & 0x00400040u);
-        rp[15][1] = kMagic | ((u[3] >> 2) & 0x00100010u) | ((u[4] >> 1) & 0x00200020u) |
-                    (u[5] & 0x00400040u);
+        // pair 15: bit 0 of words 0,1,2 (row r) / 3,4,5 (row r+8) -> code bits 0,1,2 at p = 4
+        rp[15][0] = ((wd[0] * 16u) & 0x00100010u) | ((wd[1] * 32u) & 0x00200020u) |
+                    ((wd[2] * 64u) & 0x00400040u) | e4;
+        rp[15][1] = ((wd[3] * 16u) & 0x00100010u) | ((wd[4] * 32u) & 0x00200020u) |
+                    ((wd[5] * 64u) & 0x00400040u) | e4;
 #pragma unroll
         for (int j = 0; j < 8; ++j) {
             a[j][0] = rp[2 * j][0];
@@ -164,6 +209,13 @@ __device__ __forceinline__ void extract(const uint32_t (&wd)[BITS == 4 ? 8 : 6],
     }
 }
 
+// Offset c_k = 2^(10-p) of row k of a group (k = 32c + 4j + 2h + e, pair index i = (k % 32) / 2).
+template <int BITS>
+__device__ __forceinline__ float row_offset(int i) {
+    if (BITS == 4) return (i & 1) ? 64.f : 1024.f;
+    return i < 6 ? 512.f : (i < 12 ? 64.f : (i < 15 ? 8.f : 64.f));
+}
+
 template <int BITS, int MP, int NT>
 __global__ void __launch_bounds__(kMaxWarps * 32, 2) gemm_kernel(const Params p) {
     using F = RecordFmt<BITS>;
@@ -171,237 +223,274 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 2) gemm_kernel(const Params p)
     constexpr int GPA = MP >= 8 ? 1 : 8 / MP;  // groups sharing one accumulator (columns)
     constexpr int NH = MP > 8 ? 2 : 1;          // MMAs per step (batch rows 0-7, 8-15)
 
+    // Let the next kernel on the stream start launching now: it only prefetches constant
+    // weights before its own griddepcontrol.wait, which returns once this grid has finished.
+    pdl_launch_dependents();
+    LAQ_TRACE(0);
+
     extern __shared__ __align__(128) uint8_t smem[];
     const int W = blockDim.x >> 5;
+    const int WT = W / NT;                     // warps per tile
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int tile = warp % NT, team = warp / NT;
     const int c = lane & 3, R = lane >> 2;
     const int M = p.M, GP = p.gpp, S = p.stages;
     const int T0 = blockIdx.x * NT;
     const int ntv = min(NT, p.T - T0);
+    const bool tile_ok = tile < ntv;
     const int C = gridDim.y, rank = blockIdx.y;
     const int g0 = (int)((long long)p.G * rank / C);
     const int g1 = (int)((long long)p.G * (rank + 1) / C);
 
-    // shared memory: ring | xs | zero block | S | P | part
+    // shared memory: ring [W][S][record] | x [M][GP][128] fp16 | zero block (64 B)
+    //                | s [gc][NT][16] fp16 | z [gc][NT][16] u8 | S, P [M][GP] fp32
+    //                | epilogue table [M][GP][NT][16] float2 | part [NT][MP][16] fp32
     uint8_t* ring = smem;
-    uint4* xs = reinterpret_cast<uint4*>(smem + (size_t)W * S * NT * F::kBytes);
+    uint4* xs = reinterpret_cast<uint4*>(smem + (size_t)W * S * F::kBytes);
     uint4* zblk = xs + (size_t)M * GP * 16;
-    float* ssum = reinterpret_cast<float*>(zblk + 16);
+    uint16_t* s_sm = reinterpret_cast<uint16_t*>(zblk + 4);
+    uint8_t* z_sm = reinterpret_cast<uint8_t*>(s_sm + (size_t)p.gc * NT * 16);
+    float* ssum = reinterpret_cast<float*>(z_sm + (size_t)p.gc * NT * 16);
     float* psum = ssum + M * GP;
-    float* part = psum + M * GP;
-    if (threadIdx.x < 16) zblk[threadIdx.x] = make_uint4(0u, 0u, 0u, 0u);
+    float2* ab = reinterpret_cast<float2*>(psum + M * GP);
+    float* part = reinterpret_cast<float*>(ab + (size_t)M * GP * NT * 16);
+    if (threadIdx.x < 4) zblk[threadIdx.x] = make_uint4(0u, 0u, 0u, 0u);
 
     const uint32_t ring_s = (uint32_t)__cvta_generic_to_shared(ring) +
-                            (uint32_t)(warp * S * NT * F::kBytes);
-    const uint8_t* ring_w = ring + (size_t)warp * S * NT * F::kBytes;
+                            (uint32_t)(warp * S * F::kBytes);
+    const uint8_t* ring_w = ring + (size_t)warp * S * F::kBytes;
 
-    float yacc[NT][NH][4];
+    float yacc[NH][4];
 #pragma unroll
-    for (int t = 0; t < NT; ++t)
+    for (int h = 0; h < NH; ++h)
 #pragma unroll
-        for (int h = 0; h < NH; ++h)
-#pragma unroll
-            for (int v = 0; v < 4; ++v) yacc[t][h][v] = 0.f;
+        for (int v = 0; v < 4; ++v) yacc[h][v] = 0.f;
 
-    bool waited = false;
+    bool first = true;
     for (int pa = g0; pa < g1; pa += GP) {
         const int pb = min(g1, pa + GP);
-        const int nw = (pb - pa - warp + W - 1) / W;  // groups of this warp (may be <= 0)
+        const int ng = pb - pa;
+        // groups of this warp: pa + team + i * WT, i < nw (none for a tile past the edge)
+        const int nw = tile_ok ? (ng - team + WT - 1) / WT : 0;
 
-        // Issue the copies of the warp's i-th group (records of all valid tiles) into slot i % S.
+        // Copy the warp's i-th record into the next ring slot (16 + 8 or 16 + 16 bytes per lane).
+        const uint8_t* wsrc = p.packed + ((size_t)(T0 + tile) * p.G + pa + team) * F::kBytes;
+        const size_t wstep = (size_t)WT * F::kBytes;
+        int islot = 0;
         auto issue = [&](int i) {
             if (i < nw) {
-                const int g = pa + warp + i * W;
-                const uint32_t slot = ring_s + (uint32_t)((i % S) * NT * F::kBytes);
-#pragma unroll
-                for (int t = 0; t < NT; ++t) {
-                    if (t < ntv) {
-                        const uint8_t* src =
-                            p.packed + ((size_t)(T0 + t) * p.G + g) * F::kBytes;
-                        const uint32_t dst = slot + t * F::kBytes;
-                        cp_async16(dst + lane * 16, src + lane * 16);
-                        if (F::kChunk1 == 16)
-                            cp_async16(dst + 512 + lane * 16, src + 512 + lane * 16);
-                        else
-                            cp_async8(dst + 512 + lane * 8, src + 512 + lane * 8);
-                    }
-                }
+                const uint8_t* src = wsrc + (size_t)i * wstep;
+                const uint32_t dst = ring_s + (uint32_t)(islot * F::kBytes);
+                cp_async16(dst + lane * 16, src + lane * 16);
+                if (F::kChunk1 == 16)
+                    cp_async16(dst + 512 + lane * 16, src + 512 + lane * 16);
+                else
+                    cp_async8(dst + 512 + lane * 8, src + 512 + lane * 8);
             }
             cp_async_commit();
+            islot = islot + 1 == S ? 0 : islot + 1;
         };
 
         for (int i = 0; i < S - 1; ++i) issue(i);
 
-        if (!waited) {  // X (and Y) belong to the preceding kernel until it completes
-            pdl_wait();
-            pdl_launch_dependents();
-            waited = true;
-        }
-        if (pa != g0) __syncthreads();  // every warp is done reading the previous phase's xs
-
-        // Stage x' = x * 2^-p in MMA B-fragment order, plus S_g = sum x and 1024 * S'_g.
-        {
-            const int ng = pb - pa;
-            const int sc = lane >> 3, sj = lane & 7;  // staging lane -> (c, j)
-            const int pA = pair_shift<BITS>(2 * sj), pB = pair_shift<BITS>(2 * sj + 1);
-            const __half2 fA = __float2half2_rn(__int_as_float((127 - pA) << 23));
-            const __half2 fB = __float2half2_rn(__int_as_float((127 - pB) << 23));
-            for (int e = warp; e < M * ng; e += W) {
-                const int b = e / ng, gl = e - b * ng;
-                const uint16_t* xrow = p.X + (size_t)b * p.K + (size_t)(pa + gl) * 128;
-                const uint32_t xa = *reinterpret_cast<const uint32_t*>(xrow + 16 * sj + 2 * sc);
-                const uint32_t xb =
-                    *reinterpret_cast<const uint32_t*>(xrow + 16 * sj + 8 + 2 * sc);
-                const __half2 ha = *reinterpret_cast<const __half2*>(&xa);
-                const __half2 hb = *reinterpret_cast<const __half2*>(&xb);
-                const __half2 sa = __hmul2(ha, fA), sb = __hmul2(hb, fB);
-                const float2 fa = __half22float2(ha), fb = __half22float2(hb);
-                const float2 ga = __half22float2(sa), gb = __half22float2(sb);
-                float sum = (fa.x + fa.y) + (fb.x + fb.y);
-                float psc = (ga.x + ga.y) + (gb.x + gb.y);
-                uint2 v;
-                v.x = *reinterpret_cast<const uint32_t*>(&sa);
-                v.y = *reinterpret_cast<const uint32_t*>(&sb);
-                reinterpret_cast<uint2*>(xs)[2 * (((b * GP + gl) * 4 + (sj >> 1)) * 4 + sc) +
-                                             (sj & 1)] = v;
-#pragma unroll
-                for (int o = 16; o > 0; o >>= 1) {
-                    sum += __shfl_xor_sync(0xffffffffu, sum, o);
-                    psc += __shfl_xor_sync(0xffffffffu, psc, o);
-                }
-                if (lane == 0) {
-                    ssum[b * GP + gl] = sum;
-                    psum[b * GP + gl] = 1024.f * psc;
+        if (first) {
+            // Scales and zeros of every group and tile of this CTA (32 + 16 bytes per (group,
+            // tile)), in flight together with the weight records: warp per group, lane per
+            // (tile, 16-byte piece).
+            const uint32_t ss = (uint32_t)__cvta_generic_to_shared(s_sm);
+            const uint32_t zs = (uint32_t)__cvta_generic_to_shared(z_sm);
+            const int t = lane >> 2, piece = lane & 3;
+            if (t < ntv && piece < 3) {
+                for (int gl = warp; gl < g1 - g0; gl += W) {
+                    const size_t goff = (size_t)(g0 + gl) * p.N + (size_t)(T0 + t) * 16;
+                    const uint32_t slot = (uint32_t)(gl * NT + t);
+                    if (piece < 2)
+                        cp_async16(ss + slot * 32 + piece * 16, p.s + goff + piece * 8);
+                    else
+                        cp_async16(zs + slot * 16, p.z + goff);
                 }
             }
+            cp_async_commit();
+            // X (and Y) belong to the preceding kernel on the stream until it completes.
+            pdl_wait();
+            LAQ_TRACE(1);
+            first = false;
+        } else {
+            __syncthreads();  // every warp is done reading the previous phase's X, S and P
         }
-        __syncthreads();
+
+        // Raw X of the phase (row b's groups pa..pb-1 are 256 * ng contiguous bytes), then
+        // S_g = sum_k x_k and P_g = sum_k c_k x_k per (row, group): 8 threads per group, each
+        // summing 16 consecutive rows, combined by shuffles.
+        {
+            const uint32_t xs_s = (uint32_t)__cvta_generic_to_shared(xs);
+            for (int b = 0; b < M; ++b) {
+                const uint16_t* src = p.X + (size_t)b * p.K + (size_t)pa * 128;
+                const uint32_t dst = xs_s + (uint32_t)(b * GP * 256);
+                for (int u = threadIdx.x; u < ng * 16; u += blockDim.x)
+                    cp_async16(dst + u * 16, src + u * 8);
+            }
+            cp_async_commit();
+            asm volatile("cp.async.wait_all;\n" ::: "memory");
+            __syncthreads();
+            LAQ_TRACE(6);
+            const int seg = threadIdx.x & 7;
+            for (int base = 0; base < M * ng; base += (int)(blockDim.x >> 3)) {
+                const int blk = base + (int)(threadIdx.x >> 3);
+                float sx = 0.f, px = 0.f;
+                int b = 0, gl = 0;
+                if (blk < M * ng) {
+                    b = blk / ng;
+                    gl = blk - b * ng;
+                    const uint4* src = xs + (size_t)(b * GP + gl) * 16 + seg * 2;
+#pragma unroll
+                    for (int q = 0; q < 2; ++q) {
+                        const uint4 v = src[q];
+                        const uint32_t w4[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+                        for (int e = 0; e < 4; ++e) {
+                            const float2 f = __half22float2(
+                                *reinterpret_cast<const __half2*>(&w4[e]));
+                            const float pair = f.x + f.y;
+                            sx += pair;
+                            px = fmaf(row_offset<BITS>((seg & 1) * 8 + q * 4 + e), pair, px);
+                        }
+                    }
+                }
+#pragma unroll
+                for (int o = 1; o < 8; o <<= 1) {
+                    sx += __shfl_xor_sync(0xffffffffu, sx, o);
+                    px += __shfl_xor_sync(0xffffffffu, px, o);
+                }
+                if (seg == 0 && blk < M * ng) {
+                    ssum[b * GP + gl] = sx;
+                    psum[b * GP + gl] = px;
+                }
+            }
+            __syncthreads();
+            LAQ_TRACE(7);
+            // Epilogue table: {s, s * (z * S_g + P_g)} per (row b, group, tile, column), so the
+            // group epilogue is y += s * D - s * (P + z S), one shared load per output.
+            for (int idx = threadIdx.x; idx < M * ng * NT * 16; idx += blockDim.x) {
+                const int row = idx & 15, t = (idx >> 4) % NT, rest = (idx >> 4) / NT;
+                const int b = rest / ng, gl = rest - b * ng;
+                if (t < ntv) {
+                    const int e = ((pa - g0 + gl) * NT + t) * 16 + row;
+                    const float sv = __half2float(__ushort_as_half(s_sm[e]));
+                    const float corr =
+                        fmaf((float)z_sm[e], ssum[b * GP + gl], psum[b * GP + gl]);
+                    ab[((b * GP + gl) * NT + t) * 16 + row] = make_float2(sv, sv * corr);
+                }
+            }
+            __syncthreads();
+            LAQ_TRACE(2);
+        }
 
         // Batch row and group column of this lane's B fragment (MMA column R).
         const int bl = MP <= 8 ? R / GPA : R;
         const int gil = MP <= 8 ? R % GPA : 0;
 
-        float D[NT][NH][4];
-        uint32_t sz[NT][4];  // s bits | z << 16 for the block's epilogue
+        float D[2][NH][4];  // two independent accumulator chains (even / odd k16 steps)
+        int rslot = 0;
+        // With S - 1 >= nw every record of the warp was copied in the prologue and has landed.
+        const bool streaming = S - 1 < nw;
         for (int i = 0; i < nw; ++i) {
-            issue(i + S - 1);
-            cp_async_wait(S - 1);
+            LAQ_TRACE_LOOP(0, i);
+            if (streaming) {
+                issue(i + S - 1);
+                cp_async_wait(S - 1);
+            }
+            LAQ_TRACE_LOOP(1, i);
 
             const int gi = GPA > 1 ? i % GPA : 0;
-            const int gl = warp + i * W;  // group index within the phase
+            const int gl = team + i * WT;  // group index within the phase
             if (gi == 0) {
-                // Start of an accumulator block: zero D, fetch s and z for its epilogue.
 #pragma unroll
-                for (int t = 0; t < NT; ++t) {
+                for (int a = 0; a < 2; ++a)
 #pragma unroll
                     for (int h = 0; h < NH; ++h)
 #pragma unroll
-                        for (int v = 0; v < 4; ++v) D[t][h][v] = 0.f;
-#pragma unroll
-                    for (int v = 0; v < 4; ++v) {
-                        const int col = 2 * c + (v & 1);
-                        const int giv = MP <= 8 ? col % GPA : 0;
-                        const bool ok = t < ntv && i + giv < nw &&
-                                        (MP <= 8 ? col / GPA < M : true);
-                        uint32_t val = 0;
-                        if (ok) {
-                            const size_t gidx =
-                                (size_t)(pa + warp + (i + giv) * W) * p.N +
-                                (size_t)(T0 + t) * 16 + R + 8 * (v >> 1);
-                            val = (uint32_t)__ldg(p.s + gidx) | ((uint32_t)__ldg(p.z + gidx) << 16);
-                        }
-                        sz[t][v] = val;
-                    }
-                }
+                        for (int v = 0; v < 4; ++v) D[a][h][v] = 0.f;
             }
 
-            // B fragments of this group: x' for lanes whose column belongs to it, else zeros.
+            // B fragments: x[32c .. 32c+31] of this group for lanes whose column belongs to
+            // it, zeros for the others.
             uint32_t B[NH][8][2];
 #pragma unroll
             for (int h = 0; h < NH; ++h) {
                 const int b = bl + 8 * h;
                 const bool act = gil == gi && b < M;
-                const uint4* src = act ? xs + (size_t)(b * GP + gl) * 16 : zblk;
+                const uint4* src = act ? xs + (size_t)(b * GP + gl) * 16 + c * 4 : zblk;
 #pragma unroll
                 for (int q = 0; q < 4; ++q) {
-                    const uint4 v = src[q * 4 + c];
+                    const uint4 v = src[q];
                     B[h][2 * q][0] = v.x;
                     B[h][2 * q][1] = v.y;
                     B[h][2 * q + 1][0] = v.z;
                     B[h][2 * q + 1][1] = v.w;
                 }
             }
+            LAQ_TRACE_LOOP(2, i);
 
-            const uint8_t* slot = ring_w + (size_t)(i % S) * NT * F::kBytes;
-#pragma unroll
-            for (int t = 0; t < NT; ++t) {
-                if (t < ntv) {
-                    uint32_t wd[WPL];
-                    const uint4 c0 = *reinterpret_cast<const uint4*>(slot + t * F::kBytes +
-                                                                     lane * 16);
-                    wd[0] = c0.x; wd[1] = c0.y; wd[2] = c0.z; wd[3] = c0.w;
-                    if constexpr (BITS == 4) {
-                        const uint4 c1 = *reinterpret_cast<const uint4*>(
-                            slot + t * F::kBytes + 512 + lane * 16);
-                        wd[4] = c1.x; wd[5] = c1.y; wd[6] = c1.z; wd[7] = c1.w;
-                    } else {
-                        const uint2 c1 = *reinterpret_cast<const uint2*>(
-                            slot + t * F::kBytes + 512 + lane * 8);
-                        wd[4] = c1.x; wd[5] = c1.y;
-                    }
-                    uint32_t a[8][4];
-                    extract<BITS>(wd, a);
-#pragma unroll
-                    for (int j = 0; j < 8; ++j)
-#pragma unroll
-                        for (int h = 0; h < NH; ++h)
-                            mma16816(D[t][h], a[j][0], a[j][1], a[j][2], a[j][3], B[h][j][0],
-                                     B[h][j][1]);
+            {
+                const uint8_t* slot = ring_w + (size_t)rslot * F::kBytes;
+                uint32_t wd[WPL];
+                const uint4 c0 = *reinterpret_cast<const uint4*>(slot + lane * 16);
+                wd[0] = c0.x; wd[1] = c0.y; wd[2] = c0.z; wd[3] = c0.w;
+                if constexpr (BITS == 4) {
+                    const uint4 c1 = *reinterpret_cast<const uint4*>(slot + 512 + lane * 16);
+                    wd[4] = c1.x; wd[5] = c1.y; wd[6] = c1.z; wd[7] = c1.w;
+                } else {
+                    const uint2 c1 = *reinterpret_cast<const uint2*>(slot + 512 + lane * 8);
+                    wd[4] = c1.x; wd[5] = c1.y;
                 }
+                uint32_t a[8][4];
+                extract<BITS>(wd, p.exps, a);
+#pragma unroll
+                for (int j = 0; j < 8; ++j)
+#pragma unroll
+                    for (int h = 0; h < NH; ++h)
+                        mma16816(D[j & 1][h], a[j][0], a[j][1], a[j][2], a[j][3], B[h][j][0],
+                                 B[h][j][1]);
             }
+            rslot = rslot + 1 == S ? 0 : rslot + 1;
+            LAQ_TRACE_LOOP(3, i);
 
             if (gi == GPA - 1 || i == nw - 1) {
-                // Group epilogue (Eq. (1)): y += s * (D - 1024 S' - z S) per (group, column, row).
+                // Group epilogue (Eq. (1)): y += s * (D - P - z S) per (group, column, row).
                 const int ib = i - gi;
 #pragma unroll
-                for (int t = 0; t < NT; ++t) {
+                for (int h = 0; h < NH; ++h) {
 #pragma unroll
-                    for (int h = 0; h < NH; ++h) {
-#pragma unroll
-                        for (int v = 0; v < 4; ++v) {
-                            const int col = 2 * c + (v & 1);
-                            const int b = MP <= 8 ? col / GPA : 8 * h + col;
-                            const int giv = MP <= 8 ? col % GPA : 0;
-                            if (t < ntv && b < M && ib + giv < nw) {
-                                const int lg = warp + (ib + giv) * W;
-                                const uint32_t e = sz[t][v];
-                                const float sv = __half2float(__ushort_as_half((uint16_t)e));
-                                const float zv = (float)(e >> 16);
-                                const float corr = fmaf(zv, ssum[b * GP + lg], psum[b * GP + lg]);
-                                yacc[t][h][v] = fmaf(sv, D[t][h][v] - corr, yacc[t][h][v]);
-                            }
+                    for (int v = 0; v < 4; ++v) {
+                        const int col = 2 * c + (v & 1);
+                        const int b = MP <= 8 ? col / GPA : 8 * h + col;
+                        const int giv = MP <= 8 ? col % GPA : 0;
+                        if (b < M && ib + giv < nw) {
+                            const int lg = team + (ib + giv) * WT;        // in the phase
+                            const float2 sa = ab[((b * GP + lg) * NT + tile) * 16 + R + 8 * (v >> 1)];
+                            const float d = D[0][h][v] + D[1][h][v];
+                            yacc[h][v] = fmaf(sa.x, d, yacc[h][v]) - sa.y;
                         }
                     }
                 }
             }
+            LAQ_TRACE_LOOP(4, i);
         }
         asm volatile("cp.async.wait_all;\n" ::: "memory");
     }
-    if (!waited) {
-        pdl_wait();
-        pdl_launch_dependents();
-    }
+    if (first) pdl_wait();  // a CTA without groups still writes Y after the previous kernel
+    LAQ_TRACE(3);
 
-    // ---- reduction: group columns (shuffles) -> warps (shared) -> cluster CTAs (DSMEM) ----
-    __syncthreads();  // the ring is free: reuse it for the per-warp partial sums
+    // ---- reduction: group columns (shuffles) -> warps of a tile (shared) -> cluster (DSMEM) ----
+    // Per-warp partials live in the (now idle) ring as red[W][MP][16]; b >= M is unused.
+    __syncthreads();
     float* red = reinterpret_cast<float*>(smem);
-    const int E = NT * M * 16;
-#pragma unroll
-    for (int t = 0; t < NT; ++t) {
-        float* rw = red + (size_t)warp * E + t * M * 16;
+    {
+        float* rw = red + (size_t)warp * MP * 16;
         if (MP <= 8 && GPA >= 2) {
-            float y0 = yacc[t][0][0] + yacc[t][0][1];
-            float y1 = yacc[t][0][2] + yacc[t][0][3];
+            float y0 = yacc[0][0] + yacc[0][1];
+            float y1 = yacc[0][2] + yacc[0][3];
             if (GPA >= 4) {
                 y0 += __shfl_xor_sync(0xffffffffu, y0, 1);
                 y1 += __shfl_xor_sync(0xffffffffu, y1, 1);
@@ -411,7 +500,7 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 2) gemm_kernel(const Params p)
                 y1 += __shfl_xor_sync(0xffffffffu, y1, 2);
             }
             const int b = (2 * c) / GPA;
-            if ((2 * c) % GPA == 0 && b < M) {
+            if ((2 * c) % GPA == 0) {
                 rw[b * 16 + R] = y0;
                 rw[b * 16 + R + 8] = y1;
             }
@@ -419,22 +508,23 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 2) gemm_kernel(const Params p)
 #pragma unroll
             for (int h = 0; h < NH; ++h)
 #pragma unroll
-                for (int v = 0; v < 4; ++v) {
-                    const int b = 8 * h + 2 * c + (v & 1);
-                    if (b < M) rw[b * 16 + R + 8 * (v >> 1)] = yacc[t][h][v];
-                }
+                for (int v = 0; v < 4; ++v)
+                    rw[(8 * h + 2 * c + (v & 1)) * 16 + R + 8 * (v >> 1)] = yacc[h][v];
         }
     }
     __syncthreads();
+    constexpr int E = NT * MP * 16;
     for (int e = threadIdx.x; e < E; e += blockDim.x) {
+        const int t = e / (MP * 16), r = e % (MP * 16);
         float acc = 0.f;
-        for (int w = 0; w < W; ++w) acc += red[(size_t)w * E + e];
+        for (int u = 0; u < WT; ++u) acc += red[(size_t)(u * NT + t) * MP * 16 + r];
         part[e] = acc;
     }
+    LAQ_TRACE(4);
 
     auto store = [&](int e, float acc) {
-        const int t = e / (M * 16), b = (e / 16) % M, row = e % 16;
-        if (t < ntv) {
+        const int t = e / (MP * 16), b = (e / 16) % MP, row = e % 16;
+        if (t < ntv && b < M) {
             const __half hv = __float2half_rn(acc);
             p.Y[(size_t)b * p.N + (size_t)(T0 + t) * 16 + row] = __half_as_ushort(hv);
         }
@@ -442,6 +532,7 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 2) gemm_kernel(const Params p)
     if (C == 1) {
         __syncthreads();
         for (int e = threadIdx.x; e < E; e += blockDim.x) store(e, part[e]);
+        LAQ_TRACE(5);
     } else {
         cg::cluster_group cluster = cg::this_cluster();
         cluster.sync();  // every CTA's partial sums are complete
@@ -451,6 +542,7 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 2) gemm_kernel(const Params p)
             store(e, acc);
         }
         cluster.sync();  // peers have finished reading this CTA's shared memory
+        LAQ_TRACE(5);
     }
 }
 
@@ -482,21 +574,24 @@ int nt_index(int nt) { return nt == 1 ? 0 : nt == 2 ? 1 : 2; }
 
 std::atomic<size_t> g_attr_limit[2][5][3];  // max dynamic smem already granted per kernel
 
-constexpr size_t kXsBudget = 48 * 1024;  // shared memory for staged X per phase
+constexpr size_t kXsBudget = 64 * 1024;  // shared memory for staged X (and its tables) per phase
 
 }  // namespace
 
 size_t gemm_smem_bytes(const GemmLaunch& L, int* groups_per_phase) {
     const size_t rec = L.bits == 4 ? 1024 : 768;
-    const size_t ring = (size_t)L.warps * L.stages * L.tiles_per_cta * rec;
+    const size_t ring = (size_t)L.warps * L.stages * rec;
     const int G = L.K / 128;
     const int gc = (G + L.cluster - 1) / L.cluster;
-    const size_t per_group = (size_t)L.M * (256 + 8);
+    // raw X, S and P, and the epilogue table of one group
+    const size_t per_group = (size_t)L.M * (256 + 8 + (size_t)L.tiles_per_cta * 128);
     int gpp = (int)(kXsBudget / per_group);
     if (gpp > gc) gpp = gc;
     if (gpp < 1) gpp = 1;
     if (groups_per_phase) *groups_per_phase = gpp;
-    return ring + 256 + (size_t)gpp * per_group + (size_t)L.tiles_per_cta * L.M * 16 * 4;
+    const int mp = mp_class(L.M);
+    const size_t sz = (size_t)(gc > 0 ? gc : 1) * L.tiles_per_cta * 48;  // s (32 B) + z (16 B)
+    return ring + (size_t)gpp * per_group + 64 + sz + (size_t)L.tiles_per_cta * mp * 16 * 4;
 }
 
 cudaError_t launch_gemm(const GemmLaunch& L, size_t smem_limit, cudaStream_t stream) {
@@ -508,8 +603,14 @@ cudaError_t launch_gemm(const GemmLaunch& L, size_t smem_limit, cudaStream_t str
                                     : pick_mp<3>(mp, L.tiles_per_cta);
     std::atomic<size_t>& granted = g_attr_limit[L.bits == 4][mp_index(mp)][nt_index(L.tiles_per_cta)];
     if (granted.load() < smem) {
-        const cudaError_t e = cudaFuncSetAttribute(
+        // Every instance asks for the largest shared-memory carveout, so kernels of different
+        // shapes following each other in a decode step never reconfigure L1 / shared memory.
+        cudaError_t e = cudaFuncSetAttribute(
             (const void*)fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_limit);
+        if (e != cudaSuccess) return e;
+        e = cudaFuncSetAttribute((const void*)fn,
+                                 cudaFuncAttributePreferredSharedMemoryCarveout,
+                                 (int)cudaSharedmemCarveoutMaxShared);
         if (e != cudaSuccess) return e;
         granted.store(smem_limit);
     }
@@ -526,6 +627,8 @@ cudaError_t launch_gemm(const GemmLaunch& L, size_t smem_limit, cudaStream_t str
     prm.T = L.N / 16;
     prm.stages = L.stages;
     prm.gpp = gpp;
+    prm.gc = (prm.G + L.cluster - 1) / L.cluster;
+    prm.exps = exps_for(L.bits);
 
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)((prm.T + L.tiles_per_cta - 1) / L.tiles_per_cta),

@@ -78,7 +78,7 @@ __global__ void quantize_rtn_kernel(const uint16_t* __restrict__ W, int64_t N,
     }
 }
 
-// ---- record layout (see laq.h): lane l = 4r + c owns columns r, r+8 and rows 16j+8h+2c+e ----
+// ---- record layout (see laq.h): lane l = 4r + c owns columns r, r+8 and rows 32c+4j+2h+e ----
 
 // Code at (row-in-record kk, column-in-tile nn) of record (t, g).
 __device__ __forceinline__ uint32_t code_at(const uint8_t* __restrict__ codes, int64_t N,
@@ -106,7 +106,7 @@ __global__ void pack_kernel(const uint8_t* __restrict__ codes, int64_t N, int64_
                 for (int f = 0; f < 4; ++f) {
                     const int h = f & 1, row = f >> 1;
                     const uint32_t q =
-                        code_at(codes, N, t, g, 16 * j + 8 * h + 2 * c + e, r + 8 * row) & 15u;
+                        code_at(codes, N, t, g, 32 * c + 4 * j + 2 * h + e, r + 8 * row) & 15u;
                     word |= q << (16 * e + 4 * f);
                 }
             out[(j >> 2) * 128 + 4 * lane + (j & 3)] = word;
@@ -115,7 +115,7 @@ __global__ void pack_kernel(const uint8_t* __restrict__ codes, int64_t N, int64_
         uint32_t* out = packed + rec * 192;
         // pair i = 2j + h of row (r or r+8) -> the 3-bit code at element e
         auto pair_code = [&](int i, int row, int e) -> uint32_t {
-            return code_at(codes, N, t, g, 16 * (i >> 1) + 8 * (i & 1) + 2 * c + e,
+            return code_at(codes, N, t, g, 32 * c + 4 * (i >> 1) + 2 * (i & 1) + e,
                            r + 8 * row) & 7u;
         };
 #pragma unroll
@@ -123,12 +123,12 @@ __global__ void pack_kernel(const uint8_t* __restrict__ codes, int64_t N, int64_
             uint32_t word = 0;
 #pragma unroll
             for (int e = 0; e < 2; ++e) {
-                uint32_t half = pair_code(w, 0, e)                       // bits 0-2
-                              | pair_code(6 + w, 0, e) << 3              // bits 3-5
-                              | pair_code(12 + (w >> 1), w & 1, e) << 6  // bits 6-8
-                              | pair_code(w, 1, e) << 9                  // bits 9-11
-                              | pair_code(6 + w, 1, e) << 12;            // bits 12-14
-                half |= ((pair_code(15, w >= 3 ? 1 : 0, e) >> (w % 3)) & 1u) << 15;
+                uint32_t half = (pair_code(15, w >= 3 ? 1 : 0, e) >> (w % 3)) & 1u;  // bit 0
+                half |= pair_code(w, 0, e) << 1                          // bits 1-3
+                      | pair_code(6 + w, 0, e) << 4                      // bits 4-6
+                      | pair_code(12 + (w >> 1), w & 1, e) << 7          // bits 7-9
+                      | pair_code(w, 1, e) << 10                         // bits 10-12
+                      | pair_code(6 + w, 1, e) << 13;                    // bits 13-15
                 word |= half << (16 * e);
             }
             out[w < 4 ? 4 * lane + w : 128 + 2 * lane + (w - 4)] = word;
@@ -157,7 +157,7 @@ __global__ void unpack_kernel(const uint32_t* __restrict__ packed, int64_t N, in
             for (int e = 0; e < 2; ++e)
 #pragma unroll
                 for (int f = 0; f < 4; ++f)
-                    put(16 * j + 8 * (f & 1) + 2 * c + e, r + 8 * (f >> 1),
+                    put(32 * c + 4 * j + 2 * (f & 1) + e, r + 8 * (f >> 1),
                         (word >> (16 * e + 4 * f)) & 15u);
         }
     } else {
@@ -166,7 +166,7 @@ __global__ void unpack_kernel(const uint32_t* __restrict__ packed, int64_t N, in
 #pragma unroll
         for (int w = 0; w < 6; ++w) words[w] = in[w < 4 ? 4 * lane + w : 128 + 2 * lane + (w - 4)];
         auto put_pair = [&](int i, int row, int e, uint32_t q) {
-            put(16 * (i >> 1) + 8 * (i & 1) + 2 * c + e, r + 8 * row, q);
+            put(32 * c + 4 * (i >> 1) + 2 * (i & 1) + e, r + 8 * row, q);
         };
 #pragma unroll
         for (int e = 0; e < 2; ++e) {
@@ -174,12 +174,12 @@ __global__ void unpack_kernel(const uint32_t* __restrict__ packed, int64_t N, in
 #pragma unroll
             for (int w = 0; w < 6; ++w) {
                 const uint32_t half = (words[w] >> (16 * e)) & 0xffffu;
-                put_pair(w, 0, e, half & 7u);
-                put_pair(6 + w, 0, e, (half >> 3) & 7u);
-                put_pair(12 + (w >> 1), w & 1, e, (half >> 6) & 7u);
-                put_pair(w, 1, e, (half >> 9) & 7u);
-                put_pair(6 + w, 1, e, (half >> 12) & 7u);
-                spare[w >= 3 ? 1 : 0] |= ((half >> 15) & 1u) << (w % 3);
+                spare[w >= 3 ? 1 : 0] |= (half & 1u) << (w % 3);
+                put_pair(w, 0, e, (half >> 1) & 7u);
+                put_pair(6 + w, 0, e, (half >> 4) & 7u);
+                put_pair(12 + (w >> 1), w & 1, e, (half >> 7) & 7u);
+                put_pair(w, 1, e, (half >> 10) & 7u);
+                put_pair(6 + w, 1, e, (half >> 13) & 7u);
             }
             put_pair(15, 0, e, spare[0]);
             put_pair(15, 1, e, spare[1]);

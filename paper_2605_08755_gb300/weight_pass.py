@@ -36,40 +36,72 @@ def shapes(model):
     return {"qwen3-4b": inputs.QWEN3_4B, "qwen3-8b": inputs.QWEN3_8B}[model]
 
 
+# Projections that read the same activation and may run as one GEMV over concatenated columns.
+FUSED = (("qkv", ("q", "k", "v")), ("o", ("o",)), ("gate_up", ("gate", "up")), ("down", ("down",)))
+
+
 class WeightPass:
+    """The 7 x layers projections of a decode step, launched in stream order.
+
+    With ``fuse``, q|k|v and gate|up (which share their input in a decoder) are quantized as one
+    weight over concatenated output columns and run as one GEMV each (4 launches per layer);
+    quantization is per column, so their codes, scales and zeros are those of the separate
+    projections."""
+
     def __init__(self, model="qwen3-4b", bits=3, M=1, layers=inputs.LAYERS, seed=0,
-                 outliers=False, device="cuda"):
+                 outliers=False, device="cuda", pdl=True, fuse=False):
         self.model, self.bits, self.M, self.layers = model, bits, M, layers
-        self.seed, self.outliers = seed, outliers
+        self.seed, self.outliers, self.fuse = seed, outliers, fuse
         self.device = torch.device(device)
-        self.linears = []   # [(layer, proj_index, name, QuantLinear)]
-        plan = [(layer, pi, name, K, N) for layer in range(layers)
-                for pi, (name, K, N) in enumerate(shapes(model))]
+        names = [n for n, _, _ in shapes(model)]
+        groups = ([[names.index(m) for m in members] for _, members in FUSED] if fuse
+                  else [[i] for i in range(len(names))])
+        gnames = [n for n, _ in FUSED] if fuse else names
+        plan = []
+        for layer in range(layers):
+            for gname, members in zip(gnames, groups):
+                K = shapes(model)[members[0]][1]
+                N = sum(shapes(model)[i][2] for i in members)
+                plan.append((layer, tuple(members), gname, K, N))
         xs = sum(M * K for *_, K, N in plan)
         ys = sum(M * N for *_, K, N in plan)
         self.Xbuf = torch.empty((xs,), dtype=torch.float16, device=self.device)
         self.Ybuf = torch.zeros((ys,), dtype=torch.float16, device=self.device)
+        self.linears = []   # [(layer, member projection indices, name, QuantLinear)]
         self.X, self.Y = [], []
         xo = yo = 0
-        for layer, pi, name, K, N in plan:
-            sd = inputs.proj_seed(seed, layer, pi)
-            W = self.weight(layer, pi)
-            self.linears.append((layer, pi, name, QuantLinear(W, bits)))
+        for layer, members, name, K, N in plan:
+            W = self.weight(layer, members)
+            self.linears.append((layer, members, name, QuantLinear(W, bits)))
             del W
             x = self.Xbuf[xo:xo + M * K].view(M, K)
-            x.copy_(inputs.activations_torch(M, K, sd, self.device))
+            x.copy_(inputs.activations_torch(M, K, inputs.proj_seed(seed, layer, members[0]),
+                                             self.device))
             self.X.append(x)
             self.Y.append(self.Ybuf[yo:yo + M * N].view(M, N))
             xo += M * K
             yo += M * N
-        self.configs = [None] * len(self.linears)
+        # The library's own plan for each shape; with pdl, each launch may start (and prefetch
+        # its weights, which no kernel of the pass writes) while the previous one finishes.
+        sms = torch.cuda.get_device_properties(self.device).multi_processor_count
+        self.configs = []
+        for *_, q in self.linears:
+            c = _lib.laq_gemm_plan(M, q.K, q.N, bits, sms)
+            c.pdl = 1 if pdl else 0
+            self.configs.append(c)
         torch.cuda.synchronize(self.device)
 
-    def weight(self, layer, proj_index):
-        """The fp16 weight of one projection, regenerated from its seed."""
-        _, K, N = shapes(self.model)[proj_index]
-        return inputs.weights_torch(K, N, inputs.proj_seed(self.seed, layer, proj_index),
-                                    self.device, outliers=self.outliers)
+    def weight(self, layer, members):
+        """The fp16 weight of one launch (its member projections side by side), regenerated
+        from their seeds."""
+        if isinstance(members, int):
+            members = (members,)
+        parts = []
+        for pi in members:
+            _, K, N = shapes(self.model)[pi]
+            parts.append(inputs.weights_torch(K, N, inputs.proj_seed(self.seed, layer, pi),
+                                              self.device, outliers=self.outliers))
+        return parts[0] if len(parts) == 1 else torch.cat(parts, dim=1)
 
     @property
     def launches(self):

@@ -78,6 +78,8 @@ def test_gemm_argument_validation(L):
     assert gemm(L, Y=ODD) == 5
     assert gemm(L, packed=ODD) == 5
     assert gemm(L, s=ctypes.c_void_p(0x10001)) == 5
+    assert gemm(L, s=ODD) == 5
+    assert gemm(L, z=ctypes.c_void_p(0x10008)) == 5
     # empty problems are no-ops that never touch the device
     assert gemm(L, M=0) == 0
     assert gemm(L, N=0, Y=None) == 0
@@ -96,8 +98,10 @@ def test_gemm_config_validation(L):
     assert run(cluster=3) == 9
     assert run(cluster=16) == 9
     assert run(stages=1) == 9
-    assert run(stages=9) == 9
+    assert run(stages=17) == 9
     assert run(pdl=2) == 9
+    assert run(tiles_per_cta=2, warps=3) == 9
+    assert run(tiles_per_cta=4, warps=2) == 9
     assert L.laq_gemm_wxg128_config(FAKE, 1, 256, 32, FAKE, FAKE, FAKE, 3, FAKE, None,
                                     None) == 1
 
@@ -131,10 +135,9 @@ def test_plan_is_valid_for_every_workload_shape(L, bits, M):
             assert c.tiles_per_cta in (1, 2, 4)
             assert 1 <= c.warps <= 8
             assert c.cluster in (1, 2, 4, 8) and c.cluster <= max(1, K // 128)
-            assert 2 <= c.stages <= 8
+            assert 2 <= c.stages <= 16
             assert c.pdl == 0
-            if M > 8:
-                assert c.tiles_per_cta <= 2
+            assert c.warps % c.tiles_per_cta == 0
 
 
 def test_plan_rejects_bad_arguments(L):

@@ -124,7 +124,7 @@ def test_gemm_parity_shapes(bits, M, K, N):
 
 
 CONFIGS = [laq.GemmConfig.make(nt, w, cl, st, pdl)
-           for nt, w, cl, st, pdl in itertools.product((1, 2, 4), (1, 3, 8), (1, 2, 8), (2, 3, 8),
+           for nt, w, cl, st, pdl in itertools.product((1, 2, 4), (1, 2, 3, 4, 8), (1, 2, 8), (2, 3, 16),
                                                        (0, 1))]
 
 
@@ -132,13 +132,15 @@ SMEM_OPTIN = 232448   # bytes of dynamic shared memory a CTA may opt into on sm_
 
 
 def smem_needed(M, K, bits, cfg):
-    """Mirror of the library's shared-memory budget: cp.async ring, zero block, staged X
-    (up to 48 KB per phase), per-CTA partial sums."""
+    """Mirror of the library's shared-memory budget: per-warp cp.async rings, staged X with its
+    group sums (up to 48 KB per phase), zero block, scales and zeros, per-CTA partial sums."""
     rec = 1024 if bits == 4 else 768
     gc = -(-(K // 128) // cfg.cluster)
-    gpp = max(1, min(gc, 48 * 1024 // (M * 264)))
-    return (cfg.warps * cfg.stages * cfg.tiles_per_cta * rec + 256 + gpp * M * 264
-            + cfg.tiles_per_cta * M * 64)
+    per_group = M * (264 + cfg.tiles_per_cta * 128)
+    gpp = max(1, min(gc, 64 * 1024 // per_group))
+    mp = 1 if M <= 1 else 2 if M <= 2 else 4 if M <= 4 else 8 if M <= 8 else 16
+    return (cfg.warps * cfg.stages * rec + gpp * per_group + 64 + gc * cfg.tiles_per_cta * 48
+            + cfg.tiles_per_cta * mp * 64)
 
 
 @pytest.mark.parametrize("bits", [3, 4])
@@ -149,7 +151,10 @@ def test_gemm_every_launch_configuration(bits, M):
     X = inputs.activations(M, K, seed=3 * M)
     yref = co.gemm(X, codes, s, z)
     for cfg in CONFIGS:
-        if M > 8 and cfg.tiles_per_cta == 4:
+        if cfg.warps % cfg.tiles_per_cta:
+            with pytest.raises(laq.LaqError) as e:
+                run_gemm(X, packed, s_d, z_d, bits, config=cfg)
+            assert e.value.status == 9
             continue
         if smem_needed(M, K, bits, cfg) > SMEM_OPTIN:
             with pytest.raises(laq.LaqError) as e:

@@ -29,13 +29,13 @@ def built():
 
 
 def check_projection(wp, idx, tiles=None):
-    layer, pi, name, q = wp.linears[idx]
+    layer, members, name, q = wp.linears[idx]
     K, N, bits = q.K, q.N, q.bits
     T, G = N // 16, K // 128
-    rec = 32 * bits * 4
+    rec = 256 * bits           # bytes of one 16-column x 128-row record
     if tiles is None:
         tiles = list(range(T))
-    W = wp.weight(layer, pi).cpu().numpy()
+    W = wp.weight(layer, members).cpu().numpy()
     X = wp.X[idx].cpu().numpy()
     Y = wp.Y[idx].cpu().numpy().astype(np.float64)
     s_gpu = q.s.cpu().numpy().view(np.uint16)
@@ -90,7 +90,7 @@ def test_one_qwen3_4b_layer_fully():
 
 
 def _sampled(wp, layers):
-    for idx, (layer, pi, name, q) in enumerate(wp.linears):
+    for idx, (layer, members, name, q) in enumerate(wp.linears):
         if layer in layers:
             T = q.N // 16
             check_projection(wp, idx, tiles=sorted({0, T // 2, T - 1}))
@@ -109,6 +109,16 @@ def test_qwen3_4b_pass_batch_sweep(bits, M):
     wp = WeightPass(model="qwen3-4b", bits=bits, M=M)
     replay(wp)
     _sampled(wp, layers={5, 30})
+
+
+@pytest.mark.parametrize("bits,M", [(3, 1), (4, 1), (3, 16)])
+def test_qwen3_4b_fused_pass(bits, M):
+    """q|k|v and gate|up as single GEMVs over concatenated columns (4 launches per layer)."""
+    wp = WeightPass(model="qwen3-4b", bits=bits, M=M, fuse=True)
+    assert wp.launches == 4 * 36
+    assert [n for _, _, n, _ in wp.linears[:4]] == ["qkv", "o", "gate_up", "down"]
+    replay(wp)
+    _sampled(wp, layers={0, 35})
 
 
 @pytest.mark.parametrize("M", [1, 16])
