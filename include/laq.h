@@ -43,10 +43,11 @@ typedef enum {
     LAQ_ERR_GROUP = 3,    /* group size is not 128                                       */
     LAQ_ERR_SHAPE = 4,    /* negative size, K % 128 != 0, N % 16 != 0, or a size too big */
     LAQ_ERR_ALIGN = 5,    /* a pointer breaks its alignment requirement                  */
-    LAQ_ERR_M_RANGE = 6,  /* M outside 0..16                                             */
+    LAQ_ERR_M_RANGE = 6,  /* M outside 0..16 (1..4 for laq_gemm_chain)                   */
     LAQ_ERR_CUDA = 7,     /* the CUDA runtime reported an error for the launch           */
-    LAQ_ERR_TIMEOUT = 8,  /* reserved: a bounded device-side wait gave up                */
-    LAQ_ERR_CONFIG = 9    /* an explicit launch configuration is not supported           */
+    LAQ_ERR_TIMEOUT = 8,  /* a bounded device-side wait gave up (laq_gemm_chain status)  */
+    LAQ_ERR_CONFIG = 9,   /* an explicit launch configuration is not supported           */
+    LAQ_ERR_WORKSPACE = 10 /* workspace missing, misaligned or smaller than required      */
 } laq_status;
 
 /* Human-readable name of a status code (static storage, never NULL). */
@@ -162,6 +163,62 @@ laq_status laq_gemm_plan(int64_t M, int64_t K, int64_t N, int bits, int num_sms,
 laq_status laq_gemm_wxg128_config(const void *X, int64_t M, int64_t K, int64_t N,
                                   const void *packed, const void *s, const uint8_t *z, int bits,
                                   void *Y, const laq_gemm_config *cfg, void *stream);
+
+/*
+ * One GEMV of a chain (laq_gemm_chain): Y[M][N] = X[M][K] * W_hat[K][N], with the operands and
+ * rules of laq_gemm_wxg128.  `wait_prev` != 0 marks an entry that reads results of earlier
+ * entries (its X is the output of, or computed from, an earlier Y): it starts only after every
+ * earlier entry has completed.  Entries with wait_prev == 0 join the run of entries since the
+ * last marked one (a "stage") and may execute alongside it, as q, k and v, or gate and up, of a
+ * decoder layer do.  Entry 0's flag is ignored.
+ */
+typedef struct laq_gemv {
+    const void *X;       /* fp16 [M][K], 16-byte aligned                 */
+    const void *packed;  /* laq_pack layout, 16-byte aligned             */
+    const void *s;       /* fp16 [K/128][N], 16-byte aligned             */
+    const uint8_t *z;    /* uint8 [K/128][N], 16-byte aligned            */
+    void *Y;             /* fp16 [M][N], 16-byte aligned, no overlap     */
+    int64_t M, K, N;
+    int32_t bits;
+    int32_t wait_prev;
+} laq_gemv;
+
+/* Most entries one laq_gemm_chain call takes. */
+#define LAQ_CHAIN_MAX 384
+
+/* Workspace bytes laq_gemm_chain needs for `count` entries (0 if count is out of range). */
+size_t laq_chain_workspace_bytes(int32_t count);
+
+/*
+ * Run `count` GEMVs in one persistent kernel launch on `stream`, with the results of issuing
+ * laq_gemm_wxg128 for each entry in order on that stream: the decode-step weight pass of a
+ * decoder (Sec. 5.2, "Inference": decoding streams every projection's weights once per token)
+ * without a kernel boundary between projections.  Each entry's Y is the fp32 sum of its
+ * dequantized products (Eq. (1)) rounded once to fp16, like laq_gemm_wxg128's; the two agree
+ * to fp32 rounding (their summation orders differ).
+ *
+ *   gemvs      HOST array of `count` entries (read during the call only).  All entries share
+ *              `bits` (3 or 4) and M (1..4).  K % 128 == 0, N % 16 == 0, K, N > 0.
+ *   count      0..LAQ_CHAIN_MAX (0: nothing is enqueued).
+ *   workspace  DEVICE buffer of at least laq_chain_workspace_bytes(count) bytes, 16-byte
+ *              aligned, ZERO-FILLED before its first use.  A call that completes normally
+ *              leaves it zero-filled again.  Word 0 (uint32) is the device-side status: 0, or
+ *              LAQ_ERR_TIMEOUT if a wait between stages gave up (after about a second); the
+ *              call's Y values are then undefined and the caller must zero the workspace
+ *              before the next call.  Calls sharing one workspace must not overlap in time.
+ *
+ * Restrictions: the packed codes, scales and zeros of every entry are read ahead of the chain
+ * order, so no entry may write them; an entry may not read a Y written by an entry of its own
+ * stage; the X of one stage (M * K * 2 bytes summed over its entries) must fit the kernel's
+ * shared memory beside a weight ring of at least 8 / M-class + 1 records per warp
+ * (LAQ_ERR_SHAPE otherwise; about 100 KB on GB300 at M = 1, and the more X, the shallower
+ * the ring).  Uses every SM of
+ * the device with one cooperative CTA each, so concurrent kernels on other streams wait.
+ * Returns LAQ_ERR_M_RANGE for M outside 1..4, LAQ_ERR_BITS for mixed or invalid bits,
+ * LAQ_ERR_WORKSPACE for a bad workspace, and the per-entry statuses of laq_gemm_wxg128.
+ */
+laq_status laq_gemm_chain(const laq_gemv *gemvs, int32_t count, void *workspace,
+                          size_t workspace_bytes, void *stream);
 
 #ifdef __cplusplus
 }

@@ -14,11 +14,13 @@ LIB_PATH = os.path.join(PKG, "liblaq.so")
 
 STATUS = {0: "LAQ_OK", 1: "LAQ_ERR_NULL", 2: "LAQ_ERR_BITS", 3: "LAQ_ERR_GROUP",
           4: "LAQ_ERR_SHAPE", 5: "LAQ_ERR_ALIGN", 6: "LAQ_ERR_M_RANGE", 7: "LAQ_ERR_CUDA",
-          8: "LAQ_ERR_TIMEOUT", 9: "LAQ_ERR_CONFIG"}
+          8: "LAQ_ERR_TIMEOUT", 9: "LAQ_ERR_CONFIG", 10: "LAQ_ERR_WORKSPACE"}
 
 # Symbols include/laq.h declares.
 EXPORTS = ("laq_status_str", "laq_version", "laq_packed_bytes", "laq_quantize_rtn", "laq_pack",
-           "laq_unpack", "laq_gemm_wxg128", "laq_gemm_plan", "laq_gemm_wxg128_config")
+           "laq_unpack", "laq_gemm_wxg128", "laq_gemm_plan", "laq_gemm_wxg128_config",
+           "laq_chain_workspace_bytes", "laq_gemm_chain")
+CHAIN_MAX = 384  # LAQ_CHAIN_MAX
 
 
 class LaqError(RuntimeError):
@@ -41,6 +43,14 @@ class GemmConfig(ctypes.Structure):
         return cls(tiles_per_cta, warps, cluster, stages, pdl, (ctypes.c_int32 * 3)(0, 0, 0))
 
 
+class Gemv(ctypes.Structure):
+    """struct laq_gemv: one entry of a laq_gemm_chain call."""
+    _fields_ = [("X", ctypes.c_void_p), ("packed", ctypes.c_void_p), ("s", ctypes.c_void_p),
+                ("z", ctypes.c_void_p), ("Y", ctypes.c_void_p), ("M", ctypes.c_int64),
+                ("K", ctypes.c_int64), ("N", ctypes.c_int64), ("bits", ctypes.c_int32),
+                ("wait_prev", ctypes.c_int32)]
+
+
 @functools.lru_cache(maxsize=1)
 def lib():
     if not os.path.exists(LIB_PATH):
@@ -61,8 +71,11 @@ def lib():
     L.laq_gemm_plan.argtypes = [I64, I64, I64, I, I, ctypes.POINTER(GemmConfig)]
     L.laq_gemm_wxg128_config.argtypes = [P, I64, I64, I64, P, P, P, I, P,
                                          ctypes.POINTER(GemmConfig), P]
+    L.laq_chain_workspace_bytes.argtypes = [ctypes.c_int32]
+    L.laq_chain_workspace_bytes.restype = ctypes.c_size_t
+    L.laq_gemm_chain.argtypes = [ctypes.POINTER(Gemv), ctypes.c_int32, P, ctypes.c_size_t, P]
     for name in ("laq_quantize_rtn", "laq_pack", "laq_unpack", "laq_gemm_wxg128",
-                 "laq_gemm_plan", "laq_gemm_wxg128_config"):
+                 "laq_gemm_plan", "laq_gemm_wxg128_config", "laq_gemm_chain"):
         getattr(L, name).restype = I
     return L
 
@@ -138,3 +151,49 @@ def laq_gemm_plan(M, K, N, bits, num_sms):
     cfg = GemmConfig()
     _check(lib().laq_gemm_plan(M, K, N, bits, num_sms, ctypes.byref(cfg)), "laq_gemm_plan")
     return cfg
+
+
+def laq_chain_workspace_bytes(count):
+    return int(lib().laq_chain_workspace_bytes(count))
+
+
+def chain_workspace(count, device):
+    """A zero-filled workspace for chains of up to ``count`` entries."""
+    import torch
+    n = laq_chain_workspace_bytes(count)
+    if n == 0:
+        raise ValueError(f"chain length {count} outside 0..{CHAIN_MAX}")
+    return torch.zeros((n,), dtype=torch.uint8, device=device)
+
+
+class Chain:
+    """A fixed list of GEMVs for laq_gemm_chain: entries are (X, packed, s, z, bits, Y,
+    wait_prev) with device tensors, kept alive here so the call can be replayed (or captured)."""
+
+    def __init__(self, entries):
+        self.tensors = []
+        self.array = (Gemv * max(1, len(entries)))()
+        for i, (X, packed, s, z, bits, Y, wait_prev) in enumerate(entries):
+            M, K = X.shape
+            N = s.shape[1]
+            self.array[i] = Gemv(X.data_ptr(), packed.data_ptr(), s.data_ptr(), z.data_ptr(),
+                                 Y.data_ptr(), M, K, N, bits, 1 if wait_prev else 0)
+            self.tensors.append((X, packed, s, z, Y))
+        self.count = len(entries)
+
+    def run(self, workspace, stream=None):
+        ws = workspace
+        _check(lib().laq_gemm_chain(self.array, self.count, _ptr(ws), ws.numel(),
+                                    _stream(stream)), "laq_gemm_chain")
+
+
+def laq_gemm_chain(entries, workspace, stream=None):
+    """Run ``entries`` (see ``Chain``) as one persistent launch on ``stream``."""
+    Chain(entries).run(workspace, stream)
+
+
+def chain_status(workspace):
+    """The device-side status word of a chain workspace (synchronizes the device)."""
+    import torch
+    torch.cuda.synchronize(workspace.device)
+    return int(workspace[:4].view(torch.int32)[0].item())

@@ -4,6 +4,7 @@
 #include <stdint.h>
 
 #include <atomic>
+#include <vector>
 
 #include "laq.h"
 #include "laq_internal.cuh"
@@ -183,6 +184,95 @@ laq_status run_gemm(const void* X, int64_t M, int64_t K, int64_t N, const void* 
     return from_cuda(laq::launch_gemm(L, f.smem_optin, strm));
 }
 
+
+// ---- laq_gemm_chain -------------------------------------------------------------------------
+
+constexpr int kChainMaxM = 4;
+constexpr int kChainWarps = 16;  // warps per CTA of the chain kernel
+
+size_t chain_ws_bytes(int32_t count) {
+    // status, finished-CTA counter, one arrival counter per stage (at most one per entry)
+    const size_t words = 2 + (size_t)count;
+    return (words * 4 + 255) / 256 * 256;
+}
+
+laq_status run_chain(const laq_gemv* g, int32_t count, void* workspace, size_t workspace_bytes,
+                     void* stream) {
+    if (count < 0 || count > LAQ_CHAIN_MAX) return LAQ_ERR_SHAPE;
+    if (count == 0) return LAQ_OK;
+    if (!g) return LAQ_ERR_NULL;
+    if (!workspace || !aligned(workspace, 16) || workspace_bytes < chain_ws_bytes(count))
+        return LAQ_ERR_WORKSPACE;
+    const int bits = g[0].bits;
+    laq_status st = check_bits(bits);
+    if (st != LAQ_OK) return st;
+    const int64_t M = g[0].M;
+    if (M < 1 || M > kChainMaxM) return LAQ_ERR_M_RANGE;
+    std::vector<laq::ChainEntry> ents((size_t)count);
+    std::vector<laq::ChainStage> stages((size_t)count);
+    int nst = 0;
+    int64_t xs_need = 0, stage_x = 0, stage_units = 0;
+    for (int32_t i = 0; i < count; ++i) {
+        const laq_gemv& e = g[i];
+        if (e.bits != bits) return LAQ_ERR_BITS;
+        if (e.M != M) return LAQ_ERR_M_RANGE;
+        st = check_kn(e.K, e.N, true);
+        if (st != LAQ_OK) return st;
+        if (e.K == 0 || e.N == 0) return LAQ_ERR_SHAPE;
+        if (e.K * M * 2 > (int64_t)1 << 30 || e.N / 16 > (int64_t)1 << 24) return LAQ_ERR_SHAPE;
+        if (!e.X || !e.packed || !e.s || !e.z || !e.Y) return LAQ_ERR_NULL;
+        if (!aligned(e.X, 16) || !aligned(e.packed, 16) || !aligned(e.s, 16) ||
+            !aligned(e.z, 16) || !aligned(e.Y, 16))
+            return LAQ_ERR_ALIGN;
+        if (i == 0 || e.wait_prev != 0) {
+            if (i > 0) stages[nst - 1].units = (int)stage_units;
+            stages[nst] = laq::ChainStage{i, 0, 0};
+            ++nst;
+            stage_x = 0;
+            stage_units = 0;
+        }
+        laq::ChainStage& cs = stages[nst - 1];
+        laq::ChainEntry& ce = ents[i];
+        ce.X = static_cast<const uint16_t*>(e.X);
+        ce.packed = static_cast<const uint8_t*>(e.packed);
+        ce.s = static_cast<const uint16_t*>(e.s);
+        ce.z = e.z;
+        ce.Y = static_cast<uint16_t*>(e.Y);
+        ce.K = (int)e.K;
+        ce.N = (int)e.N;
+        ce.xoff = (int)(stage_x / 16);
+        stage_x += M * e.K * 2;
+        stage_units += e.N / 16;
+        if (stage_units > ((int64_t)1 << 30)) return LAQ_ERR_SHAPE;
+        ++cs.ne;
+        if (stage_x > xs_need) xs_need = stage_x;
+    }
+    stages[nst - 1].units = (int)stage_units;
+
+    DeviceFacts f;
+    st = device_facts(&f);
+    if (st != LAQ_OK) return st;
+    const size_t slot = (size_t)(bits == 4 ? 1024 : 768) + 48;
+    // ring depth: slots for one block of 8 / M-class records plus at least one in flight
+    const int gpa = M <= 1 ? 8 : M <= 2 ? 4 : 2;
+    const size_t fixed = laq::chain_smem_bytes(bits, (int)M, 0, (int)xs_need, nst);
+    if (fixed + (size_t)kChainWarps * (gpa + 1) * slot > f.smem_optin) return LAQ_ERR_SHAPE;
+    int ring = (int)((f.smem_optin - fixed) / ((size_t)kChainWarps * slot));
+    if (ring > 16) ring = 16;
+
+    laq::ChainLaunch L;
+    L.e = ents.data();
+    L.st = stages.data();
+    L.count = count;
+    L.nstages = nst;
+    L.M = (int)M;
+    L.bits = bits;
+    L.stages = ring;
+    L.xs_bytes = (int)xs_need;
+    L.ws = static_cast<uint32_t*>(workspace);
+    return from_cuda(laq::launch_chain(L, f.sms, static_cast<cudaStream_t>(stream)));
+}
+
 }  // namespace
 
 extern "C" {
@@ -195,10 +285,11 @@ const char* laq_status_str(int status) {
         case LAQ_ERR_GROUP: return "LAQ_ERR_GROUP: group size must be 128";
         case LAQ_ERR_SHAPE: return "LAQ_ERR_SHAPE: unsupported K or N";
         case LAQ_ERR_ALIGN: return "LAQ_ERR_ALIGN: misaligned pointer";
-        case LAQ_ERR_M_RANGE: return "LAQ_ERR_M_RANGE: M must be in 0..16";
+        case LAQ_ERR_M_RANGE: return "LAQ_ERR_M_RANGE: M outside the supported range";
         case LAQ_ERR_CUDA: return "LAQ_ERR_CUDA: CUDA runtime error";
         case LAQ_ERR_TIMEOUT: return "LAQ_ERR_TIMEOUT: a device-side wait gave up";
         case LAQ_ERR_CONFIG: return "LAQ_ERR_CONFIG: unsupported launch configuration";
+        case LAQ_ERR_WORKSPACE: return "LAQ_ERR_WORKSPACE: workspace missing, misaligned or too small";
         default: return "unknown laq status";
     }
 }
@@ -274,6 +365,16 @@ laq_status laq_gemm_wxg128_config(const void* X, int64_t M, int64_t K, int64_t N
                                   void* Y, const laq_gemm_config* cfg, void* stream) {
     if (!cfg) return LAQ_ERR_NULL;
     return run_gemm(X, M, K, N, packed, s, z, bits, Y, cfg, stream);
+}
+
+size_t laq_chain_workspace_bytes(int32_t count) {
+    if (count < 0 || count > LAQ_CHAIN_MAX) return 0;
+    return chain_ws_bytes(count);
+}
+
+laq_status laq_gemm_chain(const laq_gemv* gemvs, int32_t count, void* workspace,
+                          size_t workspace_bytes, void* stream) {
+    return run_chain(gemvs, count, workspace, workspace_bytes, stream);
 }
 
 }  // extern "C"

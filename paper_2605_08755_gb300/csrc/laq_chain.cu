@@ -1,0 +1,701 @@
+// laq_chain.cu -- a chain of WbG128 GEMVs (Eq. (1) weights, M = 1..4) in one persistent launch.
+//
+// A decode step multiplies the step's activations by every projection of every layer, in an
+// order fixed by the model: q, k and v read the same input; o reads the attention output; gate
+// and up read the same input; down reads their product.  Launched one kernel per projection,
+// every GEMV pays a launch, a prologue that waits for its input, and a drain at the end, and
+// the weight stream stops at each boundary.  This kernel runs the whole chain instead:
+//
+//  * One CTA of 16 warps per SM, all resident at once (cooperative launch).  The chain is cut
+//    into stages at the entries that wait for their predecessors.  The units (16-column tiles)
+//    of a stage are split into equal contiguous ranges, one per CTA, and the CTA's records
+//    (tile x group of 128 rows) into 16 contiguous shares that differ by at most one record.
+//
+//  * Each warp streams its records, across all stages, through a private cp.async ring of
+//    `stages` slots (the packed codes plus the record's 16 scales and zeros).  Weights never
+//    depend on activations, so the ring runs ahead across stage boundaries: while a stage
+//    waits for its input, the next stages' weights are landing.
+//
+//  * Stage boundary: every CTA bumps the stage's arrival counter in global memory after its Y
+//    stores (release); a CTA with work in the next stage waits until the counter reaches the
+//    grid size (acquire), then stages X in shared memory and runs its records.  Waits are
+//    bounded: after about a second the kernel records LAQ_ERR_TIMEOUT in the workspace and
+//    every CTA returns.
+//
+//  * The record arithmetic is that of laq_gemm.cu: one LOP3 per pair of codes gives the fp16
+//    values c + q, an m16n8k16 MMA contracts them with raw x into D.  Per block of groups that
+//    share the accumulator, one more MMA per k16 step, whose A rows 0-7 hold the offsets c_k
+//    and rows 8-15 hold 1, gives P_g = sum_k c_k x_k and S_g = sum_k x_k in the layout of D,
+//    and the epilogue applies Eq. (1) as y += s * (D - P - z S).  A tile whose groups are split
+//    between warps is summed in shared memory at the end of the stage in warp order
+//    (deterministic, no atomics on Y).
+//
+//  * The last CTA to finish resets the counters, so the workspace is zero again for the next
+//    call on the stream.
+#include <cuda_fp16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <atomic>
+#include <memory>
+
+#include "laq.h"
+#include "laq_device.cuh"
+#include "laq_internal.cuh"
+
+// Compile-time trace points of thread 0 per stage (empty in the library build; a tracing build
+// defines LAQ_CHAIN_TRACE(stage, point) to timestamp them).
+#ifndef LAQ_CHAIN_TRACE
+#define LAQ_CHAIN_TRACE(stage, point) \
+    do {                              \
+    } while (0)
+#endif
+
+namespace laq {
+
+namespace {
+
+constexpr int kChainWarps = 16;
+constexpr int kChainThreads = kChainWarps * 32;
+constexpr int kSzBytes = 48;                          // 16 fp16 scales + 16 u8 zeros
+constexpr unsigned long long kWaitNs = 1000000000ull; // stage wait limit (1 s)
+constexpr int kWaitSpins = 1 << 24;                   // and an iteration limit besides
+
+struct ChainEntryDev {
+    const uint16_t* X;
+    const uint8_t* packed;
+    const uint16_t* s;
+    const uint8_t* z;
+    uint16_t* Y;
+    int K, N;
+    int xoff;   // offset of this entry's X in the stage's shared X area (16-byte units)
+};
+
+struct ChainStageDev {
+    int e0, ne;  // entries [e0, e0 + ne)
+    int units;   // 16-column tiles of the stage
+};
+
+struct ChainParams {
+    ChainEntryDev e[kChainMax];
+    ChainStageDev st[kChainMax];
+    uint32_t* ws;  // [0] status, [1] finished CTAs, [2 + s] CTAs done with stage s
+    int count, nstages, M, stages, xs_bytes;
+    Exps exps;
+};
+static_assert(sizeof(ChainParams) <= 32000, "kernel parameters must stay below 32 KB");
+
+template <int BITS>
+struct Slot {
+    static constexpr int kRec = RecordFmt<BITS>::kBytes;
+    static constexpr int kBytes = kRec + kSzBytes;  // 816 (b = 3) or 1072 (b = 4), 16-aligned
+};
+
+__device__ __forceinline__ unsigned long long globaltimer() {
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+__device__ __forceinline__ uint32_t ld_acquire(const uint32_t* p) {
+    uint32_t v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+__device__ __forceinline__ uint32_t ld_relaxed(const uint32_t* p) {
+    uint32_t v;
+    asm volatile("ld.relaxed.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+__device__ __forceinline__ uint4 ld_cg16(const void* p) {
+    uint4 v;
+    asm volatile("ld.global.cg.v4.u32 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "l"(p)
+                 : "memory");
+    return v;
+}
+
+// Wait until *cnt >= target.  Returns false when an error is already recorded in the status
+// word (checked first, so a recorded error stops every later stage), or when the wait runs out
+// (after recording LAQ_ERR_TIMEOUT).
+__device__ bool wait_count(const uint32_t* cnt, uint32_t target, uint32_t* status) {
+    const unsigned long long t0 = globaltimer();
+    for (int spin = 0; spin < kWaitSpins; ++spin) {
+        if (ld_relaxed(status) != 0u) return false;
+        if (ld_acquire(cnt) >= target) return true;
+        if ((spin & 31) == 31 && globaltimer() - t0 > kWaitNs) break;
+    }
+    atomicCAS(status, 0u, (uint32_t)LAQ_ERR_TIMEOUT);
+    return false;
+}
+
+// The CTA's contiguous unit range of a stage with `units` units (64-bit products: computed once
+// per stage at kernel start, not per use).
+__device__ __forceinline__ int2 cta_units(int units) {
+    const long long P = gridDim.x, b = blockIdx.x;
+    return make_int2((int)(units * b / P), (int)(units * (b + 1) / P));
+}
+
+// A warp's position in its record stream: stage s, entry e, tile (16-column block of the entry)
+// and group g.  Within a stage the CTA's records are its units in order, each unit's groups in
+// order; warp w takes the contiguous share [n w / 16, n (w + 1) / 16) of the CTA's n records,
+// so the warps of a CTA differ by at most one record.
+struct Cursor {
+    int s;        // stage
+    int left;     // records of the share from the current one to its end
+    int e;        // entry
+    int tile;     // tile within the entry
+    int g;        // group within the tile
+    int G;        // groups of the entry
+    int tile_hi;  // end of the CTA's tiles of this entry
+    int ubase;    // first unit of entry e within the stage
+};
+
+// Place the cursor at the first record of warp w's share of stage c.s; false if it is empty.
+__device__ bool cursor_begin(Cursor& c, const ChainParams& p, const int4* range, int w) {
+    const int4 rg = range[c.s];  // first unit, end unit, records of this CTA
+    const int r0 = (rg.z * w) >> 4, r1 = (rg.z * (w + 1)) >> 4;
+    c.left = r1 - r0;
+    if (c.left <= 0) return false;
+    int r = r0;
+    const ChainStageDev st = p.st[c.s];
+    int ubase = 0;
+    for (int q = 0; q < st.ne; ++q) {
+        const int e = st.e0 + q;
+        const int T = p.e[e].N >> 4, G = p.e[e].K >> 7;
+        const int lo = max(rg.x, ubase), hi = min(rg.y, ubase + T);
+        if (hi > lo) {
+            const int cnt = (hi - lo) * G;
+            if (r < cnt) {
+                const int t = r / G;
+                c.e = e;
+                c.G = G;
+                c.ubase = ubase;
+                c.tile = lo - ubase + t;
+                c.g = r - t * G;
+                c.tile_hi = hi - ubase;
+                return true;
+            }
+            r -= cnt;
+        }
+        ubase += T;
+    }
+    c.left = 0;  // not reached: r0 < n
+    return false;
+}
+
+// Step to the next record of the share (the caller has checked left > 1): 0 within the tile,
+// 1 to the first group of the next tile of the entry, 2 to the first record of a new entry.
+__device__ int cursor_step(Cursor& c, const ChainParams& p, const int4* range) {
+    --c.left;
+    if (++c.g < c.G) return 0;
+    c.g = 0;
+    if (++c.tile < c.tile_hi) return 1;
+    const int4 rg = range[c.s];
+    const ChainStageDev st = p.st[c.s];
+    int ubase = c.ubase + (p.e[c.e].N >> 4);
+    for (int e = c.e + 1; e < st.e0 + st.ne; ++e) {
+        const int T = p.e[e].N >> 4;
+        const int lo = max(rg.x, ubase), hi = min(rg.y, ubase + T);
+        if (hi > lo) {
+            c.e = e;
+            c.G = p.e[e].K >> 7;
+            c.ubase = ubase;
+            c.tile = lo - ubase;
+            c.tile_hi = hi - ubase;
+            return 2;
+        }
+        ubase += T;
+    }
+    return 2;  // not reached while left > 0
+}
+
+// Move to the first group of the next tile of the share (the caller has checked that records
+// remain): true if the entry changed.
+__device__ bool cursor_next_tile(Cursor& c, const ChainParams& p, const int4* range) {
+    c.g = 0;
+    if (++c.tile < c.tile_hi) return false;
+    const int4 rg = range[c.s];
+    const ChainStageDev st = p.st[c.s];
+    int ubase = c.ubase + (p.e[c.e].N >> 4);
+    for (int e = c.e + 1; e < st.e0 + st.ne; ++e) {
+        const int T = p.e[e].N >> 4;
+        const int lo = max(rg.x, ubase), hi = min(rg.y, ubase + T);
+        if (hi > lo) {
+            c.e = e;
+            c.G = p.e[e].K >> 7;
+            c.ubase = ubase;
+            c.tile = lo - ubase;
+            c.tile_hi = hi - ubase;
+            return true;
+        }
+        ubase += T;
+    }
+    return true;  // not reached while records remain
+}
+
+// The warp's record stream on the copy side of the ring (the compute side walks the same
+// shares).  A slot holds the record's packed words followed by its 16 scales and 16 zeros;
+// each lane copies 16-byte pieces of it from per-lane source pointers:
+//   b = 3: piece l (record bytes 16 l), then piece 32 + l for l < 19 (record bytes 512 + 16 l
+//          for l < 16, the scales for l = 16, 17, the zeros for l = 18);
+//   b = 4: pieces l and 32 + l (record bytes 16 l and 512 + 16 l), then for l < 3 the scales
+//          (l = 0, 1) or the zeros (l = 2).
+template <int BITS>
+struct RecordStream {
+    static constexpr int REC = RecordFmt<BITS>::kBytes;
+    Cursor c;
+    bool live;
+    const uint8_t* p1;
+    const uint8_t* p2;
+    const uint8_t* p3;
+    long long st2, st3;  // bytes to the next group's piece (p1 always moves by REC)
+
+    __device__ void point(const ChainParams& p, int lane) {
+        const ChainEntryDev& E = p.e[c.e];
+        const uint8_t* rec = E.packed + ((size_t)c.tile * c.G + c.g) * REC;
+        const size_t gz = (size_t)c.g * E.N + (size_t)c.tile * 16;  // (group, column)
+        const uint8_t* sp = reinterpret_cast<const uint8_t*>(E.s + gz);
+        const uint8_t* zp = E.z + gz;
+        p1 = rec + lane * 16;
+        if (BITS == 3) {
+            p2 = lane < 16 ? rec + 512 + lane * 16 : lane < 18 ? sp + (lane - 16) * 16 : zp;
+            st2 = lane < 16 ? REC : lane < 18 ? 2LL * E.N : (long long)E.N;
+            p3 = p2;
+            st3 = 0;
+        } else {
+            p2 = rec + 512 + lane * 16;
+            st2 = REC;
+            p3 = lane < 2 ? sp + lane * 16 : zp;
+            st3 = lane < 2 ? 2LL * E.N : (long long)E.N;
+        }
+    }
+    __device__ void seek(const ChainParams& p, const int4* range, int w, int lane) {
+        while (c.s < p.nstages && !cursor_begin(c, p, range, w)) ++c.s;
+        live = c.s < p.nstages;
+        if (live) point(p, lane);
+    }
+    __device__ void advance(const ChainParams& p, const int4* range, int w, int lane) {
+        if (c.left > 1) {
+            if (cursor_step(c, p, range) == 0) {
+                p1 += REC;
+                p2 += st2;
+                p3 += st3;
+            } else {
+                point(p, lane);
+            }
+        } else {
+            ++c.s;
+            seek(p, range, w, lane);
+        }
+    }
+};
+
+// A fragment of the (S, P) contraction for k16 step j: rows 0-7 hold the offsets c_k of the
+// step's pairs (the fp16 value of code 0 in each field: its exponent constant), rows 8-15
+// hold 1, so one more MMA per step sums P_g = sum_k c_k x_k and S_g = sum_k x_k per column.
+template <int BITS>
+__device__ __forceinline__ uint32_t ps_offset(const Exps& x, int j, int h) {
+    const int i = 2 * j + h;  // pair index
+    if (BITS == 4) return h == 0 ? x.e[0] : x.e[1];
+    return i < 6 ? x.e[0] : (i < 12 ? x.e[1] : (i < 15 ? x.e[2] : x.e[1]));
+}
+
+template <int BITS, int MP>
+__global__ void __launch_bounds__(kChainThreads, 1) chain_kernel(const __grid_constant__ ChainParams p) {
+    using F = RecordFmt<BITS>;
+    constexpr int SLOT = Slot<BITS>::kBytes;
+    constexpr int WPL = BITS == 4 ? 8 : 6;
+    constexpr int GPA = 8 / MP;  // groups sharing one accumulator (MMA columns), MP <= 4
+    constexpr uint32_t kOnes = 0x3c003c00u;
+
+    extern __shared__ __align__(128) uint8_t smem[];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int c = lane & 3, R = lane >> 2;
+    const int M = p.M, S = p.stages;
+    uint32_t* status = p.ws;
+
+    // shared memory: ring [16][S][slot] | X [xs_bytes] | zero block (64 B)
+    //                | split-tile partial sums [32][MP][16] fp32 | their tile keys [32]
+    //                | this CTA's (first unit, end unit, records) per stage [nstages] int4
+    //                | flag
+    uint8_t* ring = smem;
+    uint4* xs = reinterpret_cast<uint4*>(smem + (size_t)kChainWarps * S * SLOT);
+    uint4* zblk = xs + p.xs_bytes / 16;
+    float* red = reinterpret_cast<float*>(zblk + 4);
+    int* keys = reinterpret_cast<int*>(red + 2 * kChainWarps * MP * 16);
+    int4* range = reinterpret_cast<int4*>(keys + 2 * kChainWarps);
+    int* flag = reinterpret_cast<int*>(range + p.nstages);
+    if (threadIdx.x < 4) zblk[threadIdx.x] = make_uint4(0u, 0u, 0u, 0u);
+    for (int s = threadIdx.x; s < p.nstages; s += kChainThreads) {
+        const int2 u = cta_units(p.st[s].units);
+        // records of the CTA: its units of each entry times the entry's groups
+        int n = 0, ubase = 0;
+        const ChainStageDev st = p.st[s];
+        for (int q = 0; q < st.ne; ++q) {
+            const int T = p.e[st.e0 + q].N >> 4, G = p.e[st.e0 + q].K >> 7;
+            const int lo = max(u.x, ubase), hi = min(u.y, ubase + T);
+            if (hi > lo) n += (hi - lo) * G;
+            ubase += T;
+        }
+        range[s] = make_int4(u.x, u.y, n, 0);
+    }
+    __syncthreads();
+
+    const uint32_t ring_s = (uint32_t)__cvta_generic_to_shared(ring) +
+                            (uint32_t)(warp * S * SLOT);
+    const uint8_t* ring_w = ring + (size_t)warp * S * SLOT;
+
+    // Copy side of the ring: the next record of the warp's stream into the next slot (an
+    // empty group once the stream is exhausted, so group counting stays uniform).
+    RecordStream<BITS> is;
+    is.c.s = 0;
+    is.seek(p, range, warp, lane);
+    int islot = 0;
+    auto issue = [&]() {
+        if (is.live) {
+            const uint32_t dst = ring_s + (uint32_t)(islot * SLOT) + lane * 16;
+            cp_async16(dst, is.p1);
+            if (BITS == 3) {
+                if (lane < 19) cp_async16(dst + 512, is.p2);
+            } else {
+                cp_async16(dst + 512, is.p2);
+                if (lane < 3) cp_async16(dst + 1024, is.p3);
+            }
+            is.advance(p, range, warp, lane);
+        }
+        cp_async_commit();
+        islot = islot + 1 == S ? 0 : islot + 1;
+    };
+    // Records in flight ahead of the one being consumed: the slots of a block (GPA records)
+    // stay valid until its epilogue has read their scales and zeros.
+    const int ahead = S - GPA;
+    for (int q = 0; q < ahead; ++q) issue();
+    int rslot = 0;
+
+    const int bl = R / GPA;   // batch row of this lane's B column
+    const int gil = R % GPA;  // group position of this lane's B column
+    bool ok = true;
+
+    for (int s = 0; s < p.nstages; ++s) {
+        const ChainStageDev st = p.st[s];
+        const int u0 = range[s].x, u1 = range[s].y;
+        if (u1 <= u0) {
+            // Nothing of this stage here: report it done at once.
+            if (threadIdx.x == 0) {
+                __threadfence();
+                atomicAdd(p.ws + 2 + s, 1u);
+            }
+            continue;
+        }
+        LAQ_CHAIN_TRACE(s, 0);
+        if (threadIdx.x == 0) {
+            bool good = true;
+            if (s > 0) good = wait_count(p.ws + 2 + (s - 1), gridDim.x, status);
+            *flag = good ? 1 : 0;
+        }
+        if (threadIdx.x < 2 * kChainWarps) keys[threadIdx.x] = -1;
+        __syncthreads();  // the wait is over; every warp is done with the previous stage's X
+        LAQ_CHAIN_TRACE(s, 1);
+        if (*flag == 0) {
+            ok = false;
+            break;
+        }
+
+        // X of every entry of the stage that has a unit here (M rows of K fp16, contiguous),
+        // through L2 (ld.global.cg: written by other SMs during this kernel).
+        {
+            int ubase = 0;
+            for (int q = 0; q < st.ne; ++q) {
+                const ChainEntryDev& E = p.e[st.e0 + q];
+                const int T = E.N >> 4;
+                if (ubase < u1 && ubase + T > u0) {
+                    const int n16 = M * E.K / 8;
+                    const uint8_t* src = reinterpret_cast<const uint8_t*>(E.X);
+                    uint4* dst = xs + E.xoff;
+                    for (int u = threadIdx.x; u < n16; u += 4 * kChainThreads) {
+                        uint4 v[4];
+#pragma unroll
+                        for (int r = 0; r < 4; ++r) {
+                            const int uu = u + r * kChainThreads;
+                            if (uu < n16) v[r] = ld_cg16(src + (size_t)uu * 16);
+                        }
+#pragma unroll
+                        for (int r = 0; r < 4; ++r) {
+                            const int uu = u + r * kChainThreads;
+                            if (uu < n16) dst[uu] = v[r];
+                        }
+                    }
+                }
+                ubase += T;
+            }
+        }
+        __syncthreads();
+        LAQ_CHAIN_TRACE(s, 2);
+        LAQ_CHAIN_TRACE(s, 3);
+
+        // This warp's share of the stage, a block of up to GPA records (consecutive groups of
+        // one tile, sharing the accumulator columns) at a time.
+        Cursor cc;
+        cc.s = s;
+        if (cursor_begin(cc, p, range, warp)) {
+            int xoff = p.e[cc.e].xoff, G = cc.G;
+            int piece_g0 = cc.g;  // first group of the current piece (run of one tile)
+            bool first_piece = true;
+            float yacc[4] = {0.f, 0.f, 0.f, 0.f};
+            for (;;) {
+                const int gb = cc.g;  // first group of the block
+                const int nb = min(GPA, min(G - gb, cc.left));
+                const int rs0 = rslot;
+                float D[2][4];
+#pragma unroll
+                for (int a = 0; a < 2; ++a)
+#pragma unroll
+                    for (int v = 0; v < 4; ++v) D[a][v] = 0.f;
+#pragma unroll
+                for (int gi = 0; gi < GPA; ++gi) {
+                    if (gi < nb) {
+                        __syncwarp();  // every lane is done with the slot the next copy overwrites
+                        issue();
+                        cp_async_wait(ahead);
+                        uint32_t B[8][2];
+                        {
+                            const bool act = gil == gi && bl < M;
+                            const uint4* src =
+                                act ? xs + xoff + (size_t)(bl * G + gb + gi) * 16 + c * 4 : zblk;
+#pragma unroll
+                            for (int q = 0; q < 4; ++q) {
+                                const uint4 v = src[q];
+                                B[2 * q][0] = v.x;
+                                B[2 * q][1] = v.y;
+                                B[2 * q + 1][0] = v.z;
+                                B[2 * q + 1][1] = v.w;
+                            }
+                        }
+                        const uint8_t* slot = ring_w + (size_t)rslot * SLOT;
+                        uint32_t wd[WPL];
+                        const uint4 c0 = *reinterpret_cast<const uint4*>(slot + lane * 16);
+                        wd[0] = c0.x; wd[1] = c0.y; wd[2] = c0.z; wd[3] = c0.w;
+                        if constexpr (BITS == 4) {
+                            const uint4 c1 = *reinterpret_cast<const uint4*>(slot + 512 + lane * 16);
+                            wd[4] = c1.x; wd[5] = c1.y; wd[6] = c1.z; wd[7] = c1.w;
+                        } else {
+                            const uint2 c1 = *reinterpret_cast<const uint2*>(slot + 512 + lane * 8);
+                            wd[4] = c1.x; wd[5] = c1.y;
+                        }
+                        uint32_t a[8][4];
+                        extract<BITS>(wd, p.exps, a);
+#pragma unroll
+                        for (int j = 0; j < 8; ++j)
+                            mma16816(D[j & 1], a[j][0], a[j][1], a[j][2], a[j][3], B[j][0],
+                                     B[j][1]);
+                        rslot = rslot + 1 == S ? 0 : rslot + 1;
+                    }
+                }
+                __syncwarp();  // the scales and zeros of the block's slots came from other lanes
+
+                // S and P of the block's groups (columns), then Eq. (1): y += s (D - P - z S).
+                {
+                    float Q[4] = {0.f, 0.f, 0.f, 0.f};
+                    uint32_t B[8][2];
+                    const bool act = gil < nb && bl < M;
+                    const uint4* src = act ? xs + xoff + (size_t)(bl * G + gb + gil) * 16 + c * 4
+                                           : zblk;
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) {
+                        const uint4 v = src[q];
+                        B[2 * q][0] = v.x;
+                        B[2 * q][1] = v.y;
+                        B[2 * q + 1][0] = v.z;
+                        B[2 * q + 1][1] = v.w;
+                    }
+#pragma unroll
+                    for (int j = 0; j < 8; ++j)
+                        mma16816(Q, ps_offset<BITS>(p.exps, j, 0), kOnes,
+                                 ps_offset<BITS>(p.exps, j, 1), kOnes, B[j][0], B[j][1]);
+                    // value v of the lane: row R + 8 (v >> 1), column 2c + (v & 1) = record
+                    // (column % GPA) of the block for batch row column / GPA
+#pragma unroll
+                    for (int v1 = 0; v1 < 2; ++v1) {
+                        const int col = 2 * c + v1;
+                        const int b = col / GPA, rec = col % GPA;
+                        if (b < M && rec < nb) {
+                            int sl = rs0 + rec;
+                            sl = sl >= S ? sl - S : sl;
+                            const uint8_t* sz = ring_w + (size_t)sl * SLOT + F::kBytes;
+                            const uint16_t* ssl = reinterpret_cast<const uint16_t*>(sz);
+                            const float s0 = __half2float(__ushort_as_half(ssl[R]));
+                            const float s1 = __half2float(__ushort_as_half(ssl[R + 8]));
+                            const float z0 = (float)sz[32 + R], z1 = (float)sz[32 + R + 8];
+                            const float d0 = D[0][v1] + D[1][v1] - Q[v1];
+                            const float d1 = D[0][v1 + 2] + D[1][v1 + 2] - Q[v1];
+                            yacc[v1] = fmaf(s0, fmaf(-z0, Q[2 + v1], d0), yacc[v1]);
+                            yacc[v1 + 2] = fmaf(s1, fmaf(-z1, Q[2 + v1], d1), yacc[v1 + 2]);
+                        }
+                    }
+                }
+
+                cc.g += nb;
+                cc.left -= nb;
+                if (cc.g == G || cc.left == 0) {
+                    // End of a piece.  Columns of one batch row -> one value per (row, column).
+                    float y0 = yacc[0] + yacc[1];
+                    float y1 = yacc[2] + yacc[3];
+                    if (GPA >= 4) {
+                        y0 += __shfl_xor_sync(0xffffffffu, y0, 1);
+                        y1 += __shfl_xor_sync(0xffffffffu, y1, 1);
+                    }
+                    if (GPA >= 8) {
+                        y0 += __shfl_xor_sync(0xffffffffu, y0, 2);
+                        y1 += __shfl_xor_sync(0xffffffffu, y1, 2);
+                    }
+                    const int b = (2 * c) / GPA;
+                    const bool writer = (2 * c) % GPA == 0 && b < M;
+                    if (piece_g0 == 0 && cc.g == G) {
+                        // the whole tile: store
+                        if (writer) {
+                            const ChainEntryDev& E = p.e[cc.e];
+                            uint16_t* y = E.Y + (size_t)b * E.N + (size_t)cc.tile * 16;
+                            y[R] = __half_as_ushort(__float2half_rn(y0));
+                            y[R + 8] = __half_as_ushort(__float2half_rn(y1));
+                        }
+                    } else {
+                        // part of a tile shared with neighbouring warps: summed at stage end
+                        const int sl = 2 * warp + (first_piece ? 0 : 1);
+                        if (writer) {
+                            float* rw = red + (size_t)sl * MP * 16;
+                            rw[b * 16 + R] = y0;
+                            rw[b * 16 + R + 8] = y1;
+                        }
+                        if (lane == 0) keys[sl] = (cc.e << 20) | cc.tile;
+                    }
+#pragma unroll
+                    for (int v = 0; v < 4; ++v) yacc[v] = 0.f;
+                    first_piece = false;
+                    if (cc.left == 0) break;
+                    if (cursor_next_tile(cc, p, range)) {
+                        xoff = p.e[cc.e].xoff;
+                        G = cc.G;
+                    }
+                    piece_g0 = 0;
+                }
+            }
+        }
+        LAQ_CHAIN_TRACE(s, 4);
+        __syncthreads();  // partial sums of shared tiles are in red
+        LAQ_CHAIN_TRACE(s, 5);
+
+        // Tiles shared by several warps: sum their parts in slot (= warp) order and store.  Every
+        // warp sees the 32 slot keys, one per lane; slots with equal keys are one tile's parts.
+        {
+            const int kl = keys[lane];
+            const unsigned same = __match_any_sync(0xffffffffu, kl);
+            const int firstl = kl >= 0 && (same & ((1u << lane) - 1u)) == 0u;
+            for (int idx = threadIdx.x; idx < 2 * kChainWarps * M * 16; idx += kChainThreads) {
+                const int sl = idx / (M * 16), r = idx - sl * (M * 16);
+                const int key = __shfl_sync(0xffffffffu, kl, sl);
+                const int first = __shfl_sync(0xffffffffu, firstl, sl);
+                unsigned m = __shfl_sync(0xffffffffu, same, sl);
+                if (first) {
+                    float acc = 0.f;
+                    while (m) {
+                        const int j = __ffs(m) - 1;
+                        acc += red[(size_t)j * MP * 16 + r];
+                        m &= m - 1u;
+                    }
+                    const ChainEntryDev& E = p.e[key >> 20];
+                    const int tile = key & 0xfffff, b = r >> 4, n = r & 15;
+                    E.Y[(size_t)b * E.N + (size_t)tile * 16 + n] =
+                        __half_as_ushort(__float2half_rn(acc));
+                }
+            }
+        }
+        __syncthreads();  // every Y value of this CTA's units is stored
+        LAQ_CHAIN_TRACE(s, 7);
+        if (threadIdx.x == 0) {
+            __threadfence();
+            atomicAdd(p.ws + 2 + s, 1u);
+        }
+        LAQ_CHAIN_TRACE(s, 6);
+    }
+
+    asm volatile("cp.async.wait_all;\n" ::: "memory");
+    if (!ok) return;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        __threadfence();
+        const uint32_t prev = atomicAdd(p.ws + 1, 1u);
+        if (prev == gridDim.x - 1) {
+            // Every CTA is past its last wait: leave the counters at zero for the next call.
+            for (int s = 0; s < p.nstages; ++s) p.ws[2 + s] = 0u;
+            p.ws[1] = 0u;
+            __threadfence();
+        }
+    }
+}
+
+using ChainFn = void (*)(ChainParams);
+
+template <int BITS>
+ChainFn pick_chain(int mp) {
+    switch (mp) {
+        case 1: return chain_kernel<BITS, 1>;
+        case 2: return chain_kernel<BITS, 2>;
+        default: return chain_kernel<BITS, 4>;
+    }
+}
+
+std::atomic<size_t> g_chain_attr[2][3];  // dynamic shared memory already granted per instance
+
+}  // namespace
+
+size_t chain_smem_bytes(int bits, int M, int stages, int xs_bytes, int nstages) {
+    const int mp = M <= 1 ? 1 : M <= 2 ? 2 : 4;
+    const size_t slot = (size_t)(bits == 4 ? 1024 : 768) + kSzBytes;
+    return (size_t)kChainWarps * stages * slot + (size_t)xs_bytes + 64 +
+           (size_t)2 * kChainWarps * mp * 16 * 4 + (size_t)2 * kChainWarps * 4 +
+           (size_t)nstages * 16 + 16;
+}
+
+cudaError_t launch_chain(const ChainLaunch& L, int num_sms, cudaStream_t stream) {
+    // The parameter block is large (about 26 KB): built on the heap, copied by the launch.
+    std::unique_ptr<ChainParams> holder(new ChainParams());
+    ChainParams& P = *holder;
+    for (int i = 0; i < L.count; ++i) {
+        const ChainEntry& E = L.e[i];
+        P.e[i] = ChainEntryDev{E.X, E.packed, E.s, E.z, E.Y, E.K, E.N, E.xoff};
+    }
+    for (int s = 0; s < L.nstages; ++s) P.st[s] = ChainStageDev{L.st[s].e0, L.st[s].ne, L.st[s].units};
+    P.ws = L.ws;
+    P.count = L.count;
+    P.nstages = L.nstages;
+    P.M = L.M;
+    P.stages = L.stages;
+    P.xs_bytes = L.xs_bytes;
+    P.exps = exps_for(L.bits);
+
+    const int mp = L.M <= 1 ? 1 : L.M <= 2 ? 2 : 4;
+    const ChainFn fn = L.bits == 4 ? pick_chain<4>(mp) : pick_chain<3>(mp);
+    const size_t smem = chain_smem_bytes(L.bits, L.M, L.stages, L.xs_bytes, L.nstages);
+    std::atomic<size_t>& granted = g_chain_attr[L.bits == 4][mp == 1 ? 0 : mp == 2 ? 1 : 2];
+    cudaError_t err = cudaSuccess;
+    if (granted.load() < smem) {
+        err = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (err != cudaSuccess) return err;
+        granted.store(smem);
+    }
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)num_sms);
+    cfg.blockDim = dim3(kChainThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeCooperative;
+    attr[0].val.cooperative = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    void* args[] = {&P};
+    return cudaLaunchKernelExC(&cfg, (const void*)fn, args);
+}
+
+}  // namespace laq

@@ -28,4 +28,28 @@ struct GemmLaunch {
 size_t gemm_smem_bytes(const GemmLaunch& L, int* groups_per_phase);
 cudaError_t launch_gemm(const GemmLaunch& L, size_t smem_limit, cudaStream_t stream);
 
+// One persistent launch of a GEMV chain, fully resolved on the host.
+constexpr int kChainMax = 384;  // = LAQ_CHAIN_MAX
+struct ChainEntry {
+    const uint16_t* X;
+    const uint8_t* packed;
+    const uint16_t* s;
+    const uint8_t* z;
+    uint16_t* Y;
+    int K, N;
+    int xoff;  // X offset in the stage's shared X area, 16-byte units
+};
+struct ChainStage {
+    int e0, ne, units;
+};
+struct ChainLaunch {
+    const ChainEntry* e;
+    const ChainStage* st;
+    int count, nstages, M, bits, stages, xs_bytes;
+    uint32_t* ws;
+};
+// Dynamic shared memory of the chain kernel for a ring of `stages` slots per warp.
+size_t chain_smem_bytes(int bits, int M, int stages, int xs_bytes, int nstages);
+cudaError_t launch_chain(const ChainLaunch& L, int num_sms, cudaStream_t stream);
+
 }  // namespace laq

@@ -38,6 +38,8 @@ def shapes(model):
 
 # Projections that read the same activation and may run as one GEMV over concatenated columns.
 FUSED = (("qkv", ("q", "k", "v")), ("o", ("o",)), ("gate_up", ("gate", "up")), ("down", ("down",)))
+# Projections whose input is the previous projection's input (they need nothing new).
+SHARES_INPUT = {"k", "v", "up"}
 
 
 class WeightPass:
@@ -46,12 +48,17 @@ class WeightPass:
     With ``fuse``, q|k|v and gate|up (which share their input in a decoder) are quantized as one
     weight over concatenated output columns and run as one GEMV each (4 launches per layer);
     quantization is per column, so their codes, scales and zeros are those of the separate
-    projections."""
+    projections.
+
+    With ``chain``, the whole pass is one ``laq_gemm_chain`` launch (M <= 4) whose stages follow
+    the decoder's data flow: an entry waits for every earlier one unless it reads the input of
+    the projection before it (k and v after q, up after gate), so each layer has the four
+    dependency points q|k|v -> o -> gate|up -> down -> next layer."""
 
     def __init__(self, model="qwen3-4b", bits=3, M=1, layers=inputs.LAYERS, seed=0,
-                 outliers=False, device="cuda", pdl=True, fuse=False):
+                 outliers=False, device="cuda", pdl=True, fuse=False, chain=False):
         self.model, self.bits, self.M, self.layers = model, bits, M, layers
-        self.seed, self.outliers, self.fuse = seed, outliers, fuse
+        self.seed, self.outliers, self.fuse, self.chain = seed, outliers, fuse, chain
         self.device = torch.device(device)
         names = [n for n, _, _ in shapes(model)]
         groups = ([[names.index(m) for m in members] for _, members in FUSED] if fuse
@@ -89,6 +96,13 @@ class WeightPass:
             c = _lib.laq_gemm_plan(M, q.K, q.N, bits, sms)
             c.pdl = 1 if pdl else 0
             self.configs.append(c)
+        if chain:
+            entries = []
+            for i, (_, members, name, q) in enumerate(self.linears):
+                wait = not (name in SHARES_INPUT and i > 0)
+                entries.append((self.X[i], q.packed, q.s, q.z, bits, self.Y[i], wait))
+            self.chain_spec = _lib.Chain(entries)
+            self.ws = _lib.chain_workspace(len(entries), self.device)
         torch.cuda.synchronize(self.device)
 
     def weight(self, layer, members):
@@ -105,7 +119,7 @@ class WeightPass:
 
     @property
     def launches(self):
-        return len(self.linears)
+        return 1 if self.chain else len(self.linears)
 
     def bytes_per_pass(self):
         return sum(q.bytes_per_call(self.M) for *_, q in self.linears)
@@ -116,6 +130,13 @@ class WeightPass:
     def run(self, stream=None, events=None):
         """Launch the pass; with ``events`` (launches + 1 CUDA events) record one before each
         launch and one after the last."""
+        if self.chain:
+            if events is not None:
+                events[0].record(stream)
+            self.chain_spec.run(self.ws, stream)
+            if events is not None:
+                events[-1].record(stream)
+            return
         for i, (*_, q) in enumerate(self.linears):
             if events is not None:
                 events[i].record(stream)

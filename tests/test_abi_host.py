@@ -146,3 +146,47 @@ def test_plan_rejects_bad_arguments(L):
     assert L.laq_gemm_plan(1, 256, 32, 3, 152, None) == 1
     assert L.laq_gemm_plan(20, 256, 32, 3, 152, ctypes.byref(cfg)) == 6
     assert L.laq_gemm_plan(1, 250, 32, 3, 152, ctypes.byref(cfg)) == 4
+
+
+def chain_entry(X=FAKE, packed=FAKE, s=FAKE, z=FAKE, Y=FAKE, M=1, K=256, N=32, bits=3, wait=1):
+    return _lib.Gemv(X.value, packed.value, s.value, z.value, Y.value, M, K, N, bits, wait)
+
+
+def chain(L, entries, ws=FAKE, ws_bytes=None, count=None):
+    arr = (_lib.Gemv * max(1, len(entries)))(*entries)
+    n = len(entries) if count is None else count
+    if ws_bytes is None:
+        ws_bytes = max(L.laq_chain_workspace_bytes(max(0, min(n, _lib.CHAIN_MAX))), 256)
+    return L.laq_gemm_chain(arr, n, ws, ws_bytes, None)
+
+
+def test_chain_workspace_bytes(L):
+    assert L.laq_chain_workspace_bytes(0) == 256
+    assert L.laq_chain_workspace_bytes(252) == 1024            # 4 * (2 + 252) rounded to 256
+    assert L.laq_chain_workspace_bytes(_lib.CHAIN_MAX) >= 4 * (2 + _lib.CHAIN_MAX)
+    assert L.laq_chain_workspace_bytes(_lib.CHAIN_MAX + 1) == 0
+    assert L.laq_chain_workspace_bytes(-1) == 0
+
+
+def test_chain_argument_validation(L):
+    S = _lib.STATUS
+    code = {v: k for k, v in S.items()}
+    ok = chain_entry()
+    assert chain(L, []) == 0                                         # nothing to do
+    assert chain(L, [ok], count=_lib.CHAIN_MAX + 1) == code["LAQ_ERR_SHAPE"]
+    assert L.laq_gemm_chain(None, 1, FAKE, 256, None) == code["LAQ_ERR_NULL"]
+    assert chain(L, [ok], ws=ctypes.c_void_p(0)) == code["LAQ_ERR_WORKSPACE"]
+    assert chain(L, [ok], ws=ODD) == code["LAQ_ERR_WORKSPACE"]
+    assert chain(L, [ok] * 100, ws_bytes=256) == code["LAQ_ERR_WORKSPACE"]
+    assert chain(L, [chain_entry(bits=5)]) == code["LAQ_ERR_BITS"]
+    assert chain(L, [ok, chain_entry(bits=4)]) == code["LAQ_ERR_BITS"]
+    assert chain(L, [chain_entry(M=0)]) == code["LAQ_ERR_M_RANGE"]
+    assert chain(L, [chain_entry(M=5)]) == code["LAQ_ERR_M_RANGE"]
+    assert chain(L, [ok, chain_entry(M=2)]) == code["LAQ_ERR_M_RANGE"]
+    assert chain(L, [chain_entry(K=200)]) == code["LAQ_ERR_SHAPE"]
+    assert chain(L, [chain_entry(N=40)]) == code["LAQ_ERR_SHAPE"]
+    assert chain(L, [chain_entry(K=0)]) == code["LAQ_ERR_SHAPE"]
+    assert chain(L, [chain_entry(N=0)]) == code["LAQ_ERR_SHAPE"]
+    assert chain(L, [ok, chain_entry(Y=ctypes.c_void_p(0))]) == code["LAQ_ERR_NULL"]
+    for field in ("X", "packed", "s", "z", "Y"):
+        assert chain(L, [chain_entry(**{field: ODD})]) == code["LAQ_ERR_ALIGN"], field
