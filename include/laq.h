@@ -220,6 +220,27 @@ size_t laq_chain_workspace_bytes(int32_t count);
 laq_status laq_gemm_chain(const laq_gemv *gemvs, int32_t count, void *workspace,
                           size_t workspace_bytes, void *stream);
 
+/*
+ * laq_gemm_chain without a caller-provided workspace, for callers that cannot allocate device
+ * memory: a plug-in or custom operator whose host framework owns every device allocation and
+ * offers no scratch, or a decode loop that must not call cudaMalloc once it runs (cudaMalloc
+ * may synchronize the device and stalls every stream).  The paper has no counterpart; this is
+ * a deployment convenience of this library.
+ *
+ * Same entries, results and restrictions as laq_gemm_chain.  The counters live in a scratch
+ * array inside the library (a static device array of 1792 bytes, enough for LAQ_CHAIN_MAX
+ * entries), held by every GPU that loads the library until the process exits.  Nothing is
+ * allocated: each call clears the counters it uses (cudaMemsetAsync on `stream`) and launches.
+ *   count > LAQ_CHAIN_MAX  -> LAQ_ERR_WORKSPACE (the scratch holds no more).
+ * The first call on each device looks up the scratch array's device address (and, like every
+ * first call of a kernel variant, sets its shared-memory limit): make it before any stream
+ * capture.  All calls share the one array, so calls whose executions overlap on the GPU (other
+ * streams, or other host threads) race and give undefined results; serialize them.  A
+ * device-side timeout is not reported here (laq_gemm_chain's workspace status word is the way
+ * to observe one).
+ */
+laq_status laq_gemm_chain_static(const laq_gemv *gemvs, int32_t count, void *stream);
+
 #ifdef __cplusplus
 }
 #endif

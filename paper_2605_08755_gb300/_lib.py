@@ -19,7 +19,7 @@ STATUS = {0: "LAQ_OK", 1: "LAQ_ERR_NULL", 2: "LAQ_ERR_BITS", 3: "LAQ_ERR_GROUP",
 # Symbols include/laq.h declares.
 EXPORTS = ("laq_status_str", "laq_version", "laq_packed_bytes", "laq_quantize_rtn", "laq_pack",
            "laq_unpack", "laq_gemm_wxg128", "laq_gemm_plan", "laq_gemm_wxg128_config",
-           "laq_chain_workspace_bytes", "laq_gemm_chain")
+           "laq_chain_workspace_bytes", "laq_gemm_chain", "laq_gemm_chain_static")
 CHAIN_MAX = 384  # LAQ_CHAIN_MAX
 
 
@@ -74,8 +74,10 @@ def lib():
     L.laq_chain_workspace_bytes.argtypes = [ctypes.c_int32]
     L.laq_chain_workspace_bytes.restype = ctypes.c_size_t
     L.laq_gemm_chain.argtypes = [ctypes.POINTER(Gemv), ctypes.c_int32, P, ctypes.c_size_t, P]
+    L.laq_gemm_chain_static.argtypes = [ctypes.POINTER(Gemv), ctypes.c_int32, P]
     for name in ("laq_quantize_rtn", "laq_pack", "laq_unpack", "laq_gemm_wxg128",
-                 "laq_gemm_plan", "laq_gemm_wxg128_config", "laq_gemm_chain"):
+                 "laq_gemm_plan", "laq_gemm_wxg128_config", "laq_gemm_chain",
+                 "laq_gemm_chain_static"):
         getattr(L, name).restype = I
     return L
 
@@ -185,6 +187,11 @@ class Chain:
         ws = workspace
         _check(lib().laq_gemm_chain(self.array, self.count, _ptr(ws), ws.numel(),
                                     _stream(stream)), "laq_gemm_chain")
+
+    def run_static(self, stream=None):
+        """The same chain through laq_gemm_chain_static (the library's own scratch)."""
+        _check(lib().laq_gemm_chain_static(self.array, self.count, _stream(stream)),
+               "laq_gemm_chain_static")
 
 
 def laq_gemm_chain(entries, workspace, stream=None):

@@ -273,6 +273,33 @@ laq_status run_chain(const laq_gemv* g, int32_t count, void* workspace, size_t w
     return from_cuda(laq::launch_chain(L, f.sms, static_cast<cudaStream_t>(stream)));
 }
 
+
+// ---- laq_gemm_chain_static: the chain with library-owned scratch ----------------------------
+
+// The chain's counters for calls that pass no workspace: status, finished CTAs and one arrival
+// counter per stage, for up to LAQ_CHAIN_MAX entries (1792 bytes).  Zero at module load; every
+// GPU that loads the library keeps it until the process exits.
+constexpr size_t kStaticScratchBytes = (4 * (2 + LAQ_CHAIN_MAX) + 255) / 256 * 256;
+static __device__ __align__(256) uint32_t g_chain_scratch[kStaticScratchBytes / 4];
+
+// Device address of g_chain_scratch per device, looked up on the first call with that device
+// current (the array's name is only a host-side stand-in for it).
+std::atomic<void*> g_scratch_addr[kMaxDevices];
+
+laq_status static_scratch(void** out) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return LAQ_ERR_CUDA;
+    if (dev < 0 || dev >= kMaxDevices) return LAQ_ERR_CUDA;
+    void* ptr = g_scratch_addr[dev].load();
+    if (!ptr) {
+        if (cudaGetSymbolAddress(&ptr, g_chain_scratch) != cudaSuccess || !ptr)
+            return LAQ_ERR_CUDA;
+        g_scratch_addr[dev].store(ptr);
+    }
+    *out = ptr;
+    return LAQ_OK;
+}
+
 }  // namespace
 
 extern "C" {
@@ -375,6 +402,20 @@ size_t laq_chain_workspace_bytes(int32_t count) {
 laq_status laq_gemm_chain(const laq_gemv* gemvs, int32_t count, void* workspace,
                           size_t workspace_bytes, void* stream) {
     return run_chain(gemvs, count, workspace, workspace_bytes, stream);
+}
+
+laq_status laq_gemm_chain_static(const laq_gemv* gemvs, int32_t count, void* stream) {
+    if (count < 0 || count > LAQ_CHAIN_MAX) return LAQ_ERR_WORKSPACE;  // beyond the scratch
+    if (count == 0) return LAQ_OK;
+    if (!gemvs) return LAQ_ERR_NULL;
+    void* scratch = nullptr;
+    laq_status st = static_scratch(&scratch);
+    if (st != LAQ_OK) return st;
+    // Counters must start at zero; a previous call that gave up may have left them set.
+    const size_t used = chain_ws_bytes(count);
+    if (cudaMemsetAsync(scratch, 0, used, static_cast<cudaStream_t>(stream)) != cudaSuccess)
+        return LAQ_ERR_CUDA;
+    return run_chain(gemvs, count, scratch, used, stream);
 }
 
 }  // extern "C"

@@ -190,3 +190,12 @@ def test_chain_argument_validation(L):
     assert chain(L, [ok, chain_entry(Y=ctypes.c_void_p(0))]) == code["LAQ_ERR_NULL"]
     for field in ("X", "packed", "s", "z", "Y"):
         assert chain(L, [chain_entry(**{field: ODD})]) == code["LAQ_ERR_ALIGN"], field
+
+
+def test_chain_static_argument_validation(L):
+    code = {v: k for k, v in _lib.STATUS.items()}
+    arr = (_lib.Gemv * 1)(chain_entry())
+    assert L.laq_gemm_chain_static(arr, 0, None) == 0
+    assert L.laq_gemm_chain_static(arr, _lib.CHAIN_MAX + 1, None) == code["LAQ_ERR_WORKSPACE"]
+    assert L.laq_gemm_chain_static(arr, -1, None) == code["LAQ_ERR_WORKSPACE"]
+    assert L.laq_gemm_chain_static(None, 1, None) == code["LAQ_ERR_NULL"]
