@@ -241,6 +241,7 @@ laq_status run_chain(const laq_gemv* g, int32_t count, void* workspace, size_t w
         ce.K = (int)e.K;
         ce.N = (int)e.N;
         ce.xoff = (int)(stage_x / 16);
+        ce.psoff = (int)(stage_x / 256);  // one (S, P) pair per 128 fp16 of X
         stage_x += M * e.K * 2;
         stage_units += e.N / 16;
         if (stage_units > ((int64_t)1 << 30)) return LAQ_ERR_SHAPE;
@@ -253,10 +254,8 @@ laq_status run_chain(const laq_gemv* g, int32_t count, void* workspace, size_t w
     st = device_facts(&f);
     if (st != LAQ_OK) return st;
     const size_t slot = (size_t)(bits == 4 ? 1024 : 768) + 48;
-    // ring depth: slots for one block of 8 / M-class records plus at least one in flight
-    const int gpa = M <= 1 ? 8 : M <= 2 ? 4 : 2;
     const size_t fixed = laq::chain_smem_bytes(bits, (int)M, 0, (int)xs_need, nst);
-    if (fixed + (size_t)kChainWarps * (gpa + 1) * slot > f.smem_optin) return LAQ_ERR_SHAPE;
+    if (fixed + (size_t)kChainWarps * 2 * slot > f.smem_optin) return LAQ_ERR_SHAPE;
     int ring = (int)((f.smem_optin - fixed) / ((size_t)kChainWarps * slot));
     if (ring > 16) ring = 16;
 

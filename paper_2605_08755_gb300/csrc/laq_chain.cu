@@ -23,12 +23,12 @@
 //    every CTA returns.
 //
 //  * The record arithmetic is that of laq_gemm.cu: one LOP3 per pair of codes gives the fp16
-//    values c + q, an m16n8k16 MMA contracts them with raw x into D.  Per block of groups that
-//    share the accumulator, one more MMA per k16 step, whose A rows 0-7 hold the offsets c_k
-//    and rows 8-15 hold 1, gives P_g = sum_k c_k x_k and S_g = sum_k x_k in the layout of D,
-//    and the epilogue applies Eq. (1) as y += s * (D - P - z S).  A tile whose groups are split
-//    between warps is summed in shared memory at the end of the stage in warp order
-//    (deterministic, no atomics on Y).
+//    values c + q, an m16n8k16 MMA contracts them with raw x into D.  While X is staged, the
+//    16 lanes that load a group's 256 bytes also sum P_g = sum_k c_k x_k and S_g = sum_k x_k,
+//    and the epilogue of each block of groups that share the accumulator applies Eq. (1) as
+//    y += s * (D - P - z S), with the block's scales and zeros copied aside from the ring.  A
+//    tile whose groups are split between warps is summed in shared memory at the end of the
+//    stage in warp order (deterministic, no atomics on Y).
 //
 //  * The last CTA to finish resets the counters, so the workspace is zero again for the next
 //    call on the stream.
@@ -69,6 +69,7 @@ struct ChainEntryDev {
     uint16_t* Y;
     int K, N;
     int xoff;   // offset of this entry's X in the stage's shared X area (16-byte units)
+    int psoff;  // offset of its (S, P) pairs in the stage's table (one per row and group)
 };
 
 struct ChainStageDev {
@@ -105,6 +106,9 @@ __device__ __forceinline__ uint32_t ld_relaxed(const uint32_t* p) {
     uint32_t v;
     asm volatile("ld.relaxed.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
     return v;
+}
+__device__ __forceinline__ void red_release_add(uint32_t* p, uint32_t v) {
+    asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
 }
 __device__ __forceinline__ uint4 ld_cg16(const void* p) {
     uint4 v;
@@ -291,23 +295,12 @@ struct RecordStream {
     }
 };
 
-// A fragment of the (S, P) contraction for k16 step j: rows 0-7 hold the offsets c_k of the
-// step's pairs (the fp16 value of code 0 in each field: its exponent constant), rows 8-15
-// hold 1, so one more MMA per step sums P_g = sum_k c_k x_k and S_g = sum_k x_k per column.
-template <int BITS>
-__device__ __forceinline__ uint32_t ps_offset(const Exps& x, int j, int h) {
-    const int i = 2 * j + h;  // pair index
-    if (BITS == 4) return h == 0 ? x.e[0] : x.e[1];
-    return i < 6 ? x.e[0] : (i < 12 ? x.e[1] : (i < 15 ? x.e[2] : x.e[1]));
-}
-
 template <int BITS, int MP>
 __global__ void __launch_bounds__(kChainThreads, 1) chain_kernel(const __grid_constant__ ChainParams p) {
     using F = RecordFmt<BITS>;
     constexpr int SLOT = Slot<BITS>::kBytes;
     constexpr int WPL = BITS == 4 ? 8 : 6;
     constexpr int GPA = 8 / MP;  // groups sharing one accumulator (MMA columns), MP <= 4
-    constexpr uint32_t kOnes = 0x3c003c00u;
 
     extern __shared__ __align__(128) uint8_t smem[];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -316,13 +309,18 @@ __global__ void __launch_bounds__(kChainThreads, 1) chain_kernel(const __grid_co
     uint32_t* status = p.ws;
 
     // shared memory: ring [16][S][slot] | X [xs_bytes] | zero block (64 B)
+    //                | (S, P) per (entry, row, group) [xs_bytes / 256] float2
+    //                | scales and zeros of each warp's current block [16][GPA][48 B]
     //                | split-tile partial sums [32][MP][16] fp32 | their tile keys [32]
     //                | this CTA's (first unit, end unit, records) per stage [nstages] int4
     //                | flag
     uint8_t* ring = smem;
     uint4* xs = reinterpret_cast<uint4*>(smem + (size_t)kChainWarps * S * SLOT);
     uint4* zblk = xs + p.xs_bytes / 16;
-    float* red = reinterpret_cast<float*>(zblk + 4);
+    float2* ps = reinterpret_cast<float2*>(zblk + 4);
+    uint4* sbuf_all = reinterpret_cast<uint4*>(reinterpret_cast<uint8_t*>(ps) +
+                                               ((p.xs_bytes / 256 * 8 + 15) & ~15));
+    float* red = reinterpret_cast<float*>(sbuf_all + kChainWarps * GPA * 3);
     int* keys = reinterpret_cast<int*>(red + 2 * kChainWarps * MP * 16);
     int4* range = reinterpret_cast<int4*>(keys + 2 * kChainWarps);
     int* flag = reinterpret_cast<int*>(range + p.nstages);
@@ -345,6 +343,10 @@ __global__ void __launch_bounds__(kChainThreads, 1) chain_kernel(const __grid_co
     const uint32_t ring_s = (uint32_t)__cvta_generic_to_shared(ring) +
                             (uint32_t)(warp * S * SLOT);
     const uint8_t* ring_w = ring + (size_t)warp * S * SLOT;
+    uint4* sbuf = sbuf_all + warp * GPA * 3;  // [GPA][3] 16-byte pieces: scales x 2, zeros
+    // lanes that copied a scale / zero piece of each slot, and which piece
+    const int szp = BITS == 3 ? lane - 16 : lane;
+    const bool sz_lane = szp >= 0 && szp < 3;
 
     // Copy side of the ring: the next record of the warp's stream into the next slot (an
     // empty group once the stream is exhausted, so group counting stays uniform).
@@ -367,9 +369,8 @@ __global__ void __launch_bounds__(kChainThreads, 1) chain_kernel(const __grid_co
         cp_async_commit();
         islot = islot + 1 == S ? 0 : islot + 1;
     };
-    // Records in flight ahead of the one being consumed: the slots of a block (GPA records)
-    // stay valid until its epilogue has read their scales and zeros.
-    const int ahead = S - GPA;
+    // Records in flight ahead of the one being consumed.
+    const int ahead = S - 1;
     for (int q = 0; q < ahead; ++q) issue();
     int rslot = 0;
 
@@ -382,10 +383,7 @@ __global__ void __launch_bounds__(kChainThreads, 1) chain_kernel(const __grid_co
         const int u0 = range[s].x, u1 = range[s].y;
         if (u1 <= u0) {
             // Nothing of this stage here: report it done at once.
-            if (threadIdx.x == 0) {
-                __threadfence();
-                atomicAdd(p.ws + 2 + s, 1u);
-            }
+            if (threadIdx.x == 0) red_release_add(p.ws + 2 + s, 1u);
             continue;
         }
         LAQ_CHAIN_TRACE(s, 0);
@@ -410,20 +408,49 @@ __global__ void __launch_bounds__(kChainThreads, 1) chain_kernel(const __grid_co
                 const ChainEntryDev& E = p.e[st.e0 + q];
                 const int T = E.N >> 4;
                 if (ubase < u1 && ubase + T > u0) {
-                    const int n16 = M * E.K / 8;
+                    // 16-byte chunk uu holds x[8 uu .. 8 uu + 7] of the [M][K] rows: chunk
+                    // uu % 16 of group uu / 16 (row b, group g), rows 8 (uu % 16) + e of the
+                    // group, i.e. pairs 4 (uu % 4) + w for its four 32-bit words w.  The 16
+                    // chunks of a group sit in 16 consecutive lanes, which sum
+                    // S_g = sum_k x_k and P_g = sum_k c_k x_k by shuffles.
+                    const int n16 = M * E.K / 8;  // a multiple of 16
                     const uint8_t* src = reinterpret_cast<const uint8_t*>(E.X);
                     uint4* dst = xs + E.xoff;
-                    for (int u = threadIdx.x; u < n16; u += 4 * kChainThreads) {
+                    for (int u = 0; u < n16; u += 4 * kChainThreads) {
                         uint4 v[4];
 #pragma unroll
                         for (int r = 0; r < 4; ++r) {
-                            const int uu = u + r * kChainThreads;
-                            if (uu < n16) v[r] = ld_cg16(src + (size_t)uu * 16);
+                            const int uu = u + r * kChainThreads + (int)threadIdx.x;
+                            v[r] = uu < n16 ? ld_cg16(src + (size_t)uu * 16)
+                                            : make_uint4(0u, 0u, 0u, 0u);
                         }
+                        // a group's 16 chunks are 16 aligned lanes: n16 is a multiple of 16, so
+                        // a warp's lanes are either all past n16 or share one boundary at a
+                        // 16-lane half
 #pragma unroll
                         for (int r = 0; r < 4; ++r) {
-                            const int uu = u + r * kChainThreads;
-                            if (uu < n16) dst[uu] = v[r];
+                            // (warp-uniform) nothing of this batch for this warp
+                            if (u + r * kChainThreads + warp * 32 >= n16) break;
+                            const int uu = u + r * kChainThreads + (int)threadIdx.x;
+                            const uint32_t w4[4] = {v[r].x, v[r].y, v[r].z, v[r].w};
+                            float sx = 0.f, px = 0.f;
+#pragma unroll
+                            for (int w = 0; w < 4; ++w) {
+                                const float2 f =
+                                    __half22float2(*reinterpret_cast<const __half2*>(&w4[w]));
+                                const float pair = f.x + f.y;
+                                sx += pair;
+                                px = fmaf(row_offset<BITS>((uu & 3) * 4 + w), pair, px);
+                            }
+#pragma unroll
+                            for (int o = 1; o < 16; o <<= 1) {
+                                sx += __shfl_xor_sync(0xffffffffu, sx, o);
+                                px += __shfl_xor_sync(0xffffffffu, px, o);
+                            }
+                            if (uu < n16) {
+                                dst[uu] = v[r];
+                                if ((uu & 15) == 0) ps[E.psoff + (uu >> 4)] = make_float2(sx, px);
+                            }
                         }
                     }
                 }
@@ -439,7 +466,7 @@ __global__ void __launch_bounds__(kChainThreads, 1) chain_kernel(const __grid_co
         Cursor cc;
         cc.s = s;
         if (cursor_begin(cc, p, range, warp)) {
-            int xoff = p.e[cc.e].xoff, G = cc.G;
+            int xoff = p.e[cc.e].xoff, pso = p.e[cc.e].psoff, G = cc.G;
             int piece_g0 = cc.g;  // first group of the current piece (run of one tile)
             bool first_piece = true;
             float yacc[4] = {0.f, 0.f, 0.f, 0.f};
@@ -473,6 +500,10 @@ __global__ void __launch_bounds__(kChainThreads, 1) chain_kernel(const __grid_co
                             }
                         }
                         const uint8_t* slot = ring_w + (size_t)rslot * SLOT;
+                        // this lane's scale / zero piece of the record, for the block epilogue
+                        if (sz_lane)
+                            sbuf[gi * 3 + szp] =
+                                *reinterpret_cast<const uint4*>(slot + F::kBytes + szp * 16);
                         uint32_t wd[WPL];
                         const uint4 c0 = *reinterpret_cast<const uint4*>(slot + lane * 16);
                         wd[0] = c0.x; wd[1] = c0.y; wd[2] = c0.z; wd[3] = c0.w;
@@ -494,44 +525,24 @@ __global__ void __launch_bounds__(kChainThreads, 1) chain_kernel(const __grid_co
                 }
                 __syncwarp();  // the scales and zeros of the block's slots came from other lanes
 
-                // S and P of the block's groups (columns), then Eq. (1): y += s (D - P - z S).
-                {
-                    float Q[4] = {0.f, 0.f, 0.f, 0.f};
-                    uint32_t B[8][2];
-                    const bool act = gil < nb && bl < M;
-                    const uint4* src = act ? xs + xoff + (size_t)(bl * G + gb + gil) * 16 + c * 4
-                                           : zblk;
+                // Eq. (1) per block column (a group of one batch row): y += s (D - P - z S).
+                // Value v of the lane is row R + 8 (v >> 1), column 2c + (v & 1), i.e. record
+                // (column % GPA) of the block and batch row column / GPA.
 #pragma unroll
-                    for (int q = 0; q < 4; ++q) {
-                        const uint4 v = src[q];
-                        B[2 * q][0] = v.x;
-                        B[2 * q][1] = v.y;
-                        B[2 * q + 1][0] = v.z;
-                        B[2 * q + 1][1] = v.w;
-                    }
-#pragma unroll
-                    for (int j = 0; j < 8; ++j)
-                        mma16816(Q, ps_offset<BITS>(p.exps, j, 0), kOnes,
-                                 ps_offset<BITS>(p.exps, j, 1), kOnes, B[j][0], B[j][1]);
-                    // value v of the lane: row R + 8 (v >> 1), column 2c + (v & 1) = record
-                    // (column % GPA) of the block for batch row column / GPA
-#pragma unroll
-                    for (int v1 = 0; v1 < 2; ++v1) {
-                        const int col = 2 * c + v1;
-                        const int b = col / GPA, rec = col % GPA;
-                        if (b < M && rec < nb) {
-                            int sl = rs0 + rec;
-                            sl = sl >= S ? sl - S : sl;
-                            const uint8_t* sz = ring_w + (size_t)sl * SLOT + F::kBytes;
-                            const uint16_t* ssl = reinterpret_cast<const uint16_t*>(sz);
-                            const float s0 = __half2float(__ushort_as_half(ssl[R]));
-                            const float s1 = __half2float(__ushort_as_half(ssl[R + 8]));
-                            const float z0 = (float)sz[32 + R], z1 = (float)sz[32 + R + 8];
-                            const float d0 = D[0][v1] + D[1][v1] - Q[v1];
-                            const float d1 = D[0][v1 + 2] + D[1][v1 + 2] - Q[v1];
-                            yacc[v1] = fmaf(s0, fmaf(-z0, Q[2 + v1], d0), yacc[v1]);
-                            yacc[v1 + 2] = fmaf(s1, fmaf(-z1, Q[2 + v1], d1), yacc[v1 + 2]);
-                        }
+                for (int v1 = 0; v1 < 2; ++v1) {
+                    const int col = 2 * c + v1;
+                    const int b = col / GPA, rec = col % GPA;
+                    if (b < M && rec < nb) {
+                        const uint8_t* sz = reinterpret_cast<const uint8_t*>(sbuf + rec * 3);
+                        const uint16_t* ssl = reinterpret_cast<const uint16_t*>(sz);
+                        const float s0 = __half2float(__ushort_as_half(ssl[R]));
+                        const float s1 = __half2float(__ushort_as_half(ssl[R + 8]));
+                        const float z0 = (float)sz[32 + R], z1 = (float)sz[32 + R + 8];
+                        const float2 sp = ps[pso + b * G + gb + rec];  // (S, P)
+                        const float d0 = D[0][v1] + D[1][v1] - sp.y;
+                        const float d1 = D[0][v1 + 2] + D[1][v1 + 2] - sp.y;
+                        yacc[v1] = fmaf(s0, fmaf(-z0, sp.x, d0), yacc[v1]);
+                        yacc[v1 + 2] = fmaf(s1, fmaf(-z1, sp.x, d1), yacc[v1 + 2]);
                     }
                 }
 
@@ -575,6 +586,7 @@ __global__ void __launch_bounds__(kChainThreads, 1) chain_kernel(const __grid_co
                     if (cc.left == 0) break;
                     if (cursor_next_tile(cc, p, range)) {
                         xoff = p.e[cc.e].xoff;
+                        pso = p.e[cc.e].psoff;
                         G = cc.G;
                     }
                     piece_g0 = 0;
@@ -612,10 +624,9 @@ __global__ void __launch_bounds__(kChainThreads, 1) chain_kernel(const __grid_co
         }
         __syncthreads();  // every Y value of this CTA's units is stored
         LAQ_CHAIN_TRACE(s, 7);
-        if (threadIdx.x == 0) {
-            __threadfence();
-            atomicAdd(p.ws + 2 + s, 1u);
-        }
+        // Release: the CTA's Y stores (ordered before by the barrier) become visible before
+        // the arrival does.
+        if (threadIdx.x == 0) red_release_add(p.ws + 2 + s, 1u);
         LAQ_CHAIN_TRACE(s, 6);
     }
 
@@ -653,6 +664,7 @@ size_t chain_smem_bytes(int bits, int M, int stages, int xs_bytes, int nstages) 
     const int mp = M <= 1 ? 1 : M <= 2 ? 2 : 4;
     const size_t slot = (size_t)(bits == 4 ? 1024 : 768) + kSzBytes;
     return (size_t)kChainWarps * stages * slot + (size_t)xs_bytes + 64 +
+           ((size_t)xs_bytes / 256 * 8 + 15) / 16 * 16 + (size_t)kChainWarps * (8 / mp) * 48 +
            (size_t)2 * kChainWarps * mp * 16 * 4 + (size_t)2 * kChainWarps * 4 +
            (size_t)nstages * 16 + 16;
 }
@@ -663,7 +675,7 @@ cudaError_t launch_chain(const ChainLaunch& L, int num_sms, cudaStream_t stream)
     ChainParams& P = *holder;
     for (int i = 0; i < L.count; ++i) {
         const ChainEntry& E = L.e[i];
-        P.e[i] = ChainEntryDev{E.X, E.packed, E.s, E.z, E.Y, E.K, E.N, E.xoff};
+        P.e[i] = ChainEntryDev{E.X, E.packed, E.s, E.z, E.Y, E.K, E.N, E.xoff, E.psoff};
     }
     for (int s = 0; s < L.nstages; ++s) P.st[s] = ChainStageDev{L.st[s].e0, L.st[s].ne, L.st[s].units};
     P.ws = L.ws;

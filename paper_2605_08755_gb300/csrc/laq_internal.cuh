@@ -37,7 +37,8 @@ struct ChainEntry {
     const uint8_t* z;
     uint16_t* Y;
     int K, N;
-    int xoff;  // X offset in the stage's shared X area, 16-byte units
+    int xoff;   // X offset in the stage's shared X area, 16-byte units
+    int psoff;  // offset in the stage's (S, P) table, one per (row, group)
 };
 struct ChainStage {
     int e0, ne, units;
