@@ -210,9 +210,8 @@ size_t laq_chain_workspace_bytes(int32_t count);
  * Restrictions: the packed codes, scales and zeros of every entry are read ahead of the chain
  * order, so no entry may write them; an entry may not read a Y written by an entry of its own
  * stage; the X of one stage (M * K * 2 bytes summed over its entries) must fit the kernel's
- * shared memory beside a weight ring of at least 8 / M-class + 1 records per warp
- * (LAQ_ERR_SHAPE otherwise; about 100 KB on GB300 at M = 1, and the more X, the shallower
- * the ring).  Uses every SM of
+ * shared memory beside its weight ring and descriptors (LAQ_ERR_SHAPE otherwise; on GB300
+ * about 95 KB for a 252-entry chain, a little more for shorter ones).  Uses every SM of
  * the device with one cooperative CTA each, so concurrent kernels on other streams wait.
  * Returns LAQ_ERR_M_RANGE for M outside 1..4, LAQ_ERR_BITS for mixed or invalid bits,
  * LAQ_ERR_WORKSPACE for a bad workspace, and the per-entry statuses of laq_gemm_wxg128.

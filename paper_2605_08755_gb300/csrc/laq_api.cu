@@ -188,7 +188,6 @@ laq_status run_gemm(const void* X, int64_t M, int64_t K, int64_t N, const void* 
 // ---- laq_gemm_chain -------------------------------------------------------------------------
 
 constexpr int kChainMaxM = 4;
-constexpr int kChainWarps = 16;  // warps per CTA of the chain kernel
 
 size_t chain_ws_bytes(int32_t count) {
     // status, finished-CTA counter, one arrival counter per stage (at most one per entry)
@@ -253,11 +252,8 @@ laq_status run_chain(const laq_gemv* g, int32_t count, void* workspace, size_t w
     DeviceFacts f;
     st = device_facts(&f);
     if (st != LAQ_OK) return st;
-    const size_t slot = (size_t)(bits == 4 ? 1024 : 768) + 48;
-    const size_t fixed = laq::chain_smem_bytes(bits, (int)M, 0, (int)xs_need, nst);
-    if (fixed + (size_t)kChainWarps * 2 * slot > f.smem_optin) return LAQ_ERR_SHAPE;
-    int ring = (int)((f.smem_optin - fixed) / ((size_t)kChainWarps * slot));
-    if (ring > 16) ring = 16;
+    if (laq::chain_smem_bytes(bits, (int)M, (int)xs_need, nst, count) > f.smem_optin)
+        return LAQ_ERR_SHAPE;  // the stage's X does not fit beside the weight ring
 
     laq::ChainLaunch L;
     L.e = ents.data();
@@ -266,7 +262,6 @@ laq_status run_chain(const laq_gemv* g, int32_t count, void* workspace, size_t w
     L.nstages = nst;
     L.M = (int)M;
     L.bits = bits;
-    L.stages = ring;
     L.xs_bytes = (int)xs_need;
     L.ws = static_cast<uint32_t*>(workspace);
     return from_cuda(laq::launch_chain(L, f.sms, static_cast<cudaStream_t>(stream)));

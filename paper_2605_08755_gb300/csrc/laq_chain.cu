@@ -81,16 +81,33 @@ struct ChainParams {
     ChainEntryDev e[kChainMax];
     ChainStageDev st[kChainMax];
     uint32_t* ws;  // [0] status, [1] finished CTAs, [2 + s] CTAs done with stage s
-    int count, nstages, M, stages, xs_bytes;
+    int count, nstages, M, xs_bytes;
     Exps exps;
 };
 static_assert(sizeof(ChainParams) <= 32000, "kernel parameters must stay below 32 KB");
+
+// The entry and stage descriptors as the kernel reads them: copied from the (large) parameter
+// block into shared memory once, so stage set-up and cursor moves never wait on a
+// constant-cache miss.
+struct Tables {
+    const ChainEntryDev* e;
+    const ChainStageDev* st;
+    int nstages;
+};
 
 template <int BITS>
 struct Slot {
     static constexpr int kRec = RecordFmt<BITS>::kBytes;
     static constexpr int kBytes = kRec + kSzBytes;  // 816 (b = 3) or 1072 (b = 4), 16-aligned
+    // Ring slots per warp.  One record is consumed while the others are in flight: 16 warps x
+    // 7 x 816 B (b = 3) or 5 x 1072 B (b = 4) ~ 90 KB per SM, above the ~64 KB that HBM's
+    // bandwidth x latency needs per SM.  A compile-time depth keeps cp.async.wait_group an
+    // immediate (a runtime count costs an indirect branch per record).
+    static constexpr int kRing = BITS == 3 ? 8 : 6;
 };
+
+// Ring slots per warp of the chain kernel at `bits` (host side).
+constexpr int chain_ring(int bits) { return bits == 3 ? Slot<3>::kRing : Slot<4>::kRing; }
 
 __device__ __forceinline__ unsigned long long globaltimer() {
     unsigned long long t;
@@ -156,7 +173,7 @@ struct Cursor {
 };
 
 // Place the cursor at the first record of warp w's share of stage c.s; false if it is empty.
-__device__ bool cursor_begin(Cursor& c, const ChainParams& p, const int4* range, int w) {
+__device__ bool cursor_begin(Cursor& c, const Tables& p, const int4* range, int w) {
     const int4 rg = range[c.s];  // first unit, end unit, records of this CTA
     const int r0 = (rg.z * w) >> 4, r1 = (rg.z * (w + 1)) >> 4;
     c.left = r1 - r0;
@@ -190,7 +207,7 @@ __device__ bool cursor_begin(Cursor& c, const ChainParams& p, const int4* range,
 
 // Step to the next record of the share (the caller has checked left > 1): 0 within the tile,
 // 1 to the first group of the next tile of the entry, 2 to the first record of a new entry.
-__device__ int cursor_step(Cursor& c, const ChainParams& p, const int4* range) {
+__device__ int cursor_step(Cursor& c, const Tables& p, const int4* range) {
     --c.left;
     if (++c.g < c.G) return 0;
     c.g = 0;
@@ -216,7 +233,7 @@ __device__ int cursor_step(Cursor& c, const ChainParams& p, const int4* range) {
 
 // Move to the first group of the next tile of the share (the caller has checked that records
 // remain): true if the entry changed.
-__device__ bool cursor_next_tile(Cursor& c, const ChainParams& p, const int4* range) {
+__device__ bool cursor_next_tile(Cursor& c, const Tables& p, const int4* range) {
     c.g = 0;
     if (++c.tile < c.tile_hi) return false;
     const int4 rg = range[c.s];
@@ -255,7 +272,7 @@ struct RecordStream {
     const uint8_t* p3;
     long long st2, st3;  // bytes to the next group's piece (p1 always moves by REC)
 
-    __device__ void point(const ChainParams& p, int lane) {
+    __device__ void point(const Tables& p, int lane) {
         const ChainEntryDev& E = p.e[c.e];
         const uint8_t* rec = E.packed + ((size_t)c.tile * c.G + c.g) * REC;
         const size_t gz = (size_t)c.g * E.N + (size_t)c.tile * 16;  // (group, column)
@@ -274,12 +291,12 @@ struct RecordStream {
             st3 = lane < 2 ? 2LL * E.N : (long long)E.N;
         }
     }
-    __device__ void seek(const ChainParams& p, const int4* range, int w, int lane) {
+    __device__ void seek(const Tables& p, const int4* range, int w, int lane) {
         while (c.s < p.nstages && !cursor_begin(c, p, range, w)) ++c.s;
         live = c.s < p.nstages;
         if (live) point(p, lane);
     }
-    __device__ void advance(const ChainParams& p, const int4* range, int w, int lane) {
+    __device__ void advance(const Tables& p, const int4* range, int w, int lane) {
         if (c.left > 1) {
             if (cursor_step(c, p, range) == 0) {
                 p1 += REC;
@@ -305,7 +322,8 @@ __global__ void __launch_bounds__(kChainThreads, 1) chain_kernel(const __grid_co
     extern __shared__ __align__(128) uint8_t smem[];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int c = lane & 3, R = lane >> 2;
-    const int M = p.M, S = p.stages;
+    const int M = p.M;
+    constexpr int S = Slot<BITS>::kRing;
     uint32_t* status = p.ws;
 
     // shared memory: ring [16][S][slot] | X [xs_bytes] | zero block (64 B)
@@ -313,7 +331,7 @@ __global__ void __launch_bounds__(kChainThreads, 1) chain_kernel(const __grid_co
     //                | scales and zeros of each warp's current block [16][GPA][48 B]
     //                | split-tile partial sums [32][MP][16] fp32 | their tile keys [32]
     //                | this CTA's (first unit, end unit, records) per stage [nstages] int4
-    //                | flag
+    //                | entry descriptors [count] | stage descriptors [nstages] | flag
     uint8_t* ring = smem;
     uint4* xs = reinterpret_cast<uint4*>(smem + (size_t)kChainWarps * S * SLOT);
     uint4* zblk = xs + p.xs_bytes / 16;
@@ -323,15 +341,21 @@ __global__ void __launch_bounds__(kChainThreads, 1) chain_kernel(const __grid_co
     float* red = reinterpret_cast<float*>(sbuf_all + kChainWarps * GPA * 3);
     int* keys = reinterpret_cast<int*>(red + 2 * kChainWarps * MP * 16);
     int4* range = reinterpret_cast<int4*>(keys + 2 * kChainWarps);
-    int* flag = reinterpret_cast<int*>(range + p.nstages);
+    ChainEntryDev* ent = reinterpret_cast<ChainEntryDev*>(range + p.nstages);
+    ChainStageDev* stg = reinterpret_cast<ChainStageDev*>(ent + p.count);
+    int* flag = reinterpret_cast<int*>(stg + p.nstages);
     if (threadIdx.x < 4) zblk[threadIdx.x] = make_uint4(0u, 0u, 0u, 0u);
+    for (int i = threadIdx.x; i < p.count; i += kChainThreads) ent[i] = p.e[i];
+    for (int i = threadIdx.x; i < p.nstages; i += kChainThreads) stg[i] = p.st[i];
+    __syncthreads();
+    const Tables tb{ent, stg, p.nstages};
     for (int s = threadIdx.x; s < p.nstages; s += kChainThreads) {
-        const int2 u = cta_units(p.st[s].units);
+        const int2 u = cta_units(stg[s].units);
         // records of the CTA: its units of each entry times the entry's groups
         int n = 0, ubase = 0;
-        const ChainStageDev st = p.st[s];
+        const ChainStageDev st = stg[s];
         for (int q = 0; q < st.ne; ++q) {
-            const int T = p.e[st.e0 + q].N >> 4, G = p.e[st.e0 + q].K >> 7;
+            const int T = ent[st.e0 + q].N >> 4, G = ent[st.e0 + q].K >> 7;
             const int lo = max(u.x, ubase), hi = min(u.y, ubase + T);
             if (hi > lo) n += (hi - lo) * G;
             ubase += T;
@@ -352,7 +376,7 @@ __global__ void __launch_bounds__(kChainThreads, 1) chain_kernel(const __grid_co
     // empty group once the stream is exhausted, so group counting stays uniform).
     RecordStream<BITS> is;
     is.c.s = 0;
-    is.seek(p, range, warp, lane);
+    is.seek(tb, range, warp, lane);
     int islot = 0;
     auto issue = [&]() {
         if (is.live) {
@@ -364,13 +388,13 @@ __global__ void __launch_bounds__(kChainThreads, 1) chain_kernel(const __grid_co
                 cp_async16(dst + 512, is.p2);
                 if (lane < 3) cp_async16(dst + 1024, is.p3);
             }
-            is.advance(p, range, warp, lane);
+            is.advance(tb, range, warp, lane);
         }
         cp_async_commit();
         islot = islot + 1 == S ? 0 : islot + 1;
     };
     // Records in flight ahead of the one being consumed.
-    const int ahead = S - 1;
+    constexpr int ahead = S - 1;
     for (int q = 0; q < ahead; ++q) issue();
     int rslot = 0;
 
@@ -379,7 +403,7 @@ __global__ void __launch_bounds__(kChainThreads, 1) chain_kernel(const __grid_co
     bool ok = true;
 
     for (int s = 0; s < p.nstages; ++s) {
-        const ChainStageDev st = p.st[s];
+        const ChainStageDev st = stg[s];
         const int u0 = range[s].x, u1 = range[s].y;
         if (u1 <= u0) {
             // Nothing of this stage here: report it done at once.
@@ -405,7 +429,7 @@ __global__ void __launch_bounds__(kChainThreads, 1) chain_kernel(const __grid_co
         {
             int ubase = 0;
             for (int q = 0; q < st.ne; ++q) {
-                const ChainEntryDev& E = p.e[st.e0 + q];
+                const ChainEntryDev& E = ent[st.e0 + q];
                 const int T = E.N >> 4;
                 if (ubase < u1 && ubase + T > u0) {
                     // 16-byte chunk uu holds x[8 uu .. 8 uu + 7] of the [M][K] rows: chunk
@@ -465,8 +489,8 @@ __global__ void __launch_bounds__(kChainThreads, 1) chain_kernel(const __grid_co
         // one tile, sharing the accumulator columns) at a time.
         Cursor cc;
         cc.s = s;
-        if (cursor_begin(cc, p, range, warp)) {
-            int xoff = p.e[cc.e].xoff, pso = p.e[cc.e].psoff, G = cc.G;
+        if (cursor_begin(cc, tb, range, warp)) {
+            int xoff = ent[cc.e].xoff, pso = ent[cc.e].psoff, G = cc.G;
             int piece_g0 = cc.g;  // first group of the current piece (run of one tile)
             bool first_piece = true;
             float yacc[4] = {0.f, 0.f, 0.f, 0.f};
@@ -484,7 +508,7 @@ __global__ void __launch_bounds__(kChainThreads, 1) chain_kernel(const __grid_co
                     if (gi < nb) {
                         __syncwarp();  // every lane is done with the slot the next copy overwrites
                         issue();
-                        cp_async_wait(ahead);
+                        asm volatile("cp.async.wait_group %0;\n" ::"n"(ahead) : "memory");
                         uint32_t B[8][2];
                         {
                             const bool act = gil == gi && bl < M;
@@ -565,7 +589,7 @@ __global__ void __launch_bounds__(kChainThreads, 1) chain_kernel(const __grid_co
                     if (piece_g0 == 0 && cc.g == G) {
                         // the whole tile: store
                         if (writer) {
-                            const ChainEntryDev& E = p.e[cc.e];
+                            const ChainEntryDev& E = ent[cc.e];
                             uint16_t* y = E.Y + (size_t)b * E.N + (size_t)cc.tile * 16;
                             y[R] = __half_as_ushort(__float2half_rn(y0));
                             y[R + 8] = __half_as_ushort(__float2half_rn(y1));
@@ -584,9 +608,9 @@ __global__ void __launch_bounds__(kChainThreads, 1) chain_kernel(const __grid_co
                     for (int v = 0; v < 4; ++v) yacc[v] = 0.f;
                     first_piece = false;
                     if (cc.left == 0) break;
-                    if (cursor_next_tile(cc, p, range)) {
-                        xoff = p.e[cc.e].xoff;
-                        pso = p.e[cc.e].psoff;
+                    if (cursor_next_tile(cc, tb, range)) {
+                        xoff = ent[cc.e].xoff;
+                        pso = ent[cc.e].psoff;
                         G = cc.G;
                     }
                     piece_g0 = 0;
@@ -615,7 +639,7 @@ __global__ void __launch_bounds__(kChainThreads, 1) chain_kernel(const __grid_co
                         acc += red[(size_t)j * MP * 16 + r];
                         m &= m - 1u;
                     }
-                    const ChainEntryDev& E = p.e[key >> 20];
+                    const ChainEntryDev& E = ent[key >> 20];
                     const int tile = key & 0xfffff, b = r >> 4, n = r & 15;
                     E.Y[(size_t)b * E.N + (size_t)tile * 16 + n] =
                         __half_as_ushort(__float2half_rn(acc));
@@ -660,13 +684,15 @@ std::atomic<size_t> g_chain_attr[2][3];  // dynamic shared memory already grante
 
 }  // namespace
 
-size_t chain_smem_bytes(int bits, int M, int stages, int xs_bytes, int nstages) {
+size_t chain_smem_bytes(int bits, int M, int xs_bytes, int nstages, int count) {
+    const int stages = chain_ring(bits);
     const int mp = M <= 1 ? 1 : M <= 2 ? 2 : 4;
     const size_t slot = (size_t)(bits == 4 ? 1024 : 768) + kSzBytes;
     return (size_t)kChainWarps * stages * slot + (size_t)xs_bytes + 64 +
            ((size_t)xs_bytes / 256 * 8 + 15) / 16 * 16 + (size_t)kChainWarps * (8 / mp) * 48 +
            (size_t)2 * kChainWarps * mp * 16 * 4 + (size_t)2 * kChainWarps * 4 +
-           (size_t)nstages * 16 + 16;
+           (size_t)nstages * 16 + (size_t)count * sizeof(ChainEntryDev) +
+           (size_t)nstages * sizeof(ChainStageDev) + 16;
 }
 
 cudaError_t launch_chain(const ChainLaunch& L, int num_sms, cudaStream_t stream) {
@@ -682,13 +708,12 @@ cudaError_t launch_chain(const ChainLaunch& L, int num_sms, cudaStream_t stream)
     P.count = L.count;
     P.nstages = L.nstages;
     P.M = L.M;
-    P.stages = L.stages;
     P.xs_bytes = L.xs_bytes;
     P.exps = exps_for(L.bits);
 
     const int mp = L.M <= 1 ? 1 : L.M <= 2 ? 2 : 4;
     const ChainFn fn = L.bits == 4 ? pick_chain<4>(mp) : pick_chain<3>(mp);
-    const size_t smem = chain_smem_bytes(L.bits, L.M, L.stages, L.xs_bytes, L.nstages);
+    const size_t smem = chain_smem_bytes(L.bits, L.M, L.xs_bytes, L.nstages, L.count);
     std::atomic<size_t>& granted = g_chain_attr[L.bits == 4][mp == 1 ? 0 : mp == 2 ? 1 : 2];
     cudaError_t err = cudaSuccess;
     if (granted.load() < smem) {

@@ -46,11 +46,11 @@ struct ChainStage {
 struct ChainLaunch {
     const ChainEntry* e;
     const ChainStage* st;
-    int count, nstages, M, bits, stages, xs_bytes;
+    int count, nstages, M, bits, xs_bytes;
     uint32_t* ws;
 };
-// Dynamic shared memory of the chain kernel for a ring of `stages` slots per warp.
-size_t chain_smem_bytes(int bits, int M, int stages, int xs_bytes, int nstages);
+// Dynamic shared memory of the chain kernel (its ring depth is fixed per bit width).
+size_t chain_smem_bytes(int bits, int M, int xs_bytes, int nstages, int count);
 cudaError_t launch_chain(const ChainLaunch& L, int num_sms, cudaStream_t stream);
 
 }  // namespace laq
