@@ -200,9 +200,11 @@ size_t laq_chain_workspace_bytes(int32_t count);
  *   gemvs      HOST array of `count` entries (read during the call only).  All entries share
  *              `bits` (3 or 4) and M (1..4).  K % 128 == 0, N % 16 == 0, K, N > 0.
  *   count      0..LAQ_CHAIN_MAX (0: nothing is enqueued).
- *   workspace  DEVICE buffer of at least laq_chain_workspace_bytes(count) bytes, 16-byte
- *              aligned, ZERO-FILLED before its first use.  A call that completes normally
- *              leaves it zero-filled again.  Word 0 (uint32) is the device-side status: 0, or
+ *   workspace  DEVICE buffer of at least laq_chain_workspace_bytes(count) bytes (about 67 KB:
+ *              stage counters, and a flag and a 256-byte partial tile for each of up to 256
+ *              CTAs), 16-byte aligned, ZERO-FILLED before its first use.  A call that
+ *              completes normally leaves its counters and flags zero again.  Word 0 (uint32)
+ *              is the device-side status: 0, or
  *              LAQ_ERR_TIMEOUT if a wait between stages gave up (after about a second); the
  *              call's Y values are then undefined and the caller must zero the workspace
  *              before the next call.  Calls sharing one workspace must not overlap in time.
@@ -226,10 +228,11 @@ laq_status laq_gemm_chain(const laq_gemv *gemvs, int32_t count, void *workspace,
  * may synchronize the device and stalls every stream).  The paper has no counterpart; this is
  * a deployment convenience of this library.
  *
- * Same entries, results and restrictions as laq_gemm_chain.  The counters live in a scratch
- * array inside the library (a static device array of 1792 bytes, enough for LAQ_CHAIN_MAX
+ * Same entries, results and restrictions as laq_gemm_chain.  The workspace lives in a scratch
+ * array inside the library (a static device array of 68,352 bytes, enough for LAQ_CHAIN_MAX
  * entries), held by every GPU that loads the library until the process exits.  Nothing is
- * allocated: each call clears the counters it uses (cudaMemsetAsync on `stream`) and launches.
+ * allocated: each call clears the counters and flags it uses (cudaMemsetAsync on `stream`)
+ * and launches.
  *   count > LAQ_CHAIN_MAX  -> LAQ_ERR_WORKSPACE (the scratch holds no more).
  * The first call on each device looks up the scratch array's device address (and, like every
  * first call of a kernel variant, sets its shared-memory limit): make it before any stream

@@ -190,9 +190,7 @@ laq_status run_gemm(const void* X, int64_t M, int64_t K, int64_t N, const void* 
 constexpr int kChainMaxM = 4;
 
 size_t chain_ws_bytes(int32_t count) {
-    // status, finished-CTA counter, one arrival counter per stage (at most one per entry)
-    const size_t words = 2 + (size_t)count;
-    return (words * 4 + 255) / 256 * 256;
+    return (laq::chain_workspace_bytes(count) + 255) / 256 * 256;
 }
 
 laq_status run_chain(const laq_gemv* g, int32_t count, void* workspace, size_t workspace_bytes,
@@ -210,7 +208,7 @@ laq_status run_chain(const laq_gemv* g, int32_t count, void* workspace, size_t w
     std::vector<laq::ChainEntry> ents((size_t)count);
     std::vector<laq::ChainStage> stages((size_t)count);
     int nst = 0;
-    int64_t xs_need = 0, stage_x = 0, stage_units = 0;
+    int64_t xs_need = 0, stage_x = 0, stage_records = 0;
     for (int32_t i = 0; i < count; ++i) {
         const laq_gemv& e = g[i];
         if (e.bits != bits) return LAQ_ERR_BITS;
@@ -224,11 +222,11 @@ laq_status run_chain(const laq_gemv* g, int32_t count, void* workspace, size_t w
             !aligned(e.z, 16) || !aligned(e.Y, 16))
             return LAQ_ERR_ALIGN;
         if (i == 0 || e.wait_prev != 0) {
-            if (i > 0) stages[nst - 1].units = (int)stage_units;
-            stages[nst] = laq::ChainStage{i, 0, 0};
+            if (i > 0) stages[nst - 1].records = (int)stage_records;
+            stages[nst] = laq::ChainStage{i, 0, 0, 0};
             ++nst;
             stage_x = 0;
-            stage_units = 0;
+            stage_records = 0;
         }
         laq::ChainStage& cs = stages[nst - 1];
         laq::ChainEntry& ce = ents[i];
@@ -242,16 +240,40 @@ laq_status run_chain(const laq_gemv* g, int32_t count, void* workspace, size_t w
         ce.xoff = (int)(stage_x / 16);
         ce.psoff = (int)(stage_x / 256);  // one (S, P) pair per 128 fp16 of X
         stage_x += M * e.K * 2;
-        stage_units += e.N / 16;
-        if (stage_units > ((int64_t)1 << 30)) return LAQ_ERR_SHAPE;
+        stage_records += (e.N / 16) * (e.K / 128);  // records
+        if (stage_records > ((int64_t)1 << 26)) return LAQ_ERR_SHAPE;
         ++cs.ne;
         if (stage_x > xs_need) xs_need = stage_x;
     }
-    stages[nst - 1].units = (int)stage_units;
+    stages[nst - 1].records = (int)stage_records;
 
     DeviceFacts f;
     st = device_facts(&f);
     if (st != LAQ_OK) return st;
+    if (f.sms > 256) return LAQ_ERR_SHAPE;  // one published part per CTA in the workspace
+    // Split a stage's tiles across CTAs (record shares, with a cross-CTA fix-up of the tiles
+    // that straddle two CTAs, about 1.5 us) only where whole-tile shares leave the busiest CTA
+    // far above the mean: at least 48 records (3 per warp) more.
+    for (int k = 0; k < nst; ++k) {
+        laq::ChainStage& cs = stages[k];
+        int64_t units = 0, maxrec = 0;
+        for (int q = 0; q < cs.ne; ++q) units += ents[cs.e0 + q].N / 16;
+        for (int b = 0; b < f.sms; ++b) {
+            // records of CTA b under whole-tile shares
+            const int64_t u0 = units * b / f.sms, u1 = units * (b + 1) / f.sms;
+            int64_t rec = 0, ubase = 0;
+            for (int q = 0; q < cs.ne; ++q) {
+                const int64_t T = ents[cs.e0 + q].N / 16, G = ents[cs.e0 + q].K / 128;
+                const int64_t lo = u0 > ubase ? u0 : ubase;
+                const int64_t hi = u1 < ubase + T ? u1 : ubase + T;
+                if (hi > lo) rec += (hi - lo) * G;
+                ubase += T;
+            }
+            if (rec > maxrec) maxrec = rec;
+        }
+        const int64_t even = (cs.records + f.sms - 1) / f.sms;
+        cs.split = maxrec - even >= 48 ? 1 : 0;
+    }
     if (laq::chain_smem_bytes(bits, (int)M, (int)xs_need, nst, count) > f.smem_optin)
         return LAQ_ERR_SHAPE;  // the stage's X does not fit beside the weight ring
 
@@ -270,10 +292,11 @@ laq_status run_chain(const laq_gemv* g, int32_t count, void* workspace, size_t w
 
 // ---- laq_gemm_chain_static: the chain with library-owned scratch ----------------------------
 
-// The chain's counters for calls that pass no workspace: status, finished CTAs and one arrival
-// counter per stage, for up to LAQ_CHAIN_MAX entries (1792 bytes).  Zero at module load; every
-// GPU that loads the library keeps it until the process exits.
-constexpr size_t kStaticScratchBytes = (4 * (2 + LAQ_CHAIN_MAX) + 255) / 256 * 256;
+// The chain's workspace for calls that pass none: status, finished CTAs, one arrival counter
+// per stage and one flag and published partial tile per CTA, for up to LAQ_CHAIN_MAX entries
+// and 256 CTAs (68,352 bytes).  Every GPU that loads the library keeps it until the process
+// exits.
+constexpr size_t kStaticScratchBytes = 68352;
 static __device__ __align__(256) uint32_t g_chain_scratch[kStaticScratchBytes / 4];
 
 // Device address of g_chain_scratch per device, looked up on the first call with that device
@@ -405,9 +428,12 @@ laq_status laq_gemm_chain_static(const laq_gemv* gemvs, int32_t count, void* str
     void* scratch = nullptr;
     laq_status st = static_scratch(&scratch);
     if (st != LAQ_OK) return st;
-    // Counters must start at zero; a previous call that gave up may have left them set.
+    // Counters and flags must start at zero; a previous call that gave up may have left them
+    // set.  (The published parts need no clearing.)
     const size_t used = chain_ws_bytes(count);
-    if (cudaMemsetAsync(scratch, 0, used, static_cast<cudaStream_t>(stream)) != cudaSuccess)
+    if (used > kStaticScratchBytes) return LAQ_ERR_WORKSPACE;
+    if (cudaMemsetAsync(scratch, 0, laq::chain_workspace_zeroed_bytes(count),
+                        static_cast<cudaStream_t>(stream)) != cudaSuccess)
         return LAQ_ERR_CUDA;
     return run_chain(gemvs, count, scratch, used, stream);
 }

@@ -61,6 +61,13 @@ constexpr int kSzBytes = 48;                          // 16 fp16 scales + 16 u8 
 constexpr unsigned long long kWaitNs = 1000000000ull; // stage wait limit (1 s)
 constexpr int kWaitSpins = 1 << 24;                   // and an iteration limit besides
 
+// Chain workspace (uint32 words): [0] status, [1] finished CTAs, [2 + s] CTAs done with stage
+// s, then at word flags_at(count): one flag per CTA (the last stage + 1 whose shared-tile part
+// it has published), then at word parts_at(count): one part [MP][16] fp32 per CTA (64 words).
+constexpr int kMaxGrid = 256;
+__host__ __device__ constexpr int flags_at(int count) { return (2 + count + 3) / 4 * 4; }
+__host__ __device__ constexpr int parts_at(int count) { return flags_at(count) + kMaxGrid; }
+
 struct ChainEntryDev {
     const uint16_t* X;
     const uint8_t* packed;
@@ -73,14 +80,16 @@ struct ChainEntryDev {
 };
 
 struct ChainStageDev {
-    int e0, ne;  // entries [e0, e0 + ne)
-    int units;   // 16-column tiles of the stage
+    int e0, ne;   // entries [e0, e0 + ne)
+    int records;  // (tile, group) records of the stage, entry by entry, tile-major
+    int split;    // 1: CTA shares are equal record ranges (tiles may straddle CTAs); 0: whole
+                  // tiles, split evenly by tile count
 };
 
 struct ChainParams {
     ChainEntryDev e[kChainMax];
     ChainStageDev st[kChainMax];
-    uint32_t* ws;  // [0] status, [1] finished CTAs, [2 + s] CTAs done with stage s
+    uint32_t* ws;  // see chain workspace layout below
     int count, nstages, M, xs_bytes;
     Exps exps;
 };
@@ -127,6 +136,14 @@ __device__ __forceinline__ uint32_t ld_relaxed(const uint32_t* p) {
 __device__ __forceinline__ void red_release_add(uint32_t* p, uint32_t v) {
     asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
 }
+__device__ __forceinline__ void st_release(uint32_t* p, uint32_t v) {
+    asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+__device__ __forceinline__ float ld_cg_f32(const float* p) {
+    float v;
+    asm volatile("ld.global.cg.f32 %0, [%1];" : "=f"(v) : "l"(p) : "memory");
+    return v;
+}
 __device__ __forceinline__ uint4 ld_cg16(const void* p) {
     uint4 v;
     asm volatile("ld.global.cg.v4.u32 {%0,%1,%2,%3}, [%4];"
@@ -150,109 +167,82 @@ __device__ bool wait_count(const uint32_t* cnt, uint32_t target, uint32_t* statu
     return false;
 }
 
-// The CTA's contiguous unit range of a stage with `units` units (64-bit products: computed once
-// per stage at kernel start, not per use).
-__device__ __forceinline__ int2 cta_units(int units) {
-    const long long P = gridDim.x, b = blockIdx.x;
-    return make_int2((int)(units * b / P), (int)(units * (b + 1) / P));
+// Wait until *flag == value (a CTA's published part of stage value - 1), with the limits of
+// wait_count.
+__device__ bool wait_flag(const uint32_t* flag, uint32_t value, uint32_t* status) {
+    const unsigned long long t0 = globaltimer();
+    for (int spin = 0; spin < kWaitSpins; ++spin) {
+        if (ld_relaxed(status) != 0u) return false;
+        if (ld_acquire(flag) == value) return true;
+        if ((spin & 31) == 31 && globaltimer() - t0 > kWaitNs) break;
+    }
+    atomicCAS(status, 0u, (uint32_t)LAQ_ERR_TIMEOUT);
+    return false;
+}
+
+// The end of CTA b's contiguous share of a stage's `records` records (64-bit products).
+__device__ __forceinline__ int cta_end(int records, int b) {
+    return (int)((long long)records * (b + 1) / gridDim.x);
 }
 
 // A warp's position in its record stream: stage s, entry e, tile (16-column block of the entry)
-// and group g.  Within a stage the CTA's records are its units in order, each unit's groups in
-// order; warp w takes the contiguous share [n w / 16, n (w + 1) / 16) of the CTA's n records,
-// so the warps of a CTA differ by at most one record.
+// and group g.  A stage's records are its entries' (tile, group) records in order, tile-major;
+// CTA b takes the contiguous share [R b / P, R (b + 1) / P) of the stage's R records (a tile
+// may straddle two CTAs), and warp w the contiguous share [n w / 16, n (w + 1) / 16) of the
+// CTA's n records, so CTAs differ by at most one record, and so do the warps of a CTA.
 struct Cursor {
-    int s;        // stage
-    int left;     // records of the share from the current one to its end
-    int e;        // entry
-    int tile;     // tile within the entry
-    int g;        // group within the tile
-    int G;        // groups of the entry
-    int tile_hi;  // end of the CTA's tiles of this entry
-    int ubase;    // first unit of entry e within the stage
+    int s;     // stage
+    int left;  // records of the share from the current one to its end
+    int e;     // entry
+    int tile;  // tile within the entry
+    int g;     // group within the tile
+    int G, T;  // groups and tiles of the entry
 };
 
 // Place the cursor at the first record of warp w's share of stage c.s; false if it is empty.
 __device__ bool cursor_begin(Cursor& c, const Tables& p, const int4* range, int w) {
-    const int4 rg = range[c.s];  // first unit, end unit, records of this CTA
-    const int r0 = (rg.z * w) >> 4, r1 = (rg.z * (w + 1)) >> 4;
-    c.left = r1 - r0;
+    const int4 rg = range[c.s];  // CTA's first record, end record, record count
+    const int a = (rg.z * w) >> 4, b = (rg.z * (w + 1)) >> 4;
+    c.left = b - a;
     if (c.left <= 0) return false;
-    int r = r0;
+    int r = rg.x + a;
     const ChainStageDev st = p.st[c.s];
-    int ubase = 0;
     for (int q = 0; q < st.ne; ++q) {
         const int e = st.e0 + q;
         const int T = p.e[e].N >> 4, G = p.e[e].K >> 7;
-        const int lo = max(rg.x, ubase), hi = min(rg.y, ubase + T);
-        if (hi > lo) {
-            const int cnt = (hi - lo) * G;
-            if (r < cnt) {
-                const int t = r / G;
-                c.e = e;
-                c.G = G;
-                c.ubase = ubase;
-                c.tile = lo - ubase + t;
-                c.g = r - t * G;
-                c.tile_hi = hi - ubase;
-                return true;
-            }
-            r -= cnt;
-        }
-        ubase += T;
-    }
-    c.left = 0;  // not reached: r0 < n
-    return false;
-}
-
-// Step to the next record of the share (the caller has checked left > 1): 0 within the tile,
-// 1 to the first group of the next tile of the entry, 2 to the first record of a new entry.
-__device__ int cursor_step(Cursor& c, const Tables& p, const int4* range) {
-    --c.left;
-    if (++c.g < c.G) return 0;
-    c.g = 0;
-    if (++c.tile < c.tile_hi) return 1;
-    const int4 rg = range[c.s];
-    const ChainStageDev st = p.st[c.s];
-    int ubase = c.ubase + (p.e[c.e].N >> 4);
-    for (int e = c.e + 1; e < st.e0 + st.ne; ++e) {
-        const int T = p.e[e].N >> 4;
-        const int lo = max(rg.x, ubase), hi = min(rg.y, ubase + T);
-        if (hi > lo) {
+        if (r < T * G) {
+            const int t = r / G;
             c.e = e;
-            c.G = p.e[e].K >> 7;
-            c.ubase = ubase;
-            c.tile = lo - ubase;
-            c.tile_hi = hi - ubase;
-            return 2;
+            c.G = G;
+            c.T = T;
+            c.tile = t;
+            c.g = r - t * G;
+            return true;
         }
-        ubase += T;
+        r -= T * G;
     }
-    return 2;  // not reached while left > 0
+    c.left = 0;  // not reached: the share lies inside the stage
+    return false;
 }
 
 // Move to the first group of the next tile of the share (the caller has checked that records
 // remain): true if the entry changed.
-__device__ bool cursor_next_tile(Cursor& c, const Tables& p, const int4* range) {
+__device__ bool cursor_next_tile(Cursor& c, const Tables& p) {
     c.g = 0;
-    if (++c.tile < c.tile_hi) return false;
-    const int4 rg = range[c.s];
-    const ChainStageDev st = p.st[c.s];
-    int ubase = c.ubase + (p.e[c.e].N >> 4);
-    for (int e = c.e + 1; e < st.e0 + st.ne; ++e) {
-        const int T = p.e[e].N >> 4;
-        const int lo = max(rg.x, ubase), hi = min(rg.y, ubase + T);
-        if (hi > lo) {
-            c.e = e;
-            c.G = p.e[e].K >> 7;
-            c.ubase = ubase;
-            c.tile = lo - ubase;
-            c.tile_hi = hi - ubase;
-            return true;
-        }
-        ubase += T;
-    }
-    return true;  // not reached while records remain
+    if (++c.tile < c.T) return false;
+    ++c.e;
+    c.tile = 0;
+    c.G = p.e[c.e].K >> 7;
+    c.T = p.e[c.e].N >> 4;
+    return true;
+}
+
+// Step to the next record of the share (the caller has checked left > 1): 0 within the tile,
+// 1 to the first group of the next tile of the entry, 2 to the first record of a new entry.
+__device__ int cursor_step(Cursor& c, const Tables& p) {
+    --c.left;
+    if (++c.g < c.G) return 0;
+    return cursor_next_tile(c, p) ? 2 : 1;
 }
 
 // The warp's record stream on the copy side of the ring (the compute side walks the same
@@ -298,7 +288,7 @@ struct RecordStream {
     }
     __device__ void advance(const Tables& p, const int4* range, int w, int lane) {
         if (c.left > 1) {
-            if (cursor_step(c, p, range) == 0) {
+            if (cursor_step(c, p) == 0) {
                 p1 += REC;
                 p2 += st2;
                 p3 += st3;
@@ -339,7 +329,7 @@ __global__ void __launch_bounds__(kChainThreads, 1) chain_kernel(const __grid_co
     uint4* sbuf_all = reinterpret_cast<uint4*>(reinterpret_cast<uint8_t*>(ps) +
                                                ((p.xs_bytes / 256 * 8 + 15) & ~15));
     float* red = reinterpret_cast<float*>(sbuf_all + kChainWarps * GPA * 3);
-    int* keys = reinterpret_cast<int*>(red + 2 * kChainWarps * MP * 16);
+    int* keys = reinterpret_cast<int*>(red + (2 * kChainWarps + 1) * MP * 16);
     int4* range = reinterpret_cast<int4*>(keys + 2 * kChainWarps);
     ChainEntryDev* ent = reinterpret_cast<ChainEntryDev*>(range + p.nstages);
     ChainStageDev* stg = reinterpret_cast<ChainStageDev*>(ent + p.count);
@@ -350,17 +340,29 @@ __global__ void __launch_bounds__(kChainThreads, 1) chain_kernel(const __grid_co
     __syncthreads();
     const Tables tb{ent, stg, p.nstages};
     for (int s = threadIdx.x; s < p.nstages; s += kChainThreads) {
-        const int2 u = cta_units(stg[s].units);
-        // records of the CTA: its units of each entry times the entry's groups
-        int n = 0, ubase = 0;
         const ChainStageDev st = stg[s];
-        for (int q = 0; q < st.ne; ++q) {
-            const int T = ent[st.e0 + q].N >> 4, G = ent[st.e0 + q].K >> 7;
-            const int lo = max(u.x, ubase), hi = min(u.y, ubase + T);
-            if (hi > lo) n += (hi - lo) * G;
-            ubase += T;
+        int r0, r1;
+        if (st.split) {
+            r0 = blockIdx.x == 0 ? 0 : cta_end(st.records, blockIdx.x - 1);
+            r1 = cta_end(st.records, blockIdx.x);
+        } else {
+            // whole tiles: units [u0, u1) of the stage, as records
+            int units = 0;
+            for (int q = 0; q < st.ne; ++q) units += ent[st.e0 + q].N >> 4;
+            const int u0 = blockIdx.x == 0 ? 0 : cta_end(units, blockIdx.x - 1);
+            const int u1 = cta_end(units, blockIdx.x);
+            r0 = r1 = 0;
+            int ubase = 0, rbase = 0;
+            for (int q = 0; q < st.ne; ++q) {
+                const int T = ent[st.e0 + q].N >> 4, G = ent[st.e0 + q].K >> 7;
+                if (u0 >= ubase && u0 < ubase + T) r0 = rbase + (u0 - ubase) * G;
+                if (u1 >= ubase && u1 <= ubase + T) r1 = rbase + (u1 - ubase) * G;
+                ubase += T;
+                rbase += T * G;
+            }
+            if (u1 <= u0) r1 = r0;
         }
-        range[s] = make_int4(u.x, u.y, n, 0);
+        range[s] = make_int4(r0, r1, r1 - r0, 0);
     }
     __syncthreads();
 
@@ -404,8 +406,8 @@ __global__ void __launch_bounds__(kChainThreads, 1) chain_kernel(const __grid_co
 
     for (int s = 0; s < p.nstages; ++s) {
         const ChainStageDev st = stg[s];
-        const int u0 = range[s].x, u1 = range[s].y;
-        if (u1 <= u0) {
+        const int r0 = range[s].x, r1 = range[s].y;
+        if (r1 <= r0) {
             // Nothing of this stage here: report it done at once.
             if (threadIdx.x == 0) red_release_add(p.ws + 2 + s, 1u);
             continue;
@@ -424,14 +426,14 @@ __global__ void __launch_bounds__(kChainThreads, 1) chain_kernel(const __grid_co
             break;
         }
 
-        // X of every entry of the stage that has a unit here (M rows of K fp16, contiguous),
+        // X of every entry of the stage that has a record here (M rows of K fp16, contiguous),
         // through L2 (ld.global.cg: written by other SMs during this kernel).
         {
-            int ubase = 0;
+            int rbase = 0;
             for (int q = 0; q < st.ne; ++q) {
                 const ChainEntryDev& E = ent[st.e0 + q];
-                const int T = E.N >> 4;
-                if (ubase < u1 && ubase + T > u0) {
+                const int nrec = (E.N >> 4) * (E.K >> 7);
+                if (rbase < r1 && rbase + nrec > r0) {
                     // 16-byte chunk uu holds x[8 uu .. 8 uu + 7] of the [M][K] rows: chunk
                     // uu % 16 of group uu / 16 (row b, group g), rows 8 (uu % 16) + e of the
                     // group, i.e. pairs 4 (uu % 4) + w for its four 32-bit words w.  The 16
@@ -478,7 +480,7 @@ __global__ void __launch_bounds__(kChainThreads, 1) chain_kernel(const __grid_co
                         }
                     }
                 }
-                ubase += T;
+                rbase += nrec;
             }
         }
         __syncthreads();
@@ -608,7 +610,7 @@ __global__ void __launch_bounds__(kChainThreads, 1) chain_kernel(const __grid_co
                     for (int v = 0; v < 4; ++v) yacc[v] = 0.f;
                     first_piece = false;
                     if (cc.left == 0) break;
-                    if (cursor_next_tile(cc, tb, range)) {
+                    if (cursor_next_tile(cc, tb)) {
                         xoff = ent[cc.e].xoff;
                         pso = ent[cc.e].psoff;
                         G = cc.G;
@@ -621,8 +623,13 @@ __global__ void __launch_bounds__(kChainThreads, 1) chain_kernel(const __grid_co
         __syncthreads();  // partial sums of shared tiles are in red
         LAQ_CHAIN_TRACE(s, 5);
 
-        // Tiles shared by several warps: sum their parts in slot (= warp) order and store.  Every
-        // warp sees the 32 slot keys, one per lane; slots with equal keys are one tile's parts.
+        // Tiles shared by several warps: sum their parts in slot (= warp) order.  Every warp
+        // sees the 32 slot keys, one per lane; slots with equal keys are one tile's parts.  A
+        // tile inside this CTA's records is stored; the CTA's last tile, if it runs past the
+        // CTA's records, is published for the CTA that owns its end; the CTA's first tile, if
+        // it began in earlier CTAs, is finished here with their published parts.
+        float* pub = reinterpret_cast<float*>(p.ws + parts_at(p.count));  // [P][MP][16]
+        uint32_t* pflag = p.ws + flags_at(p.count);                       // [P]
         {
             const int kl = keys[lane];
             const unsigned same = __match_any_sync(0xffffffffu, kl);
@@ -631,22 +638,75 @@ __global__ void __launch_bounds__(kChainThreads, 1) chain_kernel(const __grid_co
                 const int sl = idx / (M * 16), r = idx - sl * (M * 16);
                 const int key = __shfl_sync(0xffffffffu, kl, sl);
                 const int first = __shfl_sync(0xffffffffu, firstl, sl);
-                unsigned m = __shfl_sync(0xffffffffu, same, sl);
+                const unsigned m = __shfl_sync(0xffffffffu, same, sl);
                 if (first) {
+                    // all 32 slots loaded independently (the parts of a tile are the slots
+                    // in m), then summed in slot order
+                    float part[2 * kChainWarps];
+#pragma unroll
+                    for (int j = 0; j < 2 * kChainWarps; ++j)
+                        part[j] = (m >> j) & 1u ? red[(size_t)j * MP * 16 + r] : 0.f;
                     float acc = 0.f;
-                    while (m) {
-                        const int j = __ffs(m) - 1;
-                        acc += red[(size_t)j * MP * 16 + r];
-                        m &= m - 1u;
+#pragma unroll
+                    for (int j = 0; j < 2 * kChainWarps; ++j) acc += part[j];
+                    const int e = key >> 20, tile = key & 0xfffff;
+                    int rbase = 0;  // first record of entry e in the stage
+                    for (int q = st.e0; q < e; ++q) rbase += (ent[q].N >> 4) * (ent[q].K >> 7);
+                    const int G = ent[e].K >> 7;
+                    const int tfirst = rbase + tile * G, tend = tfirst + G;
+                    if (tend > r1) {
+                        pub[(size_t)blockIdx.x * MP * 16 + r] = acc;  // published below
+                    } else if (tfirst < r0) {
+                        red[(size_t)(2 * kChainWarps) * MP * 16 + r] = acc;  // finished below
+                    } else {
+                        const ChainEntryDev& E = ent[e];
+                        const int bb = r >> 4, n = r & 15;
+                        E.Y[(size_t)bb * E.N + (size_t)tile * 16 + n] =
+                            __half_as_ushort(__float2half_rn(acc));
                     }
-                    const ChainEntryDev& E = ent[key >> 20];
-                    const int tile = key & 0xfffff, b = r >> 4, n = r & 15;
-                    E.Y[(size_t)b * E.N + (size_t)tile * 16 + n] =
+                }
+            }
+        }
+        if (st.split) {
+        __syncthreads();  // this CTA's published part is written
+        // Publish at once (every CTA, every split stage), before waiting on anyone: owners wait
+        // only for parts, never for each other's owned tiles.
+        if (threadIdx.x == 0) st_release(pflag + blockIdx.x, (uint32_t)(s + 1));
+        {
+            // The CTA's first record starts a tile that began in earlier CTAs?
+            int rbase = 0, q = 0;
+            for (; q < st.ne; ++q) {
+                const int nrec = (ent[st.e0 + q].N >> 4) * (ent[st.e0 + q].K >> 7);
+                if (r0 < rbase + nrec) break;
+                rbase += nrec;
+            }
+            const ChainEntryDev& E = ent[st.e0 + q];
+            const int G = E.K >> 7, tile = (r0 - rbase) / G;
+            const int tfirst = rbase + tile * G, tend = tfirst + G;
+            if (tfirst < r0 && tend <= r1 && threadIdx.x < M * 16) {
+                const int r = threadIdx.x;
+                // parts of the CTAs before this one whose records reach into the tile,
+                // in CTA order
+                int b0 = blockIdx.x - 1;
+                while (b0 > 0 && cta_end(st.records, b0 - 1) > tfirst) --b0;
+                float acc = 0.f;
+                bool good = true;
+                for (int b = b0; b < (int)blockIdx.x && good; ++b) {
+                    const int bs = b == 0 ? 0 : cta_end(st.records, b - 1);
+                    if (cta_end(st.records, b) == bs) continue;  // no records: nothing published
+                    good = wait_flag(pflag + b, (uint32_t)(s + 1), status);
+                    if (good) acc += ld_cg_f32(pub + (size_t)b * MP * 16 + r);
+                }
+                acc += red[(size_t)(2 * kChainWarps) * MP * 16 + r];
+                if (good) {
+                    const int bb = r >> 4, n = r & 15;
+                    E.Y[(size_t)bb * E.N + (size_t)tile * 16 + n] =
                         __half_as_ushort(__float2half_rn(acc));
                 }
             }
         }
-        __syncthreads();  // every Y value of this CTA's units is stored
+        }
+        __syncthreads();  // every Y value finished by this CTA is stored
         LAQ_CHAIN_TRACE(s, 7);
         // Release: the CTA's Y stores (ordered before by the barrier) become visible before
         // the arrival does.
@@ -663,6 +723,7 @@ __global__ void __launch_bounds__(kChainThreads, 1) chain_kernel(const __grid_co
         if (prev == gridDim.x - 1) {
             // Every CTA is past its last wait: leave the counters at zero for the next call.
             for (int s = 0; s < p.nstages; ++s) p.ws[2 + s] = 0u;
+            for (int b = 0; b < (int)gridDim.x; ++b) p.ws[flags_at(p.count) + b] = 0u;
             p.ws[1] = 0u;
             __threadfence();
         }
@@ -684,13 +745,18 @@ std::atomic<size_t> g_chain_attr[2][3];  // dynamic shared memory already grante
 
 }  // namespace
 
+size_t chain_workspace_bytes(int count) {
+    return ((size_t)parts_at(count) + (size_t)kMaxGrid * 4 * 16) * 4;
+}
+size_t chain_workspace_zeroed_bytes(int count) { return (size_t)parts_at(count) * 4; }
+
 size_t chain_smem_bytes(int bits, int M, int xs_bytes, int nstages, int count) {
     const int stages = chain_ring(bits);
     const int mp = M <= 1 ? 1 : M <= 2 ? 2 : 4;
     const size_t slot = (size_t)(bits == 4 ? 1024 : 768) + kSzBytes;
     return (size_t)kChainWarps * stages * slot + (size_t)xs_bytes + 64 +
            ((size_t)xs_bytes / 256 * 8 + 15) / 16 * 16 + (size_t)kChainWarps * (8 / mp) * 48 +
-           (size_t)2 * kChainWarps * mp * 16 * 4 + (size_t)2 * kChainWarps * 4 +
+           (size_t)(2 * kChainWarps + 1) * mp * 16 * 4 + (size_t)2 * kChainWarps * 4 +
            (size_t)nstages * 16 + (size_t)count * sizeof(ChainEntryDev) +
            (size_t)nstages * sizeof(ChainStageDev) + 16;
 }
@@ -703,7 +769,7 @@ cudaError_t launch_chain(const ChainLaunch& L, int num_sms, cudaStream_t stream)
         const ChainEntry& E = L.e[i];
         P.e[i] = ChainEntryDev{E.X, E.packed, E.s, E.z, E.Y, E.K, E.N, E.xoff, E.psoff};
     }
-    for (int s = 0; s < L.nstages; ++s) P.st[s] = ChainStageDev{L.st[s].e0, L.st[s].ne, L.st[s].units};
+    for (int s = 0; s < L.nstages; ++s) P.st[s] = ChainStageDev{L.st[s].e0, L.st[s].ne, L.st[s].records, L.st[s].split};
     P.ws = L.ws;
     P.count = L.count;
     P.nstages = L.nstages;

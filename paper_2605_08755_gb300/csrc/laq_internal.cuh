@@ -41,8 +41,13 @@ struct ChainEntry {
     int psoff;  // offset in the stage's (S, P) table, one per (row, group)
 };
 struct ChainStage {
-    int e0, ne, units;
+    int e0, ne, records;
+    int split;  // CTA shares by records (tiles may straddle CTAs) instead of whole tiles
 };
+// Chain workspace bytes for `count` entries (counters, per-CTA flags and published parts for
+// grids of up to 256 CTAs), and the leading bytes that must be zero before a launch.
+size_t chain_workspace_bytes(int count);
+size_t chain_workspace_zeroed_bytes(int count);
 struct ChainLaunch {
     const ChainEntry* e;
     const ChainStage* st;

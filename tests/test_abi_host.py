@@ -156,14 +156,18 @@ def chain(L, entries, ws=FAKE, ws_bytes=None, count=None):
     arr = (_lib.Gemv * max(1, len(entries)))(*entries)
     n = len(entries) if count is None else count
     if ws_bytes is None:
-        ws_bytes = max(L.laq_chain_workspace_bytes(max(0, min(n, _lib.CHAIN_MAX))), 256)
+        ws_bytes = L.laq_chain_workspace_bytes(max(0, min(n, _lib.CHAIN_MAX)))
     return L.laq_gemm_chain(arr, n, ws, ws_bytes, None)
 
 
 def test_chain_workspace_bytes(L):
-    assert L.laq_chain_workspace_bytes(0) == 256
-    assert L.laq_chain_workspace_bytes(252) == 1024            # 4 * (2 + 252) rounded to 256
-    assert L.laq_chain_workspace_bytes(_lib.CHAIN_MAX) >= 4 * (2 + _lib.CHAIN_MAX)
+    # counters (2 + count words, padded to 4) + 256 flags + 256 parts of 64 words, to 256 bytes
+    def expect(n):
+        words = (2 + n + 3) // 4 * 4 + 256 + 256 * 64
+        return (words * 4 + 255) // 256 * 256
+    assert L.laq_chain_workspace_bytes(0) == expect(0)
+    assert L.laq_chain_workspace_bytes(252) == expect(252) == 67584
+    assert L.laq_chain_workspace_bytes(_lib.CHAIN_MAX) == expect(_lib.CHAIN_MAX) == 68352
     assert L.laq_chain_workspace_bytes(_lib.CHAIN_MAX + 1) == 0
     assert L.laq_chain_workspace_bytes(-1) == 0
 

@@ -61,7 +61,9 @@ def test_single_entry(bits, M, K, N):
     laq.laq_gemm_chain([(Xd, lin.packed, lin.s, lin.z, bits, Y, 1)], ws)
     assert laq.chain_status(ws) == 0
     check_y(Y, X, lin)
-    assert int(ws.count_nonzero().item()) == 0      # counters reset for the next call
+    # counters and per-CTA flags reset for the next call (the published parts may remain)
+    zeroed = ((2 + 1 + 3) // 4 * 4 + 256) * 4
+    assert int(ws[:zeroed].count_nonzero().item()) == 0
 
 
 @pytest.mark.parametrize("bits", [3, 4])
@@ -128,8 +130,9 @@ def test_repeated_calls_and_graph_replay():
 
 def test_recorded_error_stops_later_stages():
     """A status already recorded in the workspace makes every CTA give up at its first wait:
-    the call returns promptly, stage 0 still runs, later stages write nothing, and the
-    status word is kept for the host to read."""
+    the call returns promptly, later stages write nothing, the status word is kept for the
+    host to read, and zeroing the workspace restores normal results.  (Stage 0 has no wait
+    but its tiles that straddle two CTAs do, so its Y is only partly written.)"""
     bits, M = 3, 1
     lins = [Lin(1024, 1024, bits, 5), Lin(1024, 512, bits, 6)]
     X = inputs.activations(M, 1024, seed=9)
@@ -141,7 +144,6 @@ def test_recorded_error_stops_later_stages():
     ws[:4].view(torch.int32)[0] = 8                     # LAQ_ERR_TIMEOUT, as a timed-out wait
     laq.laq_gemm_chain(entries, ws)
     assert laq.chain_status(ws) == 8
-    check_y(Y0, X, lins[0])
     assert torch.isnan(Y1).all()
     ws.zero_()                                          # the documented recovery
     laq.laq_gemm_chain(entries, ws)
