@@ -54,6 +54,16 @@ __device__ __forceinline__ void cp_async_wait(int n) {
     }
 }
 
+// 16-byte load through L2 only (the data may have been written by other SMs).
+__device__ __forceinline__ uint4 ld_cg16(const void* p) {
+    uint4 v;
+    asm volatile("ld.global.cg.v4.u32 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "l"(p)
+                 : "memory");
+    return v;
+}
+
 __device__ __forceinline__ void pdl_wait() {
     asm volatile("griddepcontrol.wait;\n" ::: "memory");
 }

@@ -12,10 +12,10 @@
 //    an fp16 whose exponent field is 25 - p has the exact value 2^(10-p) + q, so one LOP3
 //    (mask | exponent) turns two codes of a 32-bit word into A-fragment values c + q with a
 //    per-field offset c = 2^(10-p).  The m16n8k16 MMA (fp16 in, fp32 accumulate) of these
-//    against raw x gives, per group g and MMA column, D = sum_k c_k x_k + sum_k q_k x_k.  Once
-//    X is staged, each CTA computes P_g = sum_k c_k x_k and S_g = sum_k x_k per (row, group)
-//    and a table {s, s (P_g + z S_g)} per (row, group, column), so the group epilogue applies
-//    Eq. (1) as  y_n += s_gn * D - s_gn * (P_g + z_gn * S_g)  (= sum_k x_k s (q - z)).
+//    against raw x gives, per group g and MMA column, D = sum_k c_k x_k + sum_k q_k x_k.  While
+//    X is staged, the 16 lanes that load a group's 256 bytes sum P_g = sum_k c_k x_k and
+//    S_g = sum_k x_k (shuffles), so the group epilogue applies Eq. (1) directly:
+//    y_n += s_gn * (D - P_g - z_gn * S_g)  (= sum_k x_k s (q - z)).
 //    The unpack costs about 0.7 integer ops per weight; nothing else touches a weight.
 //
 //  * Inside a record, lane c's rows are k = 32c + 4j + 2h + e, so its B fragments for the 8 k16
@@ -103,17 +103,15 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 2) gemm_kernel(const Params p)
     const int g1 = (int)((long long)p.G * (rank + 1) / C);
 
     // shared memory: ring [W][S][record] | x [M][GP][128] fp16 | zero block (64 B)
-    //                | s [gc][NT][16] fp16 | z [gc][NT][16] u8 | S, P [M][GP] fp32
-    //                | epilogue table [M][GP][NT][16] float2 | part [NT][MP][16] fp32
+    //                | s [gc][NT][16] fp16 | z [gc][NT][16] u8 | (S, P) [M][GP] float2
+    //                | part [NT][MP][16] fp32
     uint8_t* ring = smem;
     uint4* xs = reinterpret_cast<uint4*>(smem + (size_t)W * S * F::kBytes);
     uint4* zblk = xs + (size_t)M * GP * 16;
     uint16_t* s_sm = reinterpret_cast<uint16_t*>(zblk + 4);
     uint8_t* z_sm = reinterpret_cast<uint8_t*>(s_sm + (size_t)p.gc * NT * 16);
-    float* ssum = reinterpret_cast<float*>(z_sm + (size_t)p.gc * NT * 16);
-    float* psum = ssum + M * GP;
-    float2* ab = reinterpret_cast<float2*>(psum + M * GP);
-    float* part = reinterpret_cast<float*>(ab + (size_t)M * GP * NT * 16);
+    float2* ps = reinterpret_cast<float2*>(z_sm + (size_t)p.gc * NT * 16);
+    float* part = reinterpret_cast<float*>(ps + (size_t)M * GP);
     if (threadIdx.x < 4) zblk[threadIdx.x] = make_uint4(0u, 0u, 0u, 0u);
 
     const uint32_t ring_s = (uint32_t)__cvta_generic_to_shared(ring) +
@@ -179,70 +177,57 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 2) gemm_kernel(const Params p)
             __syncthreads();  // every warp is done reading the previous phase's X, S and P
         }
 
-        // Raw X of the phase (row b's groups pa..pb-1 are 256 * ng contiguous bytes), then
-        // S_g = sum_k x_k and P_g = sum_k c_k x_k per (row, group): 8 threads per group, each
-        // summing 16 consecutive rows, combined by shuffles.
+        // Raw X of the phase (row b's groups pa..pb-1 are 256 * ng contiguous bytes), through
+        // L2 into registers, then shared memory.  16-byte chunk u = (b, q) holds x[8q .. 8q+7]
+        // of group q / 16 of the phase, i.e. pairs 4 (q % 4) + w of that group for its four
+        // 32-bit words w; the 16 chunks of a group sit in 16 aligned lanes, which sum
+        // S_g = sum_k x_k and P_g = sum_k c_k x_k by shuffles.
         {
-            const uint32_t xs_s = (uint32_t)__cvta_generic_to_shared(xs);
-            for (int b = 0; b < M; ++b) {
-                const uint16_t* src = p.X + (size_t)b * p.K + (size_t)pa * 128;
-                const uint32_t dst = xs_s + (uint32_t)(b * GP * 256);
-                for (int u = threadIdx.x; u < ng * 16; u += blockDim.x)
-                    cp_async16(dst + u * 16, src + u * 8);
-            }
-            cp_async_commit();
-            asm volatile("cp.async.wait_all;\n" ::: "memory");
-            __syncthreads();
-            LAQ_TRACE(6);
-            const int seg = threadIdx.x & 7;
-            for (int base = 0; base < M * ng; base += (int)(blockDim.x >> 3)) {
-                const int blk = base + (int)(threadIdx.x >> 3);
-                float sx = 0.f, px = 0.f;
-                int b = 0, gl = 0;
-                if (blk < M * ng) {
-                    b = blk / ng;
-                    gl = blk - b * ng;
-                    const uint4* src = xs + (size_t)(b * GP + gl) * 16 + seg * 2;
+            const int per_row = ng * 16;
+            const int nch = M * per_row;  // a multiple of 16
+            for (int u0 = 0; u0 < nch; u0 += 4 * (int)blockDim.x) {
+                uint4 v[4];
 #pragma unroll
-                    for (int q = 0; q < 2; ++q) {
-                        const uint4 v = src[q];
-                        const uint32_t w4[4] = {v.x, v.y, v.z, v.w};
-#pragma unroll
-                        for (int e = 0; e < 4; ++e) {
-                            const float2 f = __half22float2(
-                                *reinterpret_cast<const __half2*>(&w4[e]));
-                            const float pair = f.x + f.y;
-                            sx += pair;
-                            px = fmaf(row_offset<BITS>((seg & 1) * 8 + q * 4 + e), pair, px);
-                        }
+                for (int r = 0; r < 4; ++r) {
+                    const int u = u0 + r * (int)blockDim.x + (int)threadIdx.x;
+                    if (u < nch) {
+                        const int b = u / per_row, q = u - b * per_row;
+                        v[r] = ld_cg16(p.X + (size_t)b * p.K + (size_t)pa * 128 + q * 8);
+                    } else {
+                        v[r] = make_uint4(0u, 0u, 0u, 0u);
                     }
                 }
 #pragma unroll
-                for (int o = 1; o < 8; o <<= 1) {
-                    sx += __shfl_xor_sync(0xffffffffu, sx, o);
-                    px += __shfl_xor_sync(0xffffffffu, px, o);
-                }
-                if (seg == 0 && blk < M * ng) {
-                    ssum[b * GP + gl] = sx;
-                    psum[b * GP + gl] = px;
+                for (int r = 0; r < 4; ++r) {
+                    // (warp-uniform) nothing of this batch for this warp
+                    if (u0 + r * (int)blockDim.x + warp * 32 >= nch) break;
+                    const int u = u0 + r * (int)blockDim.x + (int)threadIdx.x;
+                    const uint32_t w4[4] = {v[r].x, v[r].y, v[r].z, v[r].w};
+                    float sx = 0.f, px = 0.f;
+#pragma unroll
+                    for (int w = 0; w < 4; ++w) {
+                        const float2 f = __half22float2(*reinterpret_cast<const __half2*>(&w4[w]));
+                        const float pair = f.x + f.y;
+                        sx += pair;
+                        px = fmaf(row_offset<BITS>((u & 3) * 4 + w), pair, px);
+                    }
+#pragma unroll
+                    for (int o = 1; o < 16; o <<= 1) {
+                        sx += __shfl_xor_sync(0xffffffffu, sx, o);
+                        px += __shfl_xor_sync(0xffffffffu, px, o);
+                    }
+                    if (u < nch) {
+                        const int b = u / per_row, q = u - b * per_row;
+                        xs[(size_t)b * GP * 16 + q] = v[r];
+                        if ((q & 15) == 0) ps[b * GP + (q >> 4)] = make_float2(sx, px);
+                    }
                 }
             }
+            // the weights issued so far and the scales and zeros have landed
+            asm volatile("cp.async.wait_all;\n" ::: "memory");
             __syncthreads();
+            LAQ_TRACE(6);
             LAQ_TRACE(7);
-            // Epilogue table: {s, s * (z * S_g + P_g)} per (row b, group, tile, column), so the
-            // group epilogue is y += s * D - s * (P + z S), one shared load per output.
-            for (int idx = threadIdx.x; idx < M * ng * NT * 16; idx += blockDim.x) {
-                const int row = idx & 15, t = (idx >> 4) % NT, rest = (idx >> 4) / NT;
-                const int b = rest / ng, gl = rest - b * ng;
-                if (t < ntv) {
-                    const int e = ((pa - g0 + gl) * NT + t) * 16 + row;
-                    const float sv = __half2float(__ushort_as_half(s_sm[e]));
-                    const float corr =
-                        fmaf((float)z_sm[e], ssum[b * GP + gl], psum[b * GP + gl]);
-                    ab[((b * GP + gl) * NT + t) * 16 + row] = make_float2(sv, sv * corr);
-                }
-            }
-            __syncthreads();
             LAQ_TRACE(2);
         }
 
@@ -328,9 +313,12 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 2) gemm_kernel(const Params p)
                         const int giv = MP <= 8 ? col % GPA : 0;
                         if (b < M && ib + giv < nw) {
                             const int lg = team + (ib + giv) * WT;        // in the phase
-                            const float2 sa = ab[((b * GP + lg) * NT + tile) * 16 + R + 8 * (v >> 1)];
-                            const float d = D[0][h][v] + D[1][h][v];
-                            yacc[h][v] = fmaf(sa.x, d, yacc[h][v]) - sa.y;
+                            const int e = ((pa - g0 + lg) * NT + tile) * 16 + R + 8 * (v >> 1);
+                            const float sv = __half2float(__ushort_as_half(s_sm[e]));
+                            const float zv = (float)z_sm[e];
+                            const float2 sp = ps[b * GP + lg];  // (S, P) of the group
+                            const float d = D[0][h][v] + D[1][h][v] - sp.y;
+                            yacc[h][v] = fmaf(sv, fmaf(-zv, sp.x, d), yacc[h][v]);
                         }
                     }
                 }
@@ -443,8 +431,8 @@ size_t gemm_smem_bytes(const GemmLaunch& L, int* groups_per_phase) {
     const size_t ring = (size_t)L.warps * L.stages * rec;
     const int G = L.K / 128;
     const int gc = (G + L.cluster - 1) / L.cluster;
-    // raw X, S and P, and the epilogue table of one group
-    const size_t per_group = (size_t)L.M * (256 + 8 + (size_t)L.tiles_per_cta * 128);
+    // raw X and (S, P) of one group
+    const size_t per_group = (size_t)L.M * (256 + 8);
     int gpp = (int)(kXsBudget / per_group);
     if (gpp > gc) gpp = gc;
     if (gpp < 1) gpp = 1;
