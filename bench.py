@@ -62,16 +62,17 @@ def load_peaks():
     return 6800.0, "fallback"
 
 
-def traffic_for(kernel, a):
-    """DRAM bytes per launch of ``kernel`` measured by ncu (profiles/traffic.json), or None when
-    no capture exists for this kernel and workload or the kernel's source changed since."""
+def traffic_for(kernel, a, variant):
+    """DRAM bytes per launch of ``kernel`` in pass form ``variant``, measured by ncu
+    (profiles/traffic.json), or None when no capture exists for this kernel and workload or the
+    kernel's source changed since."""
     import hashlib
     path = os.path.join(ROOT, "profiles", "traffic.json")
     if not os.path.exists(path):
         return None
     with open(path) as f:
         table = json.load(f)
-    entry = table.get(f"{kernel} {a.model} W{a.bits} M={a.M}")
+    entry = table.get(f"{kernel} {a.model} W{a.bits} M={a.M} {variant}")
     if not entry:
         return None
     h = hashlib.sha256()
@@ -527,7 +528,7 @@ def run_laq(a, world, rank, local):
                    "speedup_vs_fp16_torch": (fp16_us / (ms_per_step * 1e3)) if fp16_us else None,
                    "parallelism": f"replicas x{world}"},
         "roofline": {"bound": "hbm", "achieved": kernel_gbs, "peak": peak, "unit": "GB/s",
-                     "frac": kernel_gbs / peak, "traffic": traffic_for(dom[0], a),
+                     "frac": kernel_gbs / peak, "traffic": traffic_for(dom[0], a, head),
                      "kernel": dom[0], "launches_per_step": dom[1],
                      "us_per_launch": dom[3] / dom[1], "bytes_per_launch": dom[2] / dom[1],
                      "peak_kind": peak_kind,

@@ -83,7 +83,8 @@ laq_status check_gemm_args(const void* X, int64_t M, int64_t K, int64_t N, const
 
 laq_status check_config(const laq_gemm_config* c) {
     if (!c) return LAQ_ERR_NULL;
-    if (c->tiles_per_cta != 1 && c->tiles_per_cta != 2 && c->tiles_per_cta != 4)
+    if (c->tiles_per_cta != 1 && c->tiles_per_cta != 2 && c->tiles_per_cta != 4 &&
+        c->tiles_per_cta != 8)
         return LAQ_ERR_CONFIG;
     if (c->warps < 1 || c->warps > 8) return LAQ_ERR_CONFIG;
     if (c->warps % c->tiles_per_cta) return LAQ_ERR_CONFIG;  // whole warps per tile

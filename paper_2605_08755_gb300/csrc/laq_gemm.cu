@@ -401,7 +401,8 @@ KernelFn pick_nt(int nt) {
     switch (nt) {
         case 1: return gemm_kernel<BITS, MP, 1>;
         case 2: return gemm_kernel<BITS, MP, 2>;
-        default: return gemm_kernel<BITS, MP, 4>;
+        case 4: return gemm_kernel<BITS, MP, 4>;
+        default: return gemm_kernel<BITS, MP, 8>;
     }
 }
 
@@ -418,9 +419,9 @@ KernelFn pick_mp(int mp, int nt) {
 
 int mp_class(int M) { return M <= 1 ? 1 : M <= 2 ? 2 : M <= 4 ? 4 : M <= 8 ? 8 : 16; }
 int mp_index(int mp) { return mp == 1 ? 0 : mp == 2 ? 1 : mp == 4 ? 2 : mp == 8 ? 3 : 4; }
-int nt_index(int nt) { return nt == 1 ? 0 : nt == 2 ? 1 : 2; }
+int nt_index(int nt) { return nt == 1 ? 0 : nt == 2 ? 1 : nt == 4 ? 2 : 3; }
 
-std::atomic<size_t> g_attr_limit[2][5][3];  // max dynamic smem already granted per kernel
+std::atomic<size_t> g_attr_limit[2][5][4];  // max dynamic smem already granted per kernel
 
 constexpr size_t kXsBudget = 64 * 1024;  // shared memory for staged X (and its tables) per phase
 

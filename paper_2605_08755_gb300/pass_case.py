@@ -1,0 +1,55 @@
+"""One form of the decode-step weight pass, replayed a few times: the case for profiling a pass.
+
+    python -m paper_2605_08755_gb300.pass_case --variant graph_fused --bits 3 --M 1 --replays 3
+
+Builds the Qwen3-4B-shaped pass (36 layers, synthetic weights) in one of its four forms
+(``graph_252``, ``graph_fused``, ``chain_252``, ``chain_fused``), captures it into a CUDA graph
+(the capture is preceded by one eager run of the pass), replays the graph ``replays`` times and
+prints the mean device time per replay.  Under a profiler, the first replay's kernels follow the
+eager run's: for a graph form, ``-k regex:gemm_kernel -s L -c L`` with L = the printed
+``launches`` selects exactly the first replay; for a chain form, ``-k regex:chain_kernel -s 1
+-c 1`` does.
+"""
+import argparse
+import json
+
+import torch
+
+from .weight_pass import WeightPass
+
+VARIANTS = {"graph_252": (False, False), "graph_fused": (True, False),
+            "chain_252": (False, True), "chain_fused": (True, True)}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--variant", default="graph_fused", choices=sorted(VARIANTS))
+    ap.add_argument("--model", default="qwen3-4b", choices=["qwen3-4b", "qwen3-8b"])
+    ap.add_argument("--bits", type=int, default=3, choices=[3, 4])
+    ap.add_argument("--M", type=int, default=1)
+    ap.add_argument("--layers", type=int, default=36)
+    ap.add_argument("--replays", type=int, default=3)
+    a = ap.parse_args()
+    fuse, chain = VARIANTS[a.variant]
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    wp = WeightPass(model=a.model, bits=a.bits, M=a.M, layers=a.layers, device=dev,
+                    outliers=(a.model == "qwen3-8b"), fuse=fuse, chain=chain)
+    stream = torch.cuda.Stream(dev)
+    g = wp.capture(stream=stream)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        e0.record(stream)
+        for _ in range(a.replays):
+            g.replay()
+        e1.record(stream)
+    torch.cuda.synchronize(dev)
+    us = e0.elapsed_time(e1) * 1e3 / a.replays
+    print(json.dumps({"variant": a.variant, "bits": a.bits, "M": a.M, "layers": a.layers,
+                      "launches": wp.launches, "bytes_per_pass": wp.bytes_per_pass(),
+                      "us_per_pass": us, "gbs": wp.bytes_per_pass() / (us * 1e-6) / 1e9,
+                      "configs": [c.as_dict() for c in wp.configs[:4 if fuse else 7]]}))
+
+
+if __name__ == "__main__":
+    main()

@@ -93,6 +93,7 @@ def test_gemm_config_validation(L):
         return L.laq_gemm_wxg128_config(FAKE, 1, 256, 32, FAKE, FAKE, FAKE, 3, FAKE,
                                         ctypes.byref(cfg), None)
     assert run(tiles_per_cta=3) == 9
+    assert run(tiles_per_cta=16) == 9
     assert run(warps=0) == 9
     assert run(warps=9) == 9
     assert run(cluster=3) == 9
@@ -132,7 +133,7 @@ def test_plan_is_valid_for_every_workload_shape(L, bits, M):
     for K, N in sorted(shapes):
         for sms in (152, 148, 1):
             c = laq.laq_gemm_plan(M, K, N, bits, sms)
-            assert c.tiles_per_cta in (1, 2, 4)
+            assert c.tiles_per_cta in (1, 2, 4, 8)
             assert 1 <= c.warps <= 8
             assert c.cluster in (1, 2, 4, 8) and c.cluster <= max(1, K // 128)
             assert 2 <= c.stages <= 16

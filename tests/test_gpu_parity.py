@@ -124,7 +124,7 @@ def test_gemm_parity_shapes(bits, M, K, N):
 
 
 CONFIGS = [laq.GemmConfig.make(nt, w, cl, st, pdl)
-           for nt, w, cl, st, pdl in itertools.product((1, 2, 4), (1, 2, 3, 4, 8), (1, 2, 8), (2, 3, 16),
+           for nt, w, cl, st, pdl in itertools.product((1, 2, 4, 8), (1, 2, 3, 4, 8), (1, 2, 8), (2, 3, 16),
                                                        (0, 1))]
 
 
@@ -133,10 +133,10 @@ SMEM_OPTIN = 232448   # bytes of dynamic shared memory a CTA may opt into on sm_
 
 def smem_needed(M, K, bits, cfg):
     """Mirror of the library's shared-memory budget: per-warp cp.async rings, staged X with its
-    group sums (up to 48 KB per phase), zero block, scales and zeros, per-CTA partial sums."""
+    group sums (up to 64 KB per phase), zero block, scales and zeros, per-CTA partial sums."""
     rec = 1024 if bits == 4 else 768
     gc = -(-(K // 128) // cfg.cluster)
-    per_group = M * (264 + cfg.tiles_per_cta * 128)
+    per_group = M * 264
     gpp = max(1, min(gc, 64 * 1024 // per_group))
     mp = 1 if M <= 1 else 2 if M <= 2 else 4 if M <= 4 else 8 if M <= 8 else 16
     return (cfg.warps * cfg.stages * rec + gpp * per_group + 64 + gc * cfg.tiles_per_cta * 48
