@@ -4,6 +4,7 @@
 #include <stdint.h>
 
 #include <atomic>
+#include <climits>
 #include <vector>
 
 #include "laq.h"
@@ -97,37 +98,45 @@ laq_status check_config(const laq_gemm_config* c) {
 
 int ceil_div(int64_t a, int64_t b) { return (int)((a + b - 1) / b); }
 
-// Launch-shape plan.  The kernel streams each 16-column x 128-row record once, so the plan is
-// about keeping HBM busy: (1) enough CTAs to occupy every SM -- the largest tiles-per-CTA and
-// the smallest cluster (K split) that still give at least one CTA per SM; (2) eight warps
-// (fewer when a CTA owns fewer than eight groups); (3) a cp.async ring deep enough that each
-// warp keeps all but one of its groups in flight (up to 7 records per tile), capped so the ring
-// stays within 96 KB and two CTAs can share an SM.
+// Launch-shape plan: tiles per CTA (NT), K split over a cluster (C), warps and ring depth.
+//  * M = 1: the cheapest split by estimated SM time -- records per warp, x 1.3 when two CTAs
+//    share an SM (16 warps retire a record in ~0.65x the time of 8; measured on GB300), x 1.02
+//    for a cluster's reduction -- over NT, C in {1, 2, 4, 8} with at most two CTAs per SM.
+//  * M > 1: every CTA reads X for its whole K range, M rows of it -- at M = 16 with one tile
+//    per CTA that is 5x the CTA's weight bytes (b = 3).  So X is shared across 4 (M <= 4) or 8
+//    tiles per CTA and K is split over a cluster (which also splits X) until there is about one
+//    CTA per SM: 40-45% faster than the M = 1 rule on the Qwen3-4B pass at M = 4..16.
+//  * Eight warps (fewer when a CTA owns fewer groups), and a cp.async ring deep enough to hold
+//    all of a warp's records (at most 16) within 100 KB.
 void plan(int64_t M, int64_t K, int64_t N, int bits, int sms, laq_gemm_config* out) {
     const int64_t T = N / 16, G = K / kGroup;
-    const int mp = M <= 1 ? 1 : M <= 2 ? 2 : M <= 4 ? 4 : M <= 8 ? 8 : 16;
     const int64_t rec = bits == 4 ? 1024 : 768;
-    const int nts[3] = {4, 2, 1};
-    const int cls[4] = {1, 2, 4, 8};
-    int best_nt = 1, best_cl = 1;
-    int64_t best_ctas = -1;
-    bool found = false;
-    for (int b = 0; b < 4 && !found; ++b) {
-        const int cl = cls[b];
-        if (cl > 1 && cl > G) break;
-        for (int a = 0; a < 3; ++a) {
-            const int nt = nts[a];
-            const int64_t ctas = (int64_t)ceil_div(T, nt) * cl;
-            if (ctas >= sms) {
-                best_nt = nt;
-                best_cl = cl;
-                found = true;
-                break;
-            }
-            if (ctas > best_ctas) {
-                best_ctas = ctas;
-                best_nt = nt;
-                best_cl = cl;
+    int best_nt = 8, best_cl = 1;
+    if (M > 1) {
+        int nt = M <= 4 ? 4 : 8;
+        while (nt > 1 && ceil_div(T, nt) < sms / 8) nt /= 2;
+        int cl = 1;
+        while (cl < 8 && cl * 2 <= G && (int64_t)ceil_div(T, nt) * cl < sms) cl *= 2;
+        best_nt = nt;
+        best_cl = cl;
+    } else {
+        double best_cost = 1e300;
+        int64_t best_ctas = INT64_MAX;
+        for (int cl = 1; cl <= 8; cl *= 2) {
+            if (cl > 1 && cl > G) break;
+            for (int nt = 1; nt <= 8; nt *= 2) {
+                const int64_t ctas = (int64_t)ceil_div(T, nt) * cl;
+                if (ctas > 2 * (int64_t)sms) continue;
+                const int64_t gc = (G + cl - 1) / cl;
+                const int64_t per_warp = (gc + (8 / nt) - 1) / (8 / nt);
+                const double cost =
+                    (double)per_warp * (ctas > sms ? 1.3 : 1.0) * (cl > 1 ? 1.02 : 1.0);
+                if (cost < best_cost - 1e-9 || (cost < best_cost + 1e-9 && ctas < best_ctas)) {
+                    best_cost = cost;
+                    best_ctas = ctas;
+                    best_nt = nt;
+                    best_cl = cl;
+                }
             }
         }
     }
