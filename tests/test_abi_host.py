@@ -204,3 +204,16 @@ def test_chain_static_argument_validation(L):
     assert L.laq_gemm_chain_static(arr, _lib.CHAIN_MAX + 1, None) == code["LAQ_ERR_WORKSPACE"]
     assert L.laq_gemm_chain_static(arr, -1, None) == code["LAQ_ERR_WORKSPACE"]
     assert L.laq_gemm_chain_static(None, 1, None) == code["LAQ_ERR_NULL"]
+
+
+def test_plan_shares_x_across_tiles_at_m_above_one(L):
+    # M > 1: 4 (M <= 4) or 8 tiles per CTA, and a cluster K split towards one CTA per SM
+    c = laq.laq_gemm_plan(4, 9728, 2560, 3, 152)
+    assert (c.tiles_per_cta, c.cluster) == (4, 4)
+    c = laq.laq_gemm_plan(16, 2560, 19456, 3, 152)
+    assert (c.tiles_per_cta, c.cluster) == (8, 1)
+    c = laq.laq_gemm_plan(16, 9728, 2560, 3, 152)
+    assert (c.tiles_per_cta, c.cluster) == (8, 8)
+    # M = 1: the fused Qwen3-4B projections
+    assert laq.laq_gemm_plan(1, 2560, 19456, 3, 152).tiles_per_cta == 4
+    assert laq.laq_gemm_plan(1, 9728, 2560, 3, 152).tiles_per_cta == 1
