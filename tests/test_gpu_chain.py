@@ -197,3 +197,70 @@ def test_qwen3_8b_fused_pass_chain_w3_m1():
     torch.cuda.synchronize()
     assert laq.chain_status(wp.ws) == 0
     _sampled(wp, layers={0, 35})
+
+
+def test_stage_of_many_small_entries():
+    """One stage of 20 entries with K = 128..640 and N = 16..80 (single-group and single-tile
+    GEMVs, several X slots per CTA), then a stage reading one of their outputs, at M = 2."""
+    bits, M = 4, 2
+    rng = np.random.default_rng(3)
+    dims = [(128 * int(rng.integers(1, 6)), 16 * int(rng.integers(1, 6))) for _ in range(20)]
+    dims[7] = (dims[7][0], 128)   # its output is the last entry's X: K must be a multiple of 128
+    lins = [Lin(K, N, bits, seed=300 + i) for i, (K, N) in enumerate(dims)]
+    Xs = [inputs.activations(M, K, seed=400 + i) for i, (K, _) in enumerate(dims)]
+    Xd = [torch.from_numpy(X).cuda() for X in Xs]
+    Ys = [nan_like(M, N) for _, N in dims]
+    last = Lin(dims[7][1], 48, bits, seed=399)
+    Ylast = nan_like(M, 48)
+    entries = [(Xd[i], lins[i].packed, lins[i].s, lins[i].z, bits, Ys[i], 1 if i == 0 else 0)
+               for i in range(20)]
+    entries.append((Ys[7], last.packed, last.s, last.z, bits, Ylast, 1))
+    ws = laq.chain_workspace(len(entries), "cuda")
+    laq.laq_gemm_chain(entries, ws)
+    assert laq.chain_status(ws) == 0
+    refs = [check_y(Ys[i], Xs[i], lins[i]) for i in range(20)]
+    check_y(Ylast, refs[7].astype(np.float16), last)
+
+
+def test_split_stage_with_tiles_straddling_entries():
+    """Two entries of 80 tiles x 76 groups in one stage (160 tiles on the GPU's SMs: the stage
+    is split by records, so tiles straddle CTAs, some next to the entry boundary)."""
+    bits, M = 3, 1
+    lins = [Lin(9728, 1280, bits, seed=500 + i) for i in range(2)]
+    Xs = [inputs.activations(M, 9728, seed=510 + i) for i in range(2)]
+    Ys = [nan_like(M, 1280) for _ in range(2)]
+    entries = [(torch.from_numpy(Xs[i]).cuda(), lins[i].packed, lins[i].s, lins[i].z, bits,
+                Ys[i], 1 if i == 0 else 0) for i in range(2)]
+    ws = laq.chain_workspace(2, "cuda")
+    for _ in range(2):     # twice: the published parts and flags are reused
+        for Y in Ys:
+            Y.fill_(float("nan"))
+        laq.laq_gemm_chain(entries, ws)
+        assert laq.chain_status(ws) == 0
+        for i in range(2):
+            check_y(Ys[i], Xs[i], lins[i])
+
+
+def test_longest_chain():
+    """LAQ_CHAIN_MAX entries of one record each (K = 128, N = 16) in 128 stages of three, through
+    both the workspace and the static-scratch entry points: the longest parameter block, the
+    most stage counters, and 152 CTAs of which most own no record of a stage."""
+    bits, M = 3, 1
+    n = laq._lib.CHAIN_MAX
+    lins = [Lin(128, 16, bits, seed=600 + i) for i in range(3)]
+    Xs = [inputs.activations(M, 128, seed=700 + i) for i in range(n)]
+    Xd = [torch.from_numpy(X).cuda() for X in Xs]
+    Ys = [nan_like(M, 16) for _ in range(n)]
+    entries = [(Xd[i], lins[i % 3].packed, lins[i % 3].s, lins[i % 3].z, bits, Ys[i],
+                1 if i % 3 == 0 else 0) for i in range(n)]
+    spec = laq.Chain(entries)
+    ws = laq.chain_workspace(n, "cuda")
+    for run in (lambda: spec.run(ws), lambda: spec.run_static()):
+        for Y in Ys:
+            Y.fill_(float("nan"))
+        run()
+        torch.cuda.synchronize()
+        assert all(not torch.isnan(Y).any() for Y in Ys)
+        for i in range(0, n, 37):
+            check_y(Ys[i], Xs[i], lins[i % 3])
+    assert laq.chain_status(ws) == 0
