@@ -106,12 +106,19 @@ int ceil_div(int64_t a, int64_t b) { return (int)((a + b - 1) / b); }
 //    per CTA that is 5x the CTA's weight bytes (b = 3).  So X is shared across 4 (M <= 4) or 8
 //    tiles per CTA and K is split over a cluster (which also splits X) until there is about one
 //    CTA per SM: 40-45% faster than the M = 1 rule on the Qwen3-4B pass at M = 4..16.
-//  * Eight warps (fewer when a CTA owns fewer groups), and a cp.async ring deep enough to hold
-//    all of a warp's records (at most 16) within 100 KB.
+//  * M = 1 with fewer than two tiles per SM (N < 32 x SMs) and a long K, where that plan
+//    leaves a warp more than 5 records (the 2560 x 9728 down projection: 160 tiles on 152 SMs,
+//    ~10 records per warp): 4-warp CTAs of 2 tiles instead, K split over a cluster that
+//    doubles until a warp holds at most 5 records and the grid covers every SM (down: 640
+//    CTAs, 5 records per warp; measured on GB300 in the Qwen3-4B pass, W3 and W4: 1.6 us less
+//    per down launch).  Shorter K (o, q, k, v) measured best with the rule above.
+//  * Eight warps otherwise (fewer when a CTA owns fewer groups), and a cp.async ring deep
+//    enough to hold all of a warp's records (at most 16) within 100 KB.
 void plan(int64_t M, int64_t K, int64_t N, int bits, int sms, laq_gemm_config* out) {
     const int64_t T = N / 16, G = K / kGroup;
     const int64_t rec = bits == 4 ? 1024 : 768;
     int best_nt = 8, best_cl = 1;
+    int64_t warps_max = 8;
     if (M > 1) {
         int nt = M <= 4 ? 4 : 8;
         while (nt > 1 && ceil_div(T, nt) < sms / 8) nt /= 2;
@@ -139,9 +146,20 @@ void plan(int64_t M, int64_t K, int64_t N, int bits, int sms, laq_gemm_config* o
                 }
             }
         }
+        const int64_t gc8 = (G + best_cl - 1) / best_cl;
+        const int64_t wt8 = gc8 < 8 / best_nt ? gc8 : 8 / best_nt;
+        if (T >= 2 && T < 2 * (int64_t)sms && (gc8 + wt8 - 1) / wt8 > 5) {
+            best_nt = 2;
+            best_cl = 1;
+            warps_max = 4;
+            while (best_cl < 8 && 2 * best_cl <= G &&
+                   ((int64_t)best_nt * ((G + best_cl - 1) / best_cl) > 5 * warps_max ||
+                    (int64_t)ceil_div(T, best_nt) * best_cl < sms))
+                best_cl *= 2;
+        }
     }
     const int64_t gc = (G + best_cl - 1) / best_cl;
-    const int64_t wt_max = 8 / best_nt;                        // warps per tile
+    const int64_t wt_max = warps_max / best_nt;                // warps per tile
     const int64_t wt = gc < wt_max ? (gc < 1 ? 1 : gc) : wt_max;
     const int w = (int)(wt * best_nt);
     const int64_t iters = (gc + wt - 1) / wt;

@@ -216,4 +216,20 @@ def test_plan_shares_x_across_tiles_at_m_above_one(L):
     assert (c.tiles_per_cta, c.cluster) == (8, 8)
     # M = 1: the fused Qwen3-4B projections
     assert laq.laq_gemm_plan(1, 2560, 19456, 3, 152).tiles_per_cta == 4
-    assert laq.laq_gemm_plan(1, 9728, 2560, 3, 152).tiles_per_cta == 1
+    assert laq.laq_gemm_plan(1, 2560, 6144, 3, 152).tiles_per_cta == 2
+
+
+@pytest.mark.parametrize("bits", [3, 4])
+def test_plan_splits_k_of_narrow_outputs_at_m_one(L, bits):
+    # Fewer than two 16-column tiles per SM and a K long enough that 8-warp CTAs would leave a
+    # warp more than 5 records: 4-warp CTAs of 2 tiles, K split over a cluster until a warp
+    # holds at most 5 records and the grid covers every SM.
+    for K, N, cl in ((9728, 2560, 8), (12288, 4096, 8)):
+        c = laq.laq_gemm_plan(1, K, N, bits, 152)
+        assert (c.tiles_per_cta, c.warps, c.cluster) == (2, 4, cl), (K, N, c.as_dict())
+        per_warp = c.tiles_per_cta * -(-(K // 128) // c.cluster) / c.warps
+        assert per_warp <= 5 or c.cluster == 8
+        assert (N // 16 + 1) // 2 * c.cluster >= 152 or c.cluster == 8
+    # shorter K (o, q, k, v of Qwen3-4B) and wide outputs keep 8-warp CTAs
+    for K, N in ((4096, 2560), (2560, 4096), (2560, 1024), (2560, 19456), (2560, 6144)):
+        assert laq.laq_gemm_plan(1, K, N, bits, 152).warps >= 5, (K, N)
