@@ -62,10 +62,11 @@ def load_peaks():
     return 6800.0, "fallback"
 
 
-def traffic_for(kernel, a, variant):
+def traffic_for(kernel, a, variant, shapes=None):
     """DRAM bytes per launch of ``kernel`` in pass form ``variant``, measured by ncu
-    (profiles/traffic.json), or None when no capture exists for this kernel and workload or the
-    kernel's source changed since."""
+    (profiles/traffic.json), or None when no capture exists for this kernel and workload, the
+    kernel's source changed since, or the instance now runs other projections (``shapes``: the
+    sorted [K, N, launches] of its launches in one step)."""
     import hashlib
     path = os.path.join(ROOT, "profiles", "traffic.json")
     if not os.path.exists(path):
@@ -74,6 +75,8 @@ def traffic_for(kernel, a, variant):
         table = json.load(f)
     entry = table.get(f"{kernel} {a.model} W{a.bits} M={a.M} {variant}")
     if not entry:
+        return None
+    if shapes is not None and entry.get("shapes") != shapes:
         return None
     h = hashlib.sha256()
     for name in entry["sources"]:
@@ -342,7 +345,7 @@ def time_graph(graph, stream, reps, dev):
 def kernel_breakdown(wp, stream, dev, reps=200):
     """Per GEMM kernel instance (bits, M class, tiles per CTA): a CUDA graph of all of its
     launches of one step, in pass order, timed on the stream they run on; returns rows of
-    (instance, launches, algorithmic bytes per step, us per step)."""
+    (instance, launches, algorithmic bytes per step, us per step, [[K, N, launches], ...])."""
     import torch
     from paper_2605_08755_gb300 import _lib
     mp = 1 if wp.M <= 1 else 2 if wp.M <= 2 else 4 if wp.M <= 4 else 8 if wp.M <= 8 else 16
@@ -362,7 +365,11 @@ def kernel_breakdown(wp, stream, dev, reps=200):
             run(stream)
         ms = time_graph(g, stream, reps, dev)
         nbytes = sum(wp.linears[i][3].bytes_per_call(wp.M) for i in idxs)
-        rows.append((key, len(idxs), nbytes, ms * 1e3))
+        shapes = {}
+        for i in idxs:
+            kn = (wp.linears[i][3].K, wp.linears[i][3].N)
+            shapes[kn] = shapes.get(kn, 0) + 1
+        rows.append((key, len(idxs), nbytes, ms * 1e3, [[k, n, c] for (k, n), c in sorted(shapes.items())]))
         del g
     return rows
 
@@ -461,7 +468,7 @@ def run_laq(a, world, rank, local):
     # most device time (per-instance graphs of the step's launches, timed on their stream).
     if wp.chain:
         rows = [("chain_kernel<%d, %d>" % (a.bits, 1 if a.M <= 1 else 2 if a.M <= 2 else 4),
-                 1, bytes_step, ms_per_step * 1e3)]
+                 1, bytes_step, ms_per_step * 1e3, None)]
     else:
         rows = kernel_breakdown(wp, stream, dev)
     dom = max(rows, key=lambda r: r[3])
@@ -528,12 +535,13 @@ def run_laq(a, world, rank, local):
                    "speedup_vs_fp16_torch": (fp16_us / (ms_per_step * 1e3)) if fp16_us else None,
                    "parallelism": f"replicas x{world}"},
         "roofline": {"bound": "hbm", "achieved": kernel_gbs, "peak": peak, "unit": "GB/s",
-                     "frac": kernel_gbs / peak, "traffic": traffic_for(dom[0], a, head),
+                     "frac": kernel_gbs / peak, "traffic": traffic_for(dom[0], a, head, dom[4]),
                      "kernel": dom[0], "launches_per_step": dom[1],
                      "us_per_launch": dom[3] / dom[1], "bytes_per_launch": dom[2] / dom[1],
                      "peak_kind": peak_kind,
                      "instances": [{"kernel": k, "launches": n, "us_per_step": us,
-                                    "gbs": nb / (us * 1e-6) / 1e9} for k, n, nb, us in rows]},
+                                    "gbs": nb / (us * 1e-6) / 1e9, "shapes": sh}
+                                   for k, n, nb, us, sh in rows]},
         "cpu_baseline": cpu,
         "e2e": {"value": e2e_gbs, "unit": "GB/s", "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h, "us_per_step": e2e_ms * 1e3},

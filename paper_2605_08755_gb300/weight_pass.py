@@ -42,6 +42,21 @@ FUSED = (("qkv", ("q", "k", "v")), ("o", ("o",)), ("gate_up", ("gate", "up")), (
 SHARES_INPUT = {"k", "v", "up"}
 
 
+def pass_plan(model, fuse, layers):
+    """The pass's GEMVs in launch order: (layer, member projection indices, name, K, N)."""
+    names = [n for n, _, _ in shapes(model)]
+    groups = ([[names.index(m) for m in members] for _, members in FUSED] if fuse
+              else [[i] for i in range(len(names))])
+    gnames = [n for n, _ in FUSED] if fuse else names
+    plan = []
+    for layer in range(layers):
+        for gname, members in zip(gnames, groups):
+            K = shapes(model)[members[0]][1]
+            N = sum(shapes(model)[i][2] for i in members)
+            plan.append((layer, tuple(members), gname, K, N))
+    return plan
+
+
 class WeightPass:
     """The 7 x layers projections of a decode step, launched in stream order.
 
@@ -60,16 +75,7 @@ class WeightPass:
         self.model, self.bits, self.M, self.layers = model, bits, M, layers
         self.seed, self.outliers, self.fuse, self.chain = seed, outliers, fuse, chain
         self.device = torch.device(device)
-        names = [n for n, _, _ in shapes(model)]
-        groups = ([[names.index(m) for m in members] for _, members in FUSED] if fuse
-                  else [[i] for i in range(len(names))])
-        gnames = [n for n, _ in FUSED] if fuse else names
-        plan = []
-        for layer in range(layers):
-            for gname, members in zip(gnames, groups):
-                K = shapes(model)[members[0]][1]
-                N = sum(shapes(model)[i][2] for i in members)
-                plan.append((layer, tuple(members), gname, K, N))
+        plan = pass_plan(model, fuse, layers)
         xs = sum(M * K for *_, K, N in plan)
         ys = sum(M * N for *_, K, N in plan)
         self.Xbuf = torch.empty((xs,), dtype=torch.float16, device=self.device)
