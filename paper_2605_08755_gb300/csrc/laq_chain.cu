@@ -146,27 +146,40 @@ __device__ __forceinline__ float ld_cg_f32(const float* p) {
 }
 
 // Wait until *cnt >= target.  Returns false when an error is already recorded in the status
-// word (checked first, so a recorded error stops every later stage), or when the wait runs out
-// (after recording LAQ_ERR_TIMEOUT).
+// word (read together with the first poll, so a recorded error stops every later stage; while
+// waiting it is re-read every 32 polls, so that each poll is one L2 round trip), or when the
+// wait runs out (after recording LAQ_ERR_TIMEOUT).
 __device__ bool wait_count(const uint32_t* cnt, uint32_t target, uint32_t* status) {
     const unsigned long long t0 = globaltimer();
+    const uint32_t st0 = ld_relaxed(status);
+    const uint32_t c0 = ld_acquire(cnt);
+    if (st0 != 0u) return false;
+    if (c0 >= target) return true;
     for (int spin = 0; spin < kWaitSpins; ++spin) {
-        if (ld_relaxed(status) != 0u) return false;
         if (ld_acquire(cnt) >= target) return true;
-        if ((spin & 31) == 31 && globaltimer() - t0 > kWaitNs) break;
+        if ((spin & 31) == 31) {
+            if (ld_relaxed(status) != 0u) return false;
+            if (globaltimer() - t0 > kWaitNs) break;
+        }
     }
     atomicCAS(status, 0u, (uint32_t)LAQ_ERR_TIMEOUT);
     return false;
 }
 
-// Wait until *flag == value (a CTA's published part of stage value - 1), with the limits of
-// wait_count.
+// Wait until *flag == value (a CTA's published part of stage value - 1), with the limits and
+// the status checks of wait_count.
 __device__ bool wait_flag(const uint32_t* flag, uint32_t value, uint32_t* status) {
     const unsigned long long t0 = globaltimer();
+    const uint32_t st0 = ld_relaxed(status);
+    const uint32_t f0 = ld_acquire(flag);
+    if (st0 != 0u) return false;
+    if (f0 == value) return true;
     for (int spin = 0; spin < kWaitSpins; ++spin) {
-        if (ld_relaxed(status) != 0u) return false;
         if (ld_acquire(flag) == value) return true;
-        if ((spin & 31) == 31 && globaltimer() - t0 > kWaitNs) break;
+        if ((spin & 31) == 31) {
+            if (ld_relaxed(status) != 0u) return false;
+            if (globaltimer() - t0 > kWaitNs) break;
+        }
     }
     atomicCAS(status, 0u, (uint32_t)LAQ_ERR_TIMEOUT);
     return false;

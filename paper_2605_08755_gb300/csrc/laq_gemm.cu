@@ -234,96 +234,102 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 2) gemm_kernel(const Params p)
         // Batch row and group column of this lane's B fragment (MMA column R).
         const int bl = MP <= 8 ? R / GPA : R;
         const int gil = MP <= 8 ? R % GPA : 0;
+        // X of the lane's B column for the warp's record i: uint4 offset xo0[h] + i * xstep.
+        const int xstep = WT * 16;
+        int xo0[NH];
+#pragma unroll
+        for (int h = 0; h < NH; ++h) xo0[h] = ((bl + 8 * h) * GP + team) * 16 + c * 4;
 
-        float D[2][NH][4];  // two independent accumulator chains (even / odd k16 steps)
         int rslot = 0;
-        // With S - 1 >= nw every record of the warp was copied in the prologue and has landed.
+        // With S - 1 >= nw every record of the warp was copied in the prologue and has landed;
+        // record i then sits in slot i.
         const bool streaming = S - 1 < nw;
-        for (int i = 0; i < nw; ++i) {
-            LAQ_TRACE_LOOP(0, i);
-            if (streaming) {
-                issue(i + S - 1);
-                cp_async_wait(S - 1);
-            }
-            LAQ_TRACE_LOOP(1, i);
-
-            const int gi = GPA > 1 ? i % GPA : 0;
-            const int gl = team + i * WT;  // group index within the phase
-            if (gi == 0) {
+        // Records in blocks of GPA (the groups sharing one accumulator); the position in the
+        // block is a compile-time constant, so slot, X and scale offsets fold into immediates.
+        for (int i0 = 0; i0 < nw; i0 += GPA) {
+            float D[2][NH][4];  // two independent accumulator chains (even / odd k16 steps)
 #pragma unroll
-                for (int a = 0; a < 2; ++a)
+            for (int a = 0; a < 2; ++a)
 #pragma unroll
-                    for (int h = 0; h < NH; ++h)
+                for (int h = 0; h < NH; ++h)
 #pragma unroll
-                        for (int v = 0; v < 4; ++v) D[a][h][v] = 0.f;
-            }
-
-            // B fragments: x[32c .. 32c+31] of this group for lanes whose column belongs to
-            // it, zeros for the others.
-            uint32_t B[NH][8][2];
+                    for (int v = 0; v < 4; ++v) D[a][h][v] = 0.f;
 #pragma unroll
-            for (int h = 0; h < NH; ++h) {
-                const int b = bl + 8 * h;
-                const bool act = gil == gi && b < M;
-                const uint4* src = act ? xs + (size_t)(b * GP + gl) * 16 + c * 4 : zblk;
-#pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    const uint4 v = src[q];
-                    B[h][2 * q][0] = v.x;
-                    B[h][2 * q][1] = v.y;
-                    B[h][2 * q + 1][0] = v.z;
-                    B[h][2 * q + 1][1] = v.w;
+            for (int gi = 0; gi < GPA; ++gi) {
+                const int i = i0 + gi;
+                if (GPA > 1 && i >= nw) break;  // warp-uniform: the last block may be short
+                LAQ_TRACE_LOOP(0, i);
+                if (streaming) {
+                    issue(i + S - 1);
+                    cp_async_wait(S - 1);
                 }
-            }
-            LAQ_TRACE_LOOP(2, i);
+                LAQ_TRACE_LOOP(1, i);
 
-            {
-                const uint8_t* slot = ring_w + (size_t)rslot * F::kBytes;
-                uint32_t wd[WPL];
-                const uint4 c0 = *reinterpret_cast<const uint4*>(slot + lane * 16);
-                wd[0] = c0.x; wd[1] = c0.y; wd[2] = c0.z; wd[3] = c0.w;
-                if constexpr (BITS == 4) {
-                    const uint4 c1 = *reinterpret_cast<const uint4*>(slot + 512 + lane * 16);
-                    wd[4] = c1.x; wd[5] = c1.y; wd[6] = c1.z; wd[7] = c1.w;
-                } else {
-                    const uint2 c1 = *reinterpret_cast<const uint2*>(slot + 512 + lane * 8);
-                    wd[4] = c1.x; wd[5] = c1.y;
-                }
-                uint32_t a[8][4];
-                extract<BITS>(wd, p.exps, a);
-#pragma unroll
-                for (int j = 0; j < 8; ++j)
-#pragma unroll
-                    for (int h = 0; h < NH; ++h)
-                        mma16816(D[j & 1][h], a[j][0], a[j][1], a[j][2], a[j][3], B[h][j][0],
-                                 B[h][j][1]);
-            }
-            rslot = rslot + 1 == S ? 0 : rslot + 1;
-            LAQ_TRACE_LOOP(3, i);
-
-            if (gi == GPA - 1 || i == nw - 1) {
-                // Group epilogue (Eq. (1)): y += s * (D - P - z S) per (group, column, row).
-                const int ib = i - gi;
+                // B fragments: x[32c .. 32c+31] of this record's group for lanes whose column
+                // belongs to it, zeros for the others.
+                uint32_t B[NH][8][2];
 #pragma unroll
                 for (int h = 0; h < NH; ++h) {
+                    const bool act = gil == gi && bl + 8 * h < M;
+                    const uint4* src = act ? xs + xo0[h] + i * xstep : zblk;
 #pragma unroll
-                    for (int v = 0; v < 4; ++v) {
-                        const int col = 2 * c + (v & 1);
-                        const int b = MP <= 8 ? col / GPA : 8 * h + col;
-                        const int giv = MP <= 8 ? col % GPA : 0;
-                        if (b < M && ib + giv < nw) {
-                            const int lg = team + (ib + giv) * WT;        // in the phase
-                            const int e = ((pa - g0 + lg) * NT + tile) * 16 + R + 8 * (v >> 1);
-                            const float sv = __half2float(__ushort_as_half(s_sm[e]));
-                            const float zv = (float)z_sm[e];
-                            const float2 sp = ps[b * GP + lg];  // (S, P) of the group
-                            const float d = D[0][h][v] + D[1][h][v] - sp.y;
-                            yacc[h][v] = fmaf(sv, fmaf(-zv, sp.x, d), yacc[h][v]);
-                        }
+                    for (int q = 0; q < 4; ++q) {
+                        const uint4 v = src[q];
+                        B[h][2 * q][0] = v.x;
+                        B[h][2 * q][1] = v.y;
+                        B[h][2 * q + 1][0] = v.z;
+                        B[h][2 * q + 1][1] = v.w;
+                    }
+                }
+                LAQ_TRACE_LOOP(2, i);
+
+                {
+                    const uint8_t* slot = ring_w + (size_t)(streaming ? rslot : i) * F::kBytes;
+                    uint32_t wd[WPL];
+                    const uint4 c0 = *reinterpret_cast<const uint4*>(slot + lane * 16);
+                    wd[0] = c0.x; wd[1] = c0.y; wd[2] = c0.z; wd[3] = c0.w;
+                    if constexpr (BITS == 4) {
+                        const uint4 c1 = *reinterpret_cast<const uint4*>(slot + 512 + lane * 16);
+                        wd[4] = c1.x; wd[5] = c1.y; wd[6] = c1.z; wd[7] = c1.w;
+                    } else {
+                        const uint2 c1 = *reinterpret_cast<const uint2*>(slot + 512 + lane * 8);
+                        wd[4] = c1.x; wd[5] = c1.y;
+                    }
+                    uint32_t a[8][4];
+                    extract<BITS>(wd, p.exps, a);
+#pragma unroll
+                    for (int j = 0; j < 8; ++j)
+#pragma unroll
+                        for (int h = 0; h < NH; ++h)
+                            mma16816(D[j & 1][h], a[j][0], a[j][1], a[j][2], a[j][3], B[h][j][0],
+                                     B[h][j][1]);
+                }
+                if (streaming) rslot = rslot + 1 == S ? 0 : rslot + 1;
+                LAQ_TRACE_LOOP(3, i);
+            }
+
+            // Block epilogue (Eq. (1)): y += s * (D - P - z S) per (group, column, row).  Value
+            // v of the lane is MMA column 2c + (v & 1): batch row col / GPA and the block's
+            // record col % GPA (MP <= 8), or batch row 8h + col (MP = 16).
+#pragma unroll
+            for (int h = 0; h < NH; ++h) {
+#pragma unroll
+                for (int v = 0; v < 4; ++v) {
+                    const int col = 2 * c + (v & 1);
+                    const int b = MP <= 8 ? col / GPA : 8 * h + col;
+                    const int giv = MP <= 8 ? col % GPA : 0;
+                    if (b < M && i0 + giv < nw) {
+                        const int lg = team + (i0 + giv) * WT;        // in the phase
+                        const int e = ((pa - g0 + lg) * NT + tile) * 16 + R + 8 * (v >> 1);
+                        const float sv = __half2float(__ushort_as_half(s_sm[e]));
+                        const float zv = (float)z_sm[e];
+                        const float2 sp = ps[b * GP + lg];  // (S, P) of the group
+                        const float d = D[0][h][v] + D[1][h][v] - sp.y;
+                        yacc[h][v] = fmaf(sv, fmaf(-zv, sp.x, d), yacc[h][v]);
                     }
                 }
             }
-            LAQ_TRACE_LOOP(4, i);
+            LAQ_TRACE_LOOP(4, i0);
         }
         asm volatile("cp.async.wait_all;\n" ::: "memory");
     }
