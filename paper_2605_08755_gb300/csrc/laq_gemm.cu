@@ -241,76 +241,87 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 2) gemm_kernel(const Params p)
         for (int h = 0; h < NH; ++h) xo0[h] = ((bl + 8 * h) * GP + team) * 16 + c * 4;
 
         int rslot = 0;
-        // With S - 1 >= nw every record of the warp was copied in the prologue and has landed;
-        // record i then sits in slot i.
-        const bool streaming = S - 1 < nw;
-        // Records in blocks of GPA (the groups sharing one accumulator); the position in the
-        // block is a compile-time constant, so slot, X and scale offsets fold into immediates.
-        for (int i0 = 0; i0 < nw; i0 += GPA) {
-            float D[2][NH][4];  // two independent accumulator chains (even / odd k16 steps)
+        float D[2][NH][4];  // two independent accumulator chains (even / odd k16 steps)
+
+        // One record: B fragments, the packed words, extraction and the 8 k16-step MMAs.  A
+        // lane's B column belongs to the block's record gil, so only that record reads X (from
+        // xm); the others take zeros.
+        auto record = [&](const int i, const int gi, const uint4* const* xm, const bool kStream) {
+            LAQ_TRACE_LOOP(0, i);
+            if (kStream) {
+                issue(i + S - 1);
+                cp_async_wait(S - 1);
+            }
+            LAQ_TRACE_LOOP(1, i);
+            uint32_t B[NH][8][2];
+#pragma unroll
+            for (int h = 0; h < NH; ++h) {
+                const uint4* src = gil == gi && bl + 8 * h < M ? xm[h] : zblk;
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    const uint4 v = src[q];
+                    B[h][2 * q][0] = v.x;
+                    B[h][2 * q][1] = v.y;
+                    B[h][2 * q + 1][0] = v.z;
+                    B[h][2 * q + 1][1] = v.w;
+                }
+            }
+            LAQ_TRACE_LOOP(2, i);
+            const uint8_t* slot = ring_w + (size_t)(kStream ? rslot : i) * F::kBytes;
+            uint32_t wd[WPL];
+            const uint4 c0 = *reinterpret_cast<const uint4*>(slot + lane * 16);
+            wd[0] = c0.x; wd[1] = c0.y; wd[2] = c0.z; wd[3] = c0.w;
+            if constexpr (BITS == 4) {
+                const uint4 c1 = *reinterpret_cast<const uint4*>(slot + 512 + lane * 16);
+                wd[4] = c1.x; wd[5] = c1.y; wd[6] = c1.z; wd[7] = c1.w;
+            } else {
+                const uint2 c1 = *reinterpret_cast<const uint2*>(slot + 512 + lane * 8);
+                wd[4] = c1.x; wd[5] = c1.y;
+            }
+            uint32_t a[8][4];
+            extract<BITS>(wd, p.exps, a);
+#pragma unroll
+            for (int j = 0; j < 8; ++j)
+#pragma unroll
+                for (int h = 0; h < NH; ++h)
+                    mma16816(D[j & 1][h], a[j][0], a[j][1], a[j][2], a[j][3], B[h][j][0],
+                             B[h][j][1]);
+            if (kStream) rslot = rslot + 1 == S ? 0 : rslot + 1;
+            LAQ_TRACE_LOOP(3, i);
+        };
+
+        // A block of GPA records (the groups sharing one accumulator) from record i0, then its
+        // epilogue.  Without streaming (the usual case) the position in the block is a
+        // compile-time constant, so slot and X offsets fold into immediates; the streaming
+        // form keeps the loop rolled (one copy of the record code, less instruction cache).
+        // (Called with a constant flag, folded once the lambda is inlined.)
+        auto block = [&](const int i0, const bool stream) {
 #pragma unroll
             for (int a = 0; a < 2; ++a)
 #pragma unroll
                 for (int h = 0; h < NH; ++h)
 #pragma unroll
                     for (int v = 0; v < 4; ++v) D[a][h][v] = 0.f;
+            const uint4* xm[NH];
 #pragma unroll
-            for (int gi = 0; gi < GPA; ++gi) {
-                const int i = i0 + gi;
-                if (GPA > 1 && i >= nw) break;  // warp-uniform: the last block may be short
-                LAQ_TRACE_LOOP(0, i);
-                if (streaming) {
-                    issue(i + S - 1);
-                    cp_async_wait(S - 1);
+            for (int h = 0; h < NH; ++h) xm[h] = xs + xo0[h] + (i0 + gil) * xstep;
+            if (stream) {
+#pragma unroll 1
+                for (int gi = 0; gi < GPA; ++gi) {
+                    if (i0 + gi >= nw) break;  // warp-uniform
+                    record(i0 + gi, gi, xm, true);
                 }
-                LAQ_TRACE_LOOP(1, i);
-
-                // B fragments: x[32c .. 32c+31] of this record's group for lanes whose column
-                // belongs to it, zeros for the others.
-                uint32_t B[NH][8][2];
+            } else {
 #pragma unroll
-                for (int h = 0; h < NH; ++h) {
-                    const bool act = gil == gi && bl + 8 * h < M;
-                    const uint4* src = act ? xs + xo0[h] + i * xstep : zblk;
-#pragma unroll
-                    for (int q = 0; q < 4; ++q) {
-                        const uint4 v = src[q];
-                        B[h][2 * q][0] = v.x;
-                        B[h][2 * q][1] = v.y;
-                        B[h][2 * q + 1][0] = v.z;
-                        B[h][2 * q + 1][1] = v.w;
-                    }
+                for (int gi = 0; gi < GPA; ++gi) {
+                    if (i0 + gi >= nw) break;  // warp-uniform
+                    record(i0 + gi, gi, xm, false);
                 }
-                LAQ_TRACE_LOOP(2, i);
-
-                {
-                    const uint8_t* slot = ring_w + (size_t)(streaming ? rslot : i) * F::kBytes;
-                    uint32_t wd[WPL];
-                    const uint4 c0 = *reinterpret_cast<const uint4*>(slot + lane * 16);
-                    wd[0] = c0.x; wd[1] = c0.y; wd[2] = c0.z; wd[3] = c0.w;
-                    if constexpr (BITS == 4) {
-                        const uint4 c1 = *reinterpret_cast<const uint4*>(slot + 512 + lane * 16);
-                        wd[4] = c1.x; wd[5] = c1.y; wd[6] = c1.z; wd[7] = c1.w;
-                    } else {
-                        const uint2 c1 = *reinterpret_cast<const uint2*>(slot + 512 + lane * 8);
-                        wd[4] = c1.x; wd[5] = c1.y;
-                    }
-                    uint32_t a[8][4];
-                    extract<BITS>(wd, p.exps, a);
-#pragma unroll
-                    for (int j = 0; j < 8; ++j)
-#pragma unroll
-                        for (int h = 0; h < NH; ++h)
-                            mma16816(D[j & 1][h], a[j][0], a[j][1], a[j][2], a[j][3], B[h][j][0],
-                                     B[h][j][1]);
-                }
-                if (streaming) rslot = rslot + 1 == S ? 0 : rslot + 1;
-                LAQ_TRACE_LOOP(3, i);
             }
 
-            // Block epilogue (Eq. (1)): y += s * (D - P - z S) per (group, column, row).  Value
-            // v of the lane is MMA column 2c + (v & 1): batch row col / GPA and the block's
-            // record col % GPA (MP <= 8), or batch row 8h + col (MP = 16).
+            // Block epilogue (Eq. (1)): y += s * (D - P - z S) per (group, column, row).
+            // Value v of the lane is MMA column 2c + (v & 1): batch row col / GPA and the
+            // block's record col % GPA (MP <= 8), or batch row 8h + col (MP = 16).
 #pragma unroll
             for (int h = 0; h < NH; ++h) {
 #pragma unroll
@@ -330,6 +341,14 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 2) gemm_kernel(const Params p)
                 }
             }
             LAQ_TRACE_LOOP(4, i0);
+        };
+
+        // With S - 1 >= nw every record of the warp was copied in the prologue and has landed;
+        // record i then sits in slot i.
+        if (S - 1 < nw) {
+            for (int i0 = 0; i0 < nw; i0 += GPA) block(i0, true);
+        } else {
+            for (int i0 = 0; i0 < nw; i0 += GPA) block(i0, false);
         }
         asm volatile("cp.async.wait_all;\n" ::: "memory");
     }
