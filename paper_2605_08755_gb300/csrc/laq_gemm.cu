@@ -86,6 +86,9 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 2) gemm_kernel(const Params p)
     // Let the next kernel on the stream start launching now: it only prefetches constant
     // weights before its own griddepcontrol.wait, which returns once this grid has finished.
     pdl_launch_dependents();
+    // Cluster K split: arrive once now; the matching wait before the partial sums are pushed
+    // into peers' shared memory guarantees that every CTA of the cluster has started.
+    if (gridDim.y > 1) asm volatile("barrier.cluster.arrive.relaxed.aligned;\n" ::: "memory");
     LAQ_TRACE(0);
 
     extern __shared__ __align__(128) uint8_t smem[];
@@ -387,13 +390,13 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 2) gemm_kernel(const Params p)
     }
     __syncthreads();
     constexpr int E = NT * MP * 16;
-    for (int e = threadIdx.x; e < E; e += blockDim.x) {
+    // this CTA's sum of element e over its warps of the tile
+    auto local = [&](int e) {
         const int t = e / (MP * 16), r = e % (MP * 16);
         float acc = 0.f;
         for (int u = 0; u < WT; ++u) acc += red[(size_t)(u * NT + t) * MP * 16 + r];
-        part[e] = acc;
-    }
-    LAQ_TRACE(4);
+        return acc;
+    };
 
     auto store = [&](int e, float acc) {
         const int t = e / (MP * 16), b = (e / 16) % MP, row = e % 16;
@@ -403,18 +406,26 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 2) gemm_kernel(const Params p)
         }
     };
     if (C == 1) {
-        __syncthreads();
-        for (int e = threadIdx.x; e < E; e += blockDim.x) store(e, part[e]);
+        for (int e = threadIdx.x; e < E; e += blockDim.x) store(e, local(e));
+        LAQ_TRACE(4);
         LAQ_TRACE(5);
     } else {
+        // Element e belongs to CTA e % C of the cluster: each CTA pushes its partial into the
+        // owner's part[rank][e / C] (distributed shared memory), one cluster barrier, then the
+        // owner sums the C partials in rank order.  Nothing reads another CTA's shared memory
+        // after the barrier, so each CTA may finish at once.
         cg::cluster_group cluster = cg::this_cluster();
-        cluster.sync();  // every CTA's partial sums are complete
-        for (int e = rank + threadIdx.x * C; e < E; e += blockDim.x * C) {
+        const int EL = E / C;  // E is a multiple of 16, C divides 16
+        asm volatile("barrier.cluster.wait.aligned;\n" ::: "memory");
+        for (int e = threadIdx.x; e < E; e += blockDim.x)
+            cluster.map_shared_rank(part, e % C)[rank * EL + e / C] = local(e);
+        LAQ_TRACE(4);
+        cluster.sync();  // every partial has arrived at its owner
+        for (int el = threadIdx.x; el < EL; el += blockDim.x) {
             float acc = 0.f;
-            for (int q = 0; q < C; ++q) acc += cluster.map_shared_rank(part, q)[e];
-            store(e, acc);
+            for (int q = 0; q < C; ++q) acc += part[q * EL + el];
+            store(el * C + rank, acc);
         }
-        cluster.sync();  // peers have finished reading this CTA's shared memory
         LAQ_TRACE(5);
     }
 }
