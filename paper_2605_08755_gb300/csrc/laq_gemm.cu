@@ -181,48 +181,61 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 2) gemm_kernel(const Params p)
         }
 
         // Raw X of the phase (row b's groups pa..pb-1 are 256 * ng contiguous bytes), through
-        // L2 into registers, then shared memory.  16-byte chunk u = (b, q) holds x[8q .. 8q+7]
-        // of group q / 16 of the phase, i.e. pairs 4 (q % 4) + w of that group for its four
-        // 32-bit words w; the 16 chunks of a group sit in 16 aligned lanes, which sum
-        // S_g = sum_k x_k and P_g = sum_k c_k x_k by shuffles.
+        // L2 into registers, then shared memory.  16-byte chunk q of a group holds x[8q .. 8q+7],
+        // i.e. pairs 4 (q % 4) + w for its four 32-bit words w.  Unit u = (b, group, h), h < 8,
+        // loads chunks h and h + 8 of the group, whose pairs have the same offsets c_k; the 8
+        // aligned lanes of a group sum S_g = sum_k x_k and P_g = sum_k c_k x_k by shuffles.
         {
-            const int per_row = ng * 16;
-            const int nch = M * per_row;  // a multiple of 16
-            for (int u0 = 0; u0 < nch; u0 += 4 * (int)blockDim.x) {
-                uint4 v[4];
+            const int per_row = ng * 8;     // units per batch row (a multiple of 8)
+            const int nu = M * per_row;     // < 2^16
+            // u / per_row = umulhi(u, inv) exactly for u, per_row < 2^16
+            const uint32_t inv = 0xffffffffu / (uint32_t)per_row + 1u;
+            for (int u0 = 0; u0 < nu; u0 += 2 * (int)blockDim.x) {
+                uint4 v[2][2];
+                int xo[2];  // offset of the unit's first chunk in xs (uint4), -1 past the end
+                int po[2];  // its group's (S, P) slot [b][group]
 #pragma unroll
-                for (int r = 0; r < 4; ++r) {
+                for (int r = 0; r < 2; ++r) {
                     const int u = u0 + r * (int)blockDim.x + (int)threadIdx.x;
-                    if (u < nch) {
-                        const int b = u / per_row, q = u - b * per_row;
-                        v[r] = ld_cg16(p.X + (size_t)b * p.K + (size_t)pa * 128 + q * 8);
+                    if (u < nu) {
+                        const int b = (int)__umulhi((uint32_t)u, inv);
+                        const int uu = u - b * per_row;
+                        const int q = (uu >> 3) * 16 + (uu & 7);  // chunk in the row
+                        const uint16_t* src = p.X + (size_t)b * p.K + (size_t)pa * 128 + q * 8;
+                        v[r][0] = ld_cg16(src);
+                        v[r][1] = ld_cg16(src + 64);
+                        xo[r] = b * GP * 16 + q;
+                        po[r] = b * GP + (uu >> 3);
                     } else {
-                        v[r] = make_uint4(0u, 0u, 0u, 0u);
+                        v[r][0] = v[r][1] = make_uint4(0u, 0u, 0u, 0u);
+                        xo[r] = -1;
+                        po[r] = 0;
                     }
                 }
 #pragma unroll
-                for (int r = 0; r < 4; ++r) {
+                for (int r = 0; r < 2; ++r) {
                     // (warp-uniform) nothing of this batch for this warp
-                    if (u0 + r * (int)blockDim.x + warp * 32 >= nch) break;
-                    const int u = u0 + r * (int)blockDim.x + (int)threadIdx.x;
-                    const uint32_t w4[4] = {v[r].x, v[r].y, v[r].z, v[r].w};
+                    if (u0 + r * (int)blockDim.x + warp * 32 >= nu) break;
+                    const uint32_t w0[4] = {v[r][0].x, v[r][0].y, v[r][0].z, v[r][0].w};
+                    const uint32_t w1[4] = {v[r][1].x, v[r][1].y, v[r][1].z, v[r][1].w};
                     float sx = 0.f, px = 0.f;
 #pragma unroll
                     for (int w = 0; w < 4; ++w) {
-                        const float2 f = __half22float2(*reinterpret_cast<const __half2*>(&w4[w]));
-                        const float pair = f.x + f.y;
+                        const float2 f0 = __half22float2(*reinterpret_cast<const __half2*>(&w0[w]));
+                        const float2 f1 = __half22float2(*reinterpret_cast<const __half2*>(&w1[w]));
+                        const float pair = (f0.x + f0.y) + (f1.x + f1.y);
                         sx += pair;
-                        px = fmaf(row_offset<BITS>((u & 3) * 4 + w), pair, px);
+                        px = fmaf(row_offset<BITS>((lane & 3) * 4 + w), pair, px);
                     }
 #pragma unroll
-                    for (int o = 1; o < 16; o <<= 1) {
+                    for (int o = 1; o < 8; o <<= 1) {
                         sx += __shfl_xor_sync(0xffffffffu, sx, o);
                         px += __shfl_xor_sync(0xffffffffu, px, o);
                     }
-                    if (u < nch) {
-                        const int b = u / per_row, q = u - b * per_row;
-                        xs[(size_t)b * GP * 16 + q] = v[r];
-                        if ((q & 15) == 0) ps[b * GP + (q >> 4)] = make_float2(sx, px);
+                    if (xo[r] >= 0) {
+                        xs[xo[r]] = v[r][0];
+                        xs[xo[r] + 8] = v[r][1];
+                        if ((lane & 7) == 0) ps[po[r]] = make_float2(sx, px);  // unit h = 0
                     }
                 }
             }
