@@ -124,7 +124,7 @@ def test_gemm_parity_shapes(bits, M, K, N):
 
 
 CONFIGS = [laq.GemmConfig.make(nt, w, cl, st, pdl)
-           for nt, w, cl, st, pdl in itertools.product((1, 2, 4, 8), (1, 2, 3, 4, 8), (1, 2, 8), (2, 3, 16),
+           for nt, w, cl, st, pdl in itertools.product((1, 2, 4, 8), (1, 2, 3, 4, 8), (1, 2, 4, 8), (2, 3, 16),
                                                        (0, 1))]
 
 
