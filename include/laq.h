@@ -243,6 +243,76 @@ laq_status laq_gemm_chain(const laq_gemv *gemvs, int32_t count, void *workspace,
  */
 laq_status laq_gemm_chain_static(const laq_gemv *gemvs, int32_t count, void *stream);
 
+/* ======================================================================================
+ * Decoder operations around the projections: the rest of one decode step of a Qwen3-style
+ * model (the models whose decoding speed Sec. 5.2 reports).  The paper defines none of them;
+ * each follows the standard decoder definition stated below, computes in fp32 and rounds each
+ * stored tensor to fp16 once.  All tensors are caller-owned device memory, row-major, fp16
+ * unless stated; sizes are validated on the host (LAQ_ERR_SHAPE / LAQ_ERR_ALIGN /
+ * LAQ_ERR_NULL, nothing launched); values read from device memory (positions, lengths,
+ * tokens) are clamped in the kernels as stated and never index outside the given buffers.
+ * Each kernel may start while its predecessor on the stream finishes (programmatic dependent
+ * launch) and waits for it before touching memory.
+ * ====================================================================================== */
+
+/*
+ * RMSNorm with the residual add, one row per m < M (1 <= M <= 65535, H % 8 == 0, 8 <= H <=
+ * 8192; X, R, R_out, w, Y 16-byte aligned):
+ *   h = fp16(X + R)            (h = X when R is NULL)
+ *   R_out = h                  (skipped when R_out is NULL; R_out may equal R)
+ *   Y = fp16(h / sqrt(mean_k h_k^2 + eps) * w)     w: [H] weights.
+ */
+laq_status laq_rmsnorm(const void *X, const void *R, void *R_out, const void *w, int64_t M,
+                       int64_t H, float eps, void *Y, void *stream);
+
+/*
+ * Per-head RMSNorm of q and k, rotary position embedding, and the KV-cache append, for the
+ * fused q|k|v projection output qkv [M][(Hq + 2 Hkv) * D] (q heads, then k heads, then v heads).
+ * D must be 128; Hq % Hkv == 0 and Hq / Hkv <= 8.  For row m at position p = pos[m] (device):
+ *   q_h = rope(rmsnorm(q_h) * q_norm_w)  -> q_out [M][Hq][D]
+ *   k_g = rope(rmsnorm(k_g) * k_norm_w)  -> k_cache [M][Hkv][L_max][D] at [m][g][p]
+ *   v_g                                  -> v_cache (same layout) at [m][g][p]
+ * rmsnorm(x) = x / sqrt(mean(x^2) + eps); rope rotates pairs (i, i + D/2) by the angle
+ * p * theta^(-2i/D):  (x_i, x_{i+D/2}) -> (x_i cos - x_{i+D/2} sin, x_{i+D/2} cos + x_i sin).
+ * A position outside [0, L_max) still produces q but stores nothing in the caches.  qkv, q_out
+ * and the caches must be 8-byte aligned.
+ */
+laq_status laq_qk_norm_rope(const void *qkv, const void *q_norm_w, const void *k_norm_w,
+                            const int32_t *pos, int64_t M, int32_t Hq, int32_t Hkv, int32_t D,
+                            float theta, float eps, void *q_out, void *k_cache, void *v_cache,
+                            int64_t L_max, void *stream);
+
+/* Bytes of workspace laq_attention_decode needs (fp32 partials of 64-token chunks); 0 for
+ * invalid sizes. */
+size_t laq_attention_workspace_bytes(int64_t M, int32_t Hq, int64_t L_max);
+
+/*
+ * Grouped-query attention of each row's new token over its cache (decode):
+ *   out[m][h] = sum_{t < n} softmax_t(scale * q[m][h] . K[m][g][t]) V[m][g][t],  g = h / (Hq/Hkv),
+ * n = len[m] (device) clamped to [0, L_max]; a row with n = 0 gets zeros.  q, out [M][Hq][D],
+ * caches [M][Hkv][L_max][D], D = 128, Hq / Hkv <= 8.  Two launches: 64-token chunk partials
+ * (max, sum of exponentials, weighted V sum) into `workspace`, then their combination in chunk
+ * order (deterministic).  workspace_bytes >= laq_attention_workspace_bytes(M, Hq, L_max)
+ * (LAQ_ERR_WORKSPACE otherwise; 4-byte aligned).  k_cache 16-byte aligned.
+ */
+laq_status laq_attention_decode(const void *q, const void *k_cache, const void *v_cache,
+                                const int32_t *len, int64_t M, int32_t Hq, int32_t Hkv,
+                                int32_t D, int64_t L_max, float scale, void *out,
+                                void *workspace, size_t workspace_bytes, void *stream);
+
+/* h[m][i] = fp16(silu(g) * u), g = gate_up[m][i], u = gate_up[m][I + i], silu(x) = x / (1 +
+ * e^-x): the fused gate|up projection output [M][2I] -> [M][I].  I % 8 == 0, 16-byte aligned. */
+laq_status laq_silu_mul(const void *gate_up, int64_t M, int64_t I, void *h, void *stream);
+
+/* X[m] = E[tokens[m]] for the embedding table E [V][H]; a token outside [0, V) gives a zero
+ * row.  H % 8 == 0, E and X 16-byte aligned. */
+laq_status laq_embed(const void *E, const int32_t *tokens, int64_t M, int64_t V, int64_t H,
+                     void *X, void *stream);
+
+/* out[m] = argmax_v logits[m][v] over fp16 logits [M][V] (ties: the smallest index; NaN never
+ * wins; a row of NaN or -inf gives 0). */
+laq_status laq_argmax(const void *logits, int64_t M, int64_t V, int32_t *out, void *stream);
+
 #ifdef __cplusplus
 }
 #endif

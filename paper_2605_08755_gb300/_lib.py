@@ -19,7 +19,9 @@ STATUS = {0: "LAQ_OK", 1: "LAQ_ERR_NULL", 2: "LAQ_ERR_BITS", 3: "LAQ_ERR_GROUP",
 # Symbols include/laq.h declares.
 EXPORTS = ("laq_status_str", "laq_version", "laq_packed_bytes", "laq_quantize_rtn", "laq_pack",
            "laq_unpack", "laq_gemm_wxg128", "laq_gemm_plan", "laq_gemm_wxg128_config",
-           "laq_chain_workspace_bytes", "laq_gemm_chain", "laq_gemm_chain_static")
+           "laq_chain_workspace_bytes", "laq_gemm_chain", "laq_gemm_chain_static",
+           "laq_rmsnorm", "laq_qk_norm_rope", "laq_attention_workspace_bytes",
+           "laq_attention_decode", "laq_silu_mul", "laq_embed", "laq_argmax")
 CHAIN_MAX = 384  # LAQ_CHAIN_MAX
 
 
@@ -75,9 +77,19 @@ def lib():
     L.laq_chain_workspace_bytes.restype = ctypes.c_size_t
     L.laq_gemm_chain.argtypes = [ctypes.POINTER(Gemv), ctypes.c_int32, P, ctypes.c_size_t, P]
     L.laq_gemm_chain_static.argtypes = [ctypes.POINTER(Gemv), ctypes.c_int32, P]
+    F, I32, SZ = ctypes.c_float, ctypes.c_int32, ctypes.c_size_t
+    L.laq_rmsnorm.argtypes = [P, P, P, P, I64, I64, F, P, P]
+    L.laq_qk_norm_rope.argtypes = [P, P, P, P, I64, I32, I32, I32, F, F, P, P, P, I64, P]
+    L.laq_attention_workspace_bytes.argtypes = [I64, I32, I64]
+    L.laq_attention_workspace_bytes.restype = SZ
+    L.laq_attention_decode.argtypes = [P, P, P, P, I64, I32, I32, I32, I64, F, P, P, SZ, P]
+    L.laq_silu_mul.argtypes = [P, I64, I64, P, P]
+    L.laq_embed.argtypes = [P, P, I64, I64, I64, P, P]
+    L.laq_argmax.argtypes = [P, I64, I64, P, P]
     for name in ("laq_quantize_rtn", "laq_pack", "laq_unpack", "laq_gemm_wxg128",
                  "laq_gemm_plan", "laq_gemm_wxg128_config", "laq_gemm_chain",
-                 "laq_gemm_chain_static"):
+                 "laq_gemm_chain_static", "laq_rmsnorm", "laq_qk_norm_rope",
+                 "laq_attention_decode", "laq_silu_mul", "laq_embed", "laq_argmax"):
         getattr(L, name).restype = I
     return L
 
@@ -204,3 +216,87 @@ def chain_status(workspace):
     import torch
     torch.cuda.synchronize(workspace.device)
     return int(workspace[:4].view(torch.int32)[0].item())
+
+
+# ---- decoder operations around the projections (one decode step) ----
+
+def laq_rmsnorm(X, w, eps, R=None, R_out=None, Y=None, stream=None):
+    """Y = rmsnorm(X + R) * w per row (fp16 [M, H]); with R_out, also R_out = fp16(X + R)."""
+    import torch
+    M, H = X.shape
+    if Y is None:
+        Y = torch.empty_like(X)
+    _check(lib().laq_rmsnorm(_ptr(X), _ptr(R), _ptr(R_out), _ptr(w), M, H, float(eps), _ptr(Y),
+                             _stream(stream)), "laq_rmsnorm")
+    return Y
+
+
+def laq_qk_norm_rope(qkv, q_norm_w, k_norm_w, pos, Hq, Hkv, theta, eps, k_cache, v_cache,
+                     q_out=None, stream=None):
+    """qkv [M, (Hq + 2 Hkv) * 128] -> q_out [M, Hq, 128]; appends k, v at pos[m] to the caches
+    [M, Hkv, L_max, 128]."""
+    import torch
+    M = qkv.shape[0]
+    D = k_cache.shape[-1]
+    L_max = k_cache.shape[-2]
+    if q_out is None:
+        q_out = torch.empty((M, Hq, D), dtype=torch.float16, device=qkv.device)
+    _check(lib().laq_qk_norm_rope(_ptr(qkv), _ptr(q_norm_w), _ptr(k_norm_w), _ptr(pos), M, Hq,
+                                  Hkv, D, float(theta), float(eps), _ptr(q_out), _ptr(k_cache),
+                                  _ptr(v_cache), L_max, _stream(stream)), "laq_qk_norm_rope")
+    return q_out
+
+
+def attention_workspace(M, Hq, L_max, device):
+    import torch
+    n = int(lib().laq_attention_workspace_bytes(M, Hq, L_max))
+    if n == 0:
+        raise ValueError("invalid attention sizes")
+    return torch.empty((n // 4,), dtype=torch.float32, device=device)
+
+
+def laq_attention_decode(q, k_cache, v_cache, lens, scale, workspace, out=None, stream=None):
+    """out [M, Hq, 128] = GQA softmax attention of q [M, Hq, 128] over the first lens[m]
+    tokens of the caches [M, Hkv, L_max, 128]."""
+    import torch
+    M, Hq, D = q.shape
+    Hkv, L_max = k_cache.shape[1], k_cache.shape[2]
+    if out is None:
+        out = torch.empty_like(q)
+    _check(lib().laq_attention_decode(_ptr(q), _ptr(k_cache), _ptr(v_cache), _ptr(lens), M, Hq,
+                                      Hkv, D, L_max, float(scale), _ptr(out), _ptr(workspace),
+                                      workspace.numel() * workspace.element_size(),
+                                      _stream(stream)), "laq_attention_decode")
+    return out
+
+
+def laq_silu_mul(gate_up, h=None, stream=None):
+    """h [M, I] = silu(gate_up[:, :I]) * gate_up[:, I:]."""
+    import torch
+    M, I2 = gate_up.shape
+    if h is None:
+        h = torch.empty((M, I2 // 2), dtype=torch.float16, device=gate_up.device)
+    _check(lib().laq_silu_mul(_ptr(gate_up), M, I2 // 2, _ptr(h), _stream(stream)),
+           "laq_silu_mul")
+    return h
+
+
+def laq_embed(E, tokens, X=None, stream=None):
+    """X [M, H] = E[tokens] (zero rows for tokens outside the table)."""
+    import torch
+    V, H = E.shape
+    M = tokens.shape[0]
+    if X is None:
+        X = torch.empty((M, H), dtype=torch.float16, device=E.device)
+    _check(lib().laq_embed(_ptr(E), _ptr(tokens), M, V, H, _ptr(X), _stream(stream)), "laq_embed")
+    return X
+
+
+def laq_argmax(logits, out=None, stream=None):
+    """out [M] int32 = argmax over each row of fp16 logits [M, V] (ties: smallest index)."""
+    import torch
+    M, V = logits.shape
+    if out is None:
+        out = torch.empty((M,), dtype=torch.int32, device=logits.device)
+    _check(lib().laq_argmax(_ptr(logits), M, V, _ptr(out), _stream(stream)), "laq_argmax")
+    return out

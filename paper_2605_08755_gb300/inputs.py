@@ -60,3 +60,57 @@ def activations_torch(M, K, seed, device):
     g = torch.Generator(device=device)
     g.manual_seed(seed + 7_777_777)
     return torch.randn((M, K), generator=g, device=device, dtype=torch.float32).to(torch.float16)
+
+
+# ---- the rest of a decode step (synthetic stand-ins; no checkpoint is used) ----
+
+# Decoder dimensions of the two Qwen3 models (their public configurations): hidden size H,
+# q heads, kv heads, head size D, MLP width I, vocabulary V, rotary base, RMSNorm epsilon.
+DECODER = {
+    "qwen3-4b": dict(H=2560, Hq=32, Hkv=8, D=128, I=9728, V=151936, theta=1e6, eps=1e-6),
+    "qwen3-8b": dict(H=4096, Hq=32, Hkv=8, D=128, I=12288, V=151936, theta=1e6, eps=1e-6),
+}
+NORM_STD = 0.1      # norm weights ~ 1 + N(0, 0.1^2)
+EMBED_STD = 0.05    # embedding rows ~ N(0, 0.05^2)
+
+
+def norm_weight(n, seed):
+    rng = np.random.default_rng(seed + 5_555_555)
+    return (1.0 + NORM_STD * rng.standard_normal(n, dtype=np.float32)).astype(np.float16)
+
+
+def embedding(V, H, seed):
+    rng = np.random.default_rng(seed + 3_333_333)
+    return (EMBED_STD * rng.standard_normal((V, H), dtype=np.float32)).astype(np.float16)
+
+
+def kv_cache(M, Hkv, L, D, seed):
+    """Cached keys or values ~ N(0, 1) for the tokens before the new one."""
+    rng = np.random.default_rng(seed + 1_111_111)
+    return rng.standard_normal((M, Hkv, L, D), dtype=np.float32).astype(np.float16)
+
+
+def tokens(M, V, seed):
+    rng = np.random.default_rng(seed + 9_999_999)
+    return rng.integers(0, V, size=M).astype(np.int32)
+
+
+def norm_weight_torch(n, seed, device):
+    import torch
+    g = torch.Generator(device=device)
+    g.manual_seed(seed + 5_555_555)
+    return (1.0 + NORM_STD * torch.randn(n, generator=g, device=device)).to(torch.float16)
+
+
+def embedding_torch(V, H, seed, device):
+    import torch
+    g = torch.Generator(device=device)
+    g.manual_seed(seed + 3_333_333)
+    return (EMBED_STD * torch.randn((V, H), generator=g, device=device)).to(torch.float16)
+
+
+def kv_cache_torch(M, Hkv, L, D, seed, device):
+    import torch
+    g = torch.Generator(device=device)
+    g.manual_seed(seed + 1_111_111)
+    return torch.randn((M, Hkv, L, D), generator=g, device=device).to(torch.float16)
