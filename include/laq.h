@@ -293,12 +293,30 @@ size_t laq_attention_workspace_bytes(int64_t M, int32_t Hq, int64_t L_max);
  * caches [M][Hkv][L_max][D], D = 128, Hq / Hkv <= 8.  Two launches: 64-token chunk partials
  * (max, sum of exponentials, weighted V sum) into `workspace`, then their combination in chunk
  * order (deterministic).  workspace_bytes >= laq_attention_workspace_bytes(M, Hq, L_max)
- * (LAQ_ERR_WORKSPACE otherwise; 4-byte aligned).  k_cache 16-byte aligned.
+ * (LAQ_ERR_WORKSPACE otherwise; 4-byte aligned).  Both caches 16-byte aligned.
  */
 laq_status laq_attention_decode(const void *q, const void *k_cache, const void *v_cache,
                                 const int32_t *len, int64_t M, int32_t Hq, int32_t Hkv,
                                 int32_t D, int64_t L_max, float scale, void *out,
                                 void *workspace, size_t workspace_bytes, void *stream);
+
+/* Bytes of workspace laq_attention_qkv needs (the chunk partials, as for
+ * laq_attention_decode); 0 for invalid sizes. */
+size_t laq_attention_qkv_workspace_bytes(int64_t M, int32_t Hq, int32_t Hkv, int64_t L_max);
+
+/*
+ * laq_qk_norm_rope followed by laq_attention_decode with len[m] = pos[m] + 1, in two launches
+ * instead of three (same inputs, outputs and results): each attention CTA (64-token chunk, kv
+ * head, row) normalises and rotates its q heads itself, and the CTA whose chunk holds pos[m]
+ * computes the new k and v, stores them in the caches and uses them in place of the cached
+ * row; the chunk partials are then combined in chunk order.  Workspace 16-byte aligned and
+ * >= laq_attention_qkv_workspace_bytes (LAQ_ERR_WORKSPACE otherwise).
+ */
+laq_status laq_attention_qkv(const void *qkv, const void *q_norm_w, const void *k_norm_w,
+                             const int32_t *pos, int64_t M, int32_t Hq, int32_t Hkv, int32_t D,
+                             float theta, float eps, void *k_cache, void *v_cache, int64_t L_max,
+                             float scale, void *out, void *workspace, size_t workspace_bytes,
+                             void *stream);
 
 /* h[m][i] = fp16(silu(g) * u), g = gate_up[m][i], u = gate_up[m][I + i], silu(x) = x / (1 +
  * e^-x): the fused gate|up projection output [M][2I] -> [M][I].  I % 8 == 0, 16-byte aligned. */

@@ -21,7 +21,8 @@ EXPORTS = ("laq_status_str", "laq_version", "laq_packed_bytes", "laq_quantize_rt
            "laq_unpack", "laq_gemm_wxg128", "laq_gemm_plan", "laq_gemm_wxg128_config",
            "laq_chain_workspace_bytes", "laq_gemm_chain", "laq_gemm_chain_static",
            "laq_rmsnorm", "laq_qk_norm_rope", "laq_attention_workspace_bytes",
-           "laq_attention_decode", "laq_silu_mul", "laq_embed", "laq_argmax")
+           "laq_attention_decode", "laq_attention_qkv_workspace_bytes", "laq_attention_qkv",
+           "laq_silu_mul", "laq_embed", "laq_argmax")
 CHAIN_MAX = 384  # LAQ_CHAIN_MAX
 
 
@@ -83,13 +84,18 @@ def lib():
     L.laq_attention_workspace_bytes.argtypes = [I64, I32, I64]
     L.laq_attention_workspace_bytes.restype = SZ
     L.laq_attention_decode.argtypes = [P, P, P, P, I64, I32, I32, I32, I64, F, P, P, SZ, P]
+    L.laq_attention_qkv_workspace_bytes.argtypes = [I64, I32, I32, I64]
+    L.laq_attention_qkv_workspace_bytes.restype = SZ
+    L.laq_attention_qkv.argtypes = [P, P, P, P, I64, I32, I32, I32, F, F, P, P, I64, F, P, P, SZ,
+                                    P]
     L.laq_silu_mul.argtypes = [P, I64, I64, P, P]
     L.laq_embed.argtypes = [P, P, I64, I64, I64, P, P]
     L.laq_argmax.argtypes = [P, I64, I64, P, P]
     for name in ("laq_quantize_rtn", "laq_pack", "laq_unpack", "laq_gemm_wxg128",
                  "laq_gemm_plan", "laq_gemm_wxg128_config", "laq_gemm_chain",
                  "laq_gemm_chain_static", "laq_rmsnorm", "laq_qk_norm_rope",
-                 "laq_attention_decode", "laq_silu_mul", "laq_embed", "laq_argmax"):
+                 "laq_attention_decode", "laq_attention_qkv_workspace_bytes", "laq_attention_qkv",
+           "laq_silu_mul", "laq_embed", "laq_argmax"):
         getattr(L, name).restype = I
     return L
 
@@ -267,6 +273,32 @@ def laq_attention_decode(q, k_cache, v_cache, lens, scale, workspace, out=None, 
                                       Hkv, D, L_max, float(scale), _ptr(out), _ptr(workspace),
                                       workspace.numel() * workspace.element_size(),
                                       _stream(stream)), "laq_attention_decode")
+    return out
+
+
+def attention_qkv_workspace(M, Hq, Hkv, L_max, device):
+    """A workspace for laq_attention_qkv."""
+    import torch
+    n = int(lib().laq_attention_qkv_workspace_bytes(M, Hq, Hkv, L_max))
+    if n == 0:
+        raise ValueError("invalid attention sizes")
+    return torch.zeros((n,), dtype=torch.uint8, device=device)
+
+
+def laq_attention_qkv(qkv, q_norm_w, k_norm_w, pos, Hq, Hkv, theta, eps, k_cache, v_cache,
+                      scale, workspace, out=None, stream=None):
+    """laq_qk_norm_rope + laq_attention_decode (len = pos + 1) in two launches: out [M, Hq, 128];
+    appends k, v at pos[m] to the caches [M, Hkv, L_max, 128]."""
+    import torch
+    M = qkv.shape[0]
+    D, L_max = k_cache.shape[-1], k_cache.shape[-2]
+    if out is None:
+        out = torch.empty((M, Hq, D), dtype=torch.float16, device=qkv.device)
+    _check(lib().laq_attention_qkv(_ptr(qkv), _ptr(q_norm_w), _ptr(k_norm_w), _ptr(pos), M, Hq,
+                                   Hkv, D, float(theta), float(eps), _ptr(k_cache),
+                                   _ptr(v_cache), L_max, float(scale), _ptr(out),
+                                   _ptr(workspace), workspace.numel() * workspace.element_size(),
+                                   _stream(stream)), "laq_attention_qkv")
     return out
 
 

@@ -50,6 +50,46 @@ __device__ __forceinline__ uint4 pack8(const float (&f)[8]) {
     return make_uint4(w[0], w[1], w[2], w[3]);
 }
 
+
+// RMSNorm over a head (lane l holds elements 4l .. 4l+3 of the warp's head), times the norm
+// weights, then the rotate-half rotation at position p; every lane of the warp takes part.
+__device__ __forceinline__ void norm_rope4(const float (&x)[4], const __half* __restrict__ wn,
+                                           int lane, int64_t p, float log2_theta, float eps,
+                                           float (&o)[4]) {
+    float ss = 0.f;
+#pragma unroll
+    for (int e = 0; e < 4; ++e) ss = fmaf(x[e], x[e], ss);
+    ss = warp_sum(ss);
+    const float inv = rsqrtf(ss / (float)kHeadDim + eps);
+    float y[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) y[e] = x[e] * inv * __half2float(wn[4 * lane + e]);
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+        const float partner = __shfl_xor_sync(0xffffffffu, y[e], 16);
+        const int i = (4 * lane + e) & (kHeadDim / 2 - 1);  // frequency index
+        const float inv_freq = exp2f(-(2.f * (float)i / (float)kHeadDim) * log2_theta);
+        float sn, cs;
+        sincosf((float)p * inv_freq, &sn, &cs);
+        o[e] = lane < 16 ? y[e] * cs - partner * sn : y[e] * cs + partner * sn;
+    }
+}
+
+__device__ __forceinline__ void load4(const __half* src, float (&x)[4]) {
+    const uint2 raw = *reinterpret_cast<const uint2*>(src);
+    const float2 a = __half22float2(*reinterpret_cast<const __half2*>(&raw.x));
+    const float2 b = __half22float2(*reinterpret_cast<const __half2*>(&raw.y));
+    x[0] = a.x; x[1] = a.y; x[2] = b.x; x[3] = b.y;
+}
+
+__device__ __forceinline__ uint2 round4(const float (&o)[4]) {
+    const __half2 lo = __floats2half2_rn(o[0], o[1]), hi = __floats2half2_rn(o[2], o[3]);
+    uint2 w;
+    w.x = *reinterpret_cast<const uint32_t*>(&lo);
+    w.y = *reinterpret_cast<const uint32_t*>(&hi);
+    return w;
+}
+
 // ---- RMSNorm with the residual add ----
 // Row m: h = X + R (rounded to fp16; h = X without R), R_out = h, Y = h / sqrt(mean(h^2) + eps)
 // * w.  One CTA per row; each thread keeps up to kRmsChunks 8-element chunks in registers.
@@ -169,18 +209,22 @@ __global__ void __launch_bounds__(128) qk_norm_rope_kernel(
 }
 
 // ---- attention: per-chunk partials ----
-// CTA (chunk c, kv head g, row m) over tokens [64c, 64c + 64) of the row's len[m] cached tokens,
-// for the G = Hq / Hkv q heads of g at once (their K and V rows are read once): scores
-// s = scale * q . k, chunk max, p = exp(s - max), sum p and acc = sum p v, written as partial
-// [m][h][c] = (acc[D], max, sum).  Chunks at or past len[m] write nothing.
+// CTA (chunk c, kv head g, row m) over tokens [64c, 64c + 64) of the row's cached tokens, for
+// the G = Hq / Hkv q heads of g at once (their K and V rows are read once): the chunk's K and V
+// rows (2 x 16 KB) are copied to shared memory with every copy in flight at once, then scores
+// s = scale * q . k, the chunk max, p = exp(s - max), sum p and acc = sum p v, written as
+// partial [m][h][c] = (acc[D], max, sum).  Chunks at or past the row's length write nothing.
 __global__ void __launch_bounds__(128) attn_partial_kernel(
     const __half* __restrict__ q, const __half* __restrict__ k_cache,
     const __half* __restrict__ v_cache, const int32_t* __restrict__ len, int Hq, int Hkv,
     int64_t L_max, float scale, float* part, int nchunk) {
     pdl_launch_dependents();
     pdl_wait();
+    __shared__ __align__(16) __half ks[kChunk][kHeadDim];
+    __shared__ __align__(16) __half vs[kChunk][kHeadDim];
     __shared__ float qs[kMaxGroup][kHeadDim];
     __shared__ float sc[kMaxGroup][kChunk];
+    __shared__ float mx[kMaxGroup], sm[kMaxGroup];
     const int c = blockIdx.x, g = blockIdx.y, m = blockIdx.z;
     const int G = Hq / Hkv;
     const int L = (int)min((int64_t)max(len[m], 0), L_max);  // cached tokens of row m
@@ -188,19 +232,29 @@ __global__ void __launch_bounds__(128) attn_partial_kernel(
     if (t0 >= L) return;
     const int nt = min(kChunk, L - t0);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const size_t kv0 = ((size_t)m * Hkv + g) * L_max + t0;  // row of token t0
+    {
+        const uint32_t kss = (uint32_t)__cvta_generic_to_shared(&ks[0][0]);
+        const uint32_t vss = (uint32_t)__cvta_generic_to_shared(&vs[0][0]);
+        for (int u = threadIdx.x; u < nt * (kHeadDim / 8); u += blockDim.x) {  // 16-byte pieces
+            cp_async16(kss + 16 * u, k_cache + kv0 * kHeadDim + 8 * u);
+            cp_async16(vss + 16 * u, v_cache + kv0 * kHeadDim + 8 * u);
+        }
+        cp_async_commit();
+    }
     for (int i = threadIdx.x; i < G * kHeadDim; i += blockDim.x) {
         const int j = i / kHeadDim, d = i % kHeadDim;
         qs[j][d] = scale * __half2float(q[((size_t)m * Hq + g * G + j) * kHeadDim + d]);
     }
+    asm volatile("cp.async.wait_all;\n" ::: "memory");
     __syncthreads();
-    const size_t kv0 = ((size_t)m * Hkv + g) * L_max + t0;  // row of token t0
     // Scores: a half-warp per token, lane l & 15 holding elements 8 (l & 15) .. +7.
     const int hl = lane & 15;
     for (int base = 0; base < nt; base += 8) {
         const int tt = base + 2 * warp + (lane >> 4);
         float kv[8];
         if (tt < nt) {
-            unpack8(*reinterpret_cast<const uint4*>(k_cache + (kv0 + tt) * kHeadDim + 8 * hl), kv);
+            unpack8(*reinterpret_cast<const uint4*>(&ks[tt][8 * hl]), kv);
         } else {
 #pragma unroll
             for (int e = 0; e < 8; ++e) kv[e] = 0.f;
@@ -217,7 +271,6 @@ __global__ void __launch_bounds__(128) attn_partial_kernel(
         }
     }
     __syncthreads();
-    __shared__ float mx[kMaxGroup], sm[kMaxGroup];
     for (int j = warp; j < G; j += 4) {
         const float a = lane < nt ? sc[j][lane] : -INFINITY;
         const float b = lane + 32 < nt ? sc[j][lane + 32] : -INFINITY;
@@ -241,7 +294,7 @@ __global__ void __launch_bounds__(128) attn_partial_kernel(
 #pragma unroll
     for (int j = 0; j < kMaxGroup; ++j) acc[j] = 0.f;
     for (int tt = 0; tt < nt; ++tt) {
-        const float vv = __half2float(v_cache[(kv0 + tt) * kHeadDim + d]);
+        const float vv = __half2float(vs[tt][d]);
 #pragma unroll
         for (int j = 0; j < kMaxGroup; ++j)
             if (j < G) acc[j] = fmaf(sc[j][tt], vv, acc[j]);
@@ -260,28 +313,197 @@ __global__ void __launch_bounds__(128) attn_partial_kernel(
 
 // ---- attention: combine the chunk partials in chunk order ----
 // out[m][h][d] = sum_c e^(max_c - M) acc_c[d] / sum_c e^(max_c - M) sum_c, M = max_c max_c.
+// Each chunk's (max, sum) is read by one thread into shared memory (in parallel); the per-d
+// sums then read the acc values with 8 independent loads in flight, summing in chunk order.
+constexpr int kCombineMax = 1024;  // chunks held in shared memory per pass
+// `len` holds the token counts, or (len_is_pos) the new tokens' positions: count = pos + 1.
 __global__ void __launch_bounds__(128) attn_combine_kernel(const float* __restrict__ part,
                                                            const int32_t* __restrict__ len,
-                                                           int Hq, int nchunk, __half* out) {
+                                                           int len_is_pos, int Hq, int nchunk,
+                                                           __half* out) {
     pdl_launch_dependents();
     pdl_wait();
+    __shared__ float fs[kCombineMax], ss[kCombineMax];
+    __shared__ float red[4];
     const int h = blockIdx.x, m = blockIdx.y, d = threadIdx.x;
-    const int nc = (int)((min((int64_t)max(len[m], 0), (int64_t)nchunk * kChunk) + kChunk - 1) /
+    const int64_t n = (int64_t)len[m] + (len_is_pos ? 1 : 0);
+    const int nc = (int)((min(max(n, (int64_t)0), (int64_t)nchunk * kChunk) + kChunk - 1) /
                          kChunk);
     if (nc == 0) {  // no cached token: zeros
         out[((size_t)m * Hq + h) * kHeadDim + d] = __float2half_rn(0.f);
         return;
     }
     const float* pp = part + ((size_t)m * Hq + h) * nchunk * kPartial;
-    float M = -INFINITY;
-    for (int c = 0; c < nc; ++c) M = fmaxf(M, pp[(size_t)c * kPartial + kHeadDim]);
+    // M = max over all chunks (in passes of kCombineMax; max is order-independent)
+    float lm = -INFINITY;
+    for (int cc = d; cc < nc; cc += blockDim.x) lm = fmaxf(lm, pp[(size_t)cc * kPartial + kHeadDim]);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) lm = fmaxf(lm, __shfl_xor_sync(0xffffffffu, lm, o));
+    if ((d & 31) == 0) red[d >> 5] = lm;
+    __syncthreads();
+    const float M = fmaxf(fmaxf(red[0], red[1]), fmaxf(red[2], red[3]));
     float num = 0.f, den = 0.f;
-    for (int c = 0; c < nc; ++c) {
-        const float f = expf(pp[(size_t)c * kPartial + kHeadDim] - M);
-        num = fmaf(f, pp[(size_t)c * kPartial + d], num);
-        den = fmaf(f, pp[(size_t)c * kPartial + kHeadDim + 1], den);
+    for (int c0 = 0; c0 < nc; c0 += kCombineMax) {
+        const int n = min(kCombineMax, nc - c0);
+        __syncthreads();  // the previous pass is done with fs / ss
+        for (int cc = d; cc < n; cc += blockDim.x) {
+            fs[cc] = expf(pp[(size_t)(c0 + cc) * kPartial + kHeadDim] - M);
+            ss[cc] = pp[(size_t)(c0 + cc) * kPartial + kHeadDim + 1];
+        }
+        __syncthreads();
+        int cc = 0;
+        for (; cc + 8 <= n; cc += 8) {
+            float a[8];
+#pragma unroll
+            for (int u = 0; u < 8; ++u) a[u] = pp[(size_t)(c0 + cc + u) * kPartial + d];
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                num = fmaf(fs[cc + u], a[u], num);
+                den = fmaf(fs[cc + u], ss[cc + u], den);
+            }
+        }
+        for (; cc < n; ++cc) {
+            num = fmaf(fs[cc], pp[(size_t)(c0 + cc) * kPartial + d], num);
+            den = fmaf(fs[cc], ss[cc], den);
+        }
     }
     out[((size_t)m * Hq + h) * kHeadDim + d] = __float2half_rn(num / den);
+}
+
+// ---- attention partials with the q/k norm, rotation and cache append folded in ----
+// CTA (chunk c, kv head g, row m), n = clamp(pos[m] + 1, 0, L_max) tokens: the CTA normalises
+// and rotates its G q heads (warp j: head g G + j), stages its chunk's cached K and V, and if
+// the chunk holds position pos[m] (< L_max) computes the new k (norm, rotation) and v, stores
+// them in the caches and uses them in place of the staged row.  Then the chunk partial as in
+// attn_partial_kernel, combined by attn_combine_kernel with len = n.
+__global__ void __launch_bounds__(128) attn_qkv_kernel(
+    const __half* __restrict__ qkv, const __half* __restrict__ qw, const __half* __restrict__ kw,
+    const int32_t* __restrict__ pos, int Hq, int Hkv, float log2_theta, float eps,
+    __half* k_cache, __half* v_cache, int64_t L_max, float scale, float* part, int nchunk) {
+    pdl_launch_dependents();
+    pdl_wait();
+    __shared__ __align__(16) float ksf[kChunk * kHeadDim / 2];  // K rows (fp16), later f_c
+    __shared__ __align__(16) float vsf[kChunk * kHeadDim / 2];  // V rows (fp16), later sum_c
+    __shared__ float qs[kMaxGroup][kHeadDim];
+    __shared__ float sc[kMaxGroup][kChunk];
+    __shared__ float mx[kMaxGroup], sm[kMaxGroup];
+    __half(*ks)[kHeadDim] = reinterpret_cast<__half(*)[kHeadDim]>(ksf);
+    __half(*vs)[kHeadDim] = reinterpret_cast<__half(*)[kHeadDim]>(vsf);
+    const int c = blockIdx.x, g = blockIdx.y, m = blockIdx.z;
+    const int G = Hq / Hkv, nh = Hq + 2 * Hkv;
+    const int64_t p = pos[m];
+    const int n = (int)min(max(p + 1, (int64_t)0), L_max);  // tokens attended
+    const int t0 = c * kChunk;
+    if (t0 >= n) return;
+    const int nt = min(kChunk, n - t0);
+    const bool holds_new = p >= t0 && p < t0 + nt;  // (then p < L_max)
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const size_t kv0 = ((size_t)m * Hkv + g) * L_max + t0;
+    {
+        const uint32_t kss = (uint32_t)__cvta_generic_to_shared(ksf);
+        const uint32_t vss = (uint32_t)__cvta_generic_to_shared(vsf);
+        for (int u = threadIdx.x; u < nt * (kHeadDim / 8); u += blockDim.x) {
+            cp_async16(kss + 16 * u, k_cache + kv0 * kHeadDim + 8 * u);
+            cp_async16(vss + 16 * u, v_cache + kv0 * kHeadDim + 8 * u);
+        }
+        cp_async_commit();
+    }
+    const __half* row = qkv + (size_t)m * nh * kHeadDim;
+    for (int j = warp; j < G; j += 4) {
+        float x[4], o[4];
+        load4(row + (size_t)(g * G + j) * kHeadDim + 4 * lane, x);
+        norm_rope4(x, qw, lane, p, log2_theta, eps, o);
+        const uint2 r = round4(o);  // the fp16 q of the separate path
+        const float2 a = __half22float2(*reinterpret_cast<const __half2*>(&r.x));
+        const float2 b = __half22float2(*reinterpret_cast<const __half2*>(&r.y));
+        qs[j][4 * lane] = scale * a.x;
+        qs[j][4 * lane + 1] = scale * a.y;
+        qs[j][4 * lane + 2] = scale * b.x;
+        qs[j][4 * lane + 3] = scale * b.y;
+    }
+    uint2 knew = make_uint2(0u, 0u), vnew = make_uint2(0u, 0u);
+    if (holds_new && warp < 2) {
+        if (warp == 0) {
+            float x[4], o[4];
+            load4(row + (size_t)(Hq + g) * kHeadDim + 4 * lane, x);
+            norm_rope4(x, kw, lane, p, log2_theta, eps, o);
+            knew = round4(o);
+        } else {
+            vnew = *reinterpret_cast<const uint2*>(row + (size_t)(Hq + Hkv + g) * kHeadDim +
+                                                   4 * lane);
+        }
+    }
+    asm volatile("cp.async.wait_all;\n" ::: "memory");
+    __syncthreads();
+    if (holds_new && warp < 2) {  // the new token replaces the staged (stale) row
+        const int tt = (int)(p - t0);
+        __half* cache = warp == 0 ? k_cache : v_cache;
+        const uint2 w = warp == 0 ? knew : vnew;
+        *reinterpret_cast<uint2*>(warp == 0 ? &ks[tt][4 * lane] : &vs[tt][4 * lane]) = w;
+        *reinterpret_cast<uint2*>(cache + (kv0 + tt) * kHeadDim + 4 * lane) = w;
+    }
+    __syncthreads();
+    const int hl = lane & 15;
+    for (int base = 0; base < nt; base += 8) {
+        const int tt = base + 2 * warp + (lane >> 4);
+        float kv[8];
+        if (tt < nt) {
+            unpack8(*reinterpret_cast<const uint4*>(&ks[tt][8 * hl]), kv);
+        } else {
+#pragma unroll
+            for (int e = 0; e < 8; ++e) kv[e] = 0.f;
+        }
+#pragma unroll
+        for (int j = 0; j < kMaxGroup; ++j) {
+            if (j >= G) break;  // uniform
+            float s = 0.f;
+#pragma unroll
+            for (int e = 0; e < 8; ++e) s = fmaf(qs[j][8 * hl + e], kv[e], s);
+#pragma unroll
+            for (int o = 8; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+            if (hl == 0 && tt < nt) sc[j][tt] = s;
+        }
+    }
+    __syncthreads();
+    for (int j = warp; j < G; j += 4) {
+        const float a = lane < nt ? sc[j][lane] : -INFINITY;
+        const float b = lane + 32 < nt ? sc[j][lane + 32] : -INFINITY;
+        float v = fmaxf(a, b);
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+        const float pa = lane < nt ? expf(a - v) : 0.f;
+        const float pb = lane + 32 < nt ? expf(b - v) : 0.f;
+        if (lane < nt) sc[j][lane] = pa;
+        if (lane + 32 < nt) sc[j][lane + 32] = pb;
+        const float s = warp_sum(pa + pb);
+        if (lane == 0) {
+            mx[j] = v;
+            sm[j] = s;
+        }
+    }
+    __syncthreads();
+    const int d = threadIdx.x;
+    {
+        float acc[kMaxGroup];
+#pragma unroll
+        for (int j = 0; j < kMaxGroup; ++j) acc[j] = 0.f;
+        for (int tt = 0; tt < nt; ++tt) {
+            const float vv = __half2float(vs[tt][d]);
+#pragma unroll
+            for (int j = 0; j < kMaxGroup; ++j)
+                if (j < G) acc[j] = fmaf(sc[j][tt], vv, acc[j]);
+        }
+#pragma unroll
+        for (int j = 0; j < kMaxGroup; ++j) {
+            if (j >= G) break;
+            float* pp = part + (((size_t)m * Hq + g * G + j) * nchunk + c) * kPartial;
+            pp[d] = acc[j];
+            if (d == 0) {
+                pp[kHeadDim] = mx[j];
+                pp[kHeadDim + 1] = sm[j];
+            }
+        }
+    }
 }
 
 // ---- SiLU(gate) * up ----
@@ -319,8 +541,11 @@ __global__ void __launch_bounds__(256) embed_kernel(const __half* __restrict__ E
 
 // ---- greedy argmax (ties: the smallest index; NaN never wins) ----
 constexpr int kArgThreads = 1024;
+// (bv, bi) starts at (-inf, none); a value must beat it strictly, ties between real candidates
+// go to the smaller index, so -inf and NaN never win.
+constexpr int kNone = 0x7fffffff;
 __device__ __forceinline__ void better(float& bv, int& bi, float v, int i) {
-    if (v > bv || (v == bv && i < bi)) {
+    if (v > bv || (v == bv && bi != kNone && i < bi)) {
         bv = v;
         bi = i;
     }
@@ -334,8 +559,31 @@ __global__ void __launch_bounds__(kArgThreads) argmax_kernel(const __half* __res
     const int m = blockIdx.x;
     const __half* row = logits + (size_t)m * V;
     float bv = -INFINITY;
-    int bi = 0x7fffffff;
-    for (int64_t i = threadIdx.x; i < V; i += kArgThreads) better(bv, bi, __half2float(row[i]), (int)i);
+    int bi = kNone;
+    if (((uintptr_t)row & 15u) == 0 && V % 8 == 0) {
+        // 16-byte loads, four in flight per thread
+        const int64_t n8 = V / 8;
+        for (int64_t b = threadIdx.x; b < n8; b += 4 * kArgThreads) {
+            uint4 u[4];
+#pragma unroll
+            for (int r = 0; r < 4; ++r) {
+                const int64_t i8 = b + r * kArgThreads;
+                u[r] = i8 < n8 ? *reinterpret_cast<const uint4*>(row + 8 * i8)
+                               : make_uint4(0xfc00fc00u, 0xfc00fc00u, 0xfc00fc00u, 0xfc00fc00u);
+            }
+#pragma unroll
+            for (int r = 0; r < 4; ++r) {
+                float f[8];
+                unpack8(u[r], f);
+                const int i0 = (int)(8 * (b + r * kArgThreads));
+#pragma unroll
+                for (int e = 0; e < 8; ++e) better(bv, bi, f[e], i0 + e);
+            }
+        }
+    } else {
+        for (int64_t i = threadIdx.x; i < V; i += kArgThreads)
+            better(bv, bi, __half2float(row[i]), (int)i);
+    }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
         const float v = __shfl_xor_sync(0xffffffffu, bv, o);
@@ -351,7 +599,7 @@ __global__ void __launch_bounds__(kArgThreads) argmax_kernel(const __half* __res
         float v = bvs[0];
         int i = bis[0];
         for (int k = 1; k < kArgThreads / 32; ++k) better(v, i, bvs[k], bis[k]);
-        out[m] = i == 0x7fffffff ? 0 : i;  // all NaN / -inf: index 0
+        out[m] = i == kNone ? 0 : i;  // no value above -inf: index 0
     }
 }
 
@@ -431,7 +679,7 @@ laq_status laq_attention_decode(const void* q, const void* k_cache, const void* 
     if (D != kHeadDim || M < 1 || M > 65535 || Hq < 1 || Hkv < 1 || Hq % Hkv ||
         Hq / Hkv > kMaxGroup || Hkv > 65535 || L_max < 1 || !(scale > 0.f))
         return LAQ_ERR_SHAPE;
-    if (!aligned16(k_cache) || ((uintptr_t)q & 1u) || ((uintptr_t)v_cache & 1u) ||
+    if (!aligned16(k_cache) || !aligned16(v_cache) || ((uintptr_t)q & 1u) ||
         ((uintptr_t)out & 1u) || ((uintptr_t)workspace & 3u))
         return LAQ_ERR_ALIGN;
     if (workspace_bytes < laq_attention_workspace_bytes(M, Hq, L_max)) return LAQ_ERR_WORKSPACE;
@@ -446,7 +694,44 @@ laq_status laq_attention_decode(const void* q, const void* k_cache, const void* 
                                scale, static_cast<float*>(workspace), (int)nchunk);
     if (st != LAQ_OK) return st;
     return launch_pdl(attn_combine_kernel, dim3((unsigned)Hq, (unsigned)M), dim3(kHeadDim), s,
-                      static_cast<const float*>(workspace), len, (int)Hq, (int)nchunk,
+                      static_cast<const float*>(workspace), len, 0, (int)Hq, (int)nchunk,
+                      static_cast<__half*>(out));
+}
+
+size_t laq_attention_qkv_workspace_bytes(int64_t M, int32_t Hq, int32_t Hkv, int64_t L_max) {
+    if (M < 1 || Hq < 1 || Hkv < 1 || L_max < 1) return 0;
+    return laq_attention_workspace_bytes(M, Hq, L_max);
+}
+
+laq_status laq_attention_qkv(const void* qkv, const void* q_norm_w, const void* k_norm_w,
+                             const int32_t* pos, int64_t M, int32_t Hq, int32_t Hkv, int32_t D,
+                             float theta, float eps, void* k_cache, void* v_cache, int64_t L_max,
+                             float scale, void* out, void* workspace, size_t workspace_bytes,
+                             void* stream) {
+    if (!qkv || !q_norm_w || !k_norm_w || !pos || !k_cache || !v_cache || !out || !workspace)
+        return LAQ_ERR_NULL;
+    if (D != kHeadDim || M < 1 || M > 65535 || Hq < 1 || Hkv < 1 || Hq % Hkv ||
+        Hq / Hkv > kMaxGroup || Hkv > 65535 || L_max < 1 || !(theta > 1.f) || !(eps >= 0.f) ||
+        !(scale > 0.f))
+        return LAQ_ERR_SHAPE;
+    if (((uintptr_t)qkv & 7u) || !aligned16(k_cache) || !aligned16(v_cache) ||
+        ((uintptr_t)out & 1u) || !aligned16(workspace))
+        return LAQ_ERR_ALIGN;
+    if (workspace_bytes < laq_attention_qkv_workspace_bytes(M, Hq, Hkv, L_max))
+        return LAQ_ERR_WORKSPACE;
+    const int64_t nchunk = (L_max + kChunk - 1) / kChunk;
+    if (nchunk > 0x7fffffff) return LAQ_ERR_SHAPE;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    laq_status st = launch_pdl(attn_qkv_kernel, dim3((unsigned)nchunk, (unsigned)Hkv, (unsigned)M),
+                               dim3(128), s, static_cast<const __half*>(qkv),
+                               static_cast<const __half*>(q_norm_w),
+                               static_cast<const __half*>(k_norm_w), pos, (int)Hq, (int)Hkv,
+                               log2f(theta), eps, static_cast<__half*>(k_cache),
+                               static_cast<__half*>(v_cache), L_max, scale,
+                               static_cast<float*>(workspace), (int)nchunk);
+    if (st != LAQ_OK) return st;
+    return launch_pdl(attn_combine_kernel, dim3((unsigned)Hq, (unsigned)M), dim3(kHeadDim), s,
+                      static_cast<const float*>(workspace), pos, 1, (int)Hq, (int)nchunk,
                       static_cast<__half*>(out));
 }
 

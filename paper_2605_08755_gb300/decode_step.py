@@ -25,9 +25,10 @@ from .weight_pass import QuantLinear, WeightPass
 
 class DecodeStep:
     def __init__(self, model="qwen3-4b", bits=3, M=1, layers=inputs.LAYERS, context=2048,
-                 vocab=None, seed=0, device="cuda"):
+                 vocab=None, seed=0, device="cuda", fused_attention=True):
         dims = inputs.DECODER[model]
         self.model, self.bits, self.M, self.layers = model, bits, M, layers
+        self.fused_attention = fused_attention
         self.context, self.seed = context, seed
         self.H, self.Hq, self.Hkv, self.D, self.I = (dims[k] for k in ("H", "Hq", "Hkv", "D", "I"))
         self.V = vocab or dims["V"]
@@ -76,7 +77,8 @@ class DecodeStep:
         self.d = torch.empty((M, H), **f16)
         self.logits = torch.empty((M, V), **f16)
         self.next = torch.empty((M,), dtype=torch.int32, device=dev)
-        self.ws = _lib.attention_workspace(M, Hq, context, dev)
+        self.ws = (_lib.attention_qkv_workspace(M, Hq, Hkv, context, dev) if fused_attention
+                   else _lib.attention_workspace(M, Hq, context, dev))
         self.scale = 1.0 / math.sqrt(D)
 
     def gemv(self, X, q, Y, cfg, stream):
@@ -96,11 +98,16 @@ class DecodeStep:
                 L.laq_rmsnorm(self.d, nw["in_w"], self.eps, R=self.r, R_out=self.r, Y=self.h,
                               stream=stream)
             self.gemv(self.h, qkv, self.qkv, cf[0], stream)
-            L.laq_qk_norm_rope(self.qkv, nw["q_w"], nw["k_w"], self.pos, self.Hq, self.Hkv,
-                               self.theta, self.eps, self.kc[l], self.vc[l], q_out=self.q,
-                               stream=stream)
-            L.laq_attention_decode(self.q, self.kc[l], self.vc[l], self.lens, self.scale,
-                                   self.ws, out=self.att, stream=stream)
+            if self.fused_attention:  # norm, rotation, cache append and attention: two launches
+                L.laq_attention_qkv(self.qkv, nw["q_w"], nw["k_w"], self.pos, self.Hq, self.Hkv,
+                                    self.theta, self.eps, self.kc[l], self.vc[l], self.scale,
+                                    self.ws, out=self.att, stream=stream)
+            else:
+                L.laq_qk_norm_rope(self.qkv, nw["q_w"], nw["k_w"], self.pos, self.Hq, self.Hkv,
+                                   self.theta, self.eps, self.kc[l], self.vc[l], q_out=self.q,
+                                   stream=stream)
+                L.laq_attention_decode(self.q, self.kc[l], self.vc[l], self.lens, self.scale,
+                                       self.ws, out=self.att, stream=stream)
             self.gemv(self.att, o, self.o, cf[1], stream)
             L.laq_rmsnorm(self.o, nw["post_w"], self.eps, R=self.r, R_out=self.r, Y=self.h,
                           stream=stream)
@@ -113,9 +120,10 @@ class DecodeStep:
 
     @property
     def launches(self):
-        # embed, norm, per layer 4 GEMVs + 2 norms (1 in layer 0) + rope + 2 attention + silu,
-        # final norm, LM head, argmax
-        return 2 + self.layers * 10 - 1 + 3
+        # embed, norm, per layer 4 GEMVs + 2 norms (1 in layer 0) + attention (2 fused, else
+        # rope + 2) + silu, final norm, LM head, argmax
+        per_layer = 9 if self.fused_attention else 10
+        return 2 + self.layers * per_layer - 1 + 3
 
     def capture(self, stream=None):
         self.run()

@@ -132,6 +132,44 @@ def test_attention_workspace_too_small():
     assert e.value.status == 10
 
 
+# ---- attention with the q/k norm, rotation and cache append folded in ----
+
+def oracle_attention_qkv(qkv, qw, kw, pos, Hq, Hkv, kc0, vc0, scale):
+    q, k, v = dec.qk_norm_rope(qkv, qw, kw, pos, Hq, Hkv, 1e6, 1e-6, 128)
+    kc, vc = kc0.copy(), vc0.copy()
+    L = kc.shape[2]
+    for m, p in enumerate(pos):
+        if 0 <= p < L:
+            kc[m, :, p], vc[m, :, p] = k[m], v[m]
+    lens = [min(max(p + 1, 0), L) for p in pos]
+    return dec.attention(q, kc, vc, lens, scale), kc, vc
+
+
+@pytest.mark.parametrize("pos", [[0], [63], [64], [100, 5], [255, 127, 191], [300], [-1, 70]])
+def test_attention_qkv(pos):
+    M, Hq, Hkv, D, L = len(pos), 32, 8, 128, 256
+    qkv = f16(RNG.standard_normal((M, (Hq + 2 * Hkv) * D)) * 2)
+    qw, kw = inputs.norm_weight(D, 21), inputs.norm_weight(D, 22)
+    kc0, vc0 = inputs.kv_cache(M, Hkv, L, D, 23), inputs.kv_cache(M, Hkv, L, D, 24)
+    scale = 1 / math.sqrt(D)
+    ref, rk, rv = oracle_attention_qkv(qkv, qw, kw, pos, Hq, Hkv, kc0, vc0, scale)
+    kc, vc = dev(kc0), dev(vc0)
+    ws = _lib.attention_qkv_workspace(M, Hq, Hkv, L, DEV)
+    args = (dev(qkv), dev(qw), dev(kw), dev(np.array(pos, np.int32)), Hq, Hkv, 1e6, 1e-6, kc, vc,
+            scale, ws)
+    out1 = host(_lib.laq_attention_qkv(*args))
+    out2 = host(_lib.laq_attention_qkv(*args))   # a repeated call agrees bit for bit
+    close(out1, ref, "attention_qkv")
+    assert np.array_equal(out1, out2)
+    close(host(kc), rk, "k cache")
+    kh, vh = host(kc), host(vc)
+    for m, p in enumerate(pos):
+        if not 0 <= p < L:
+            assert np.array_equal(kh[m], kc0[m]) and np.array_equal(vh[m], vc0[m])
+        if p < 0:
+            assert not out1[m].any()
+
+
 # ---- SiLU * up, embedding, argmax ----
 
 @pytest.mark.parametrize("M,I", [(1, 9728), (4, 24)])
@@ -151,17 +189,23 @@ def test_embed_and_argmax():
     logits[2, :] = np.nan
     logits[2, 5000] = 1.0                          # NaN never wins
     logits[3, :] = -np.inf                         # no winner: 0
+    logits[3, 7] = np.nan
     got = host(_lib.laq_argmax(dev(logits)))
     assert list(got) == list(dec.argmax(logits))
     assert got[1] == 77 and got[2] == 5000 and got[3] == 0
+    # unaligned rows (V % 8 != 0) take the scalar path
+    odd = f16(RNG.standard_normal((3, 1001)))
+    odd[2, 1000] = 9.0
+    assert list(host(_lib.laq_argmax(dev(odd)))) == list(dec.argmax(odd))
 
 
 # ---- one whole decode step (2 layers, real Qwen3-4B widths, small vocabulary) ----
 
-@pytest.mark.parametrize("bits,M", [(3, 1), (4, 2)])
-def test_decode_step(bits, M):
+@pytest.mark.parametrize("bits,M,fused", [(3, 1, True), (4, 2, True), (3, 2, False)])
+def test_decode_step(bits, M, fused):
     from paper_2605_08755_gb300.decode_step import DecodeStep
-    st = DecodeStep(bits=bits, M=M, layers=2, context=96, vocab=4096, seed=3)
+    st = DecodeStep(bits=bits, M=M, layers=2, context=96, vocab=4096, seed=3,
+                    fused_attention=fused)
     kc0 = [host(c).copy() for c in st.kc]
     vc0 = [host(c).copy() for c in st.vc]
     tokens = host(st.tokens)
