@@ -53,9 +53,21 @@ __device__ __forceinline__ uint4 pack8(const float (&f)[8]) {
 
 // RMSNorm over a head (lane l holds elements 4l .. 4l+3 of the warp's head), times the norm
 // weights, then the rotate-half rotation at position p; every lane of the warp takes part.
+// The rotation angles of lane l's elements 4l .. 4l+3 at position p: cos and sin of
+// p * theta^(-2i/D), i = the element's index mod D/2 (the same for every head).
+__device__ __forceinline__ void rope_angles(int lane, int64_t p, float log2_theta,
+                                            float (&cs)[4], float (&sn)[4]) {
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+        const int i = (4 * lane + e) & (kHeadDim / 2 - 1);  // frequency index
+        const float inv_freq = exp2f(-(2.f * (float)i / (float)kHeadDim) * log2_theta);
+        sincosf((float)p * inv_freq, &sn[e], &cs[e]);
+    }
+}
+
 __device__ __forceinline__ void norm_rope4(const float (&x)[4], const __half* __restrict__ wn,
-                                           int lane, int64_t p, float log2_theta, float eps,
-                                           float (&o)[4]) {
+                                           int lane, const float (&cs)[4], const float (&sn)[4],
+                                           float eps, float (&o)[4]) {
     float ss = 0.f;
 #pragma unroll
     for (int e = 0; e < 4; ++e) ss = fmaf(x[e], x[e], ss);
@@ -67,11 +79,7 @@ __device__ __forceinline__ void norm_rope4(const float (&x)[4], const __half* __
 #pragma unroll
     for (int e = 0; e < 4; ++e) {
         const float partner = __shfl_xor_sync(0xffffffffu, y[e], 16);
-        const int i = (4 * lane + e) & (kHeadDim / 2 - 1);  // frequency index
-        const float inv_freq = exp2f(-(2.f * (float)i / (float)kHeadDim) * log2_theta);
-        float sn, cs;
-        sincosf((float)p * inv_freq, &sn, &cs);
-        o[e] = lane < 16 ? y[e] * cs - partner * sn : y[e] * cs + partner * sn;
+        o[e] = lane < 16 ? y[e] * cs[e] - partner * sn[e] : y[e] * cs[e] + partner * sn[e];
     }
 }
 
@@ -176,25 +184,9 @@ __global__ void __launch_bounds__(128) qk_norm_rope_kernel(
         const float2 b = __half22float2(*reinterpret_cast<const __half2*>(&raw.y));
         x[0] = a.x; x[1] = a.y; x[2] = b.x; x[3] = b.y;
     }
-    float ss = 0.f;
-#pragma unroll
-    for (int e = 0; e < 4; ++e) ss = fmaf(x[e], x[e], ss);
-    ss = warp_sum(ss);
-    const float inv = rsqrtf(ss / (float)kHeadDim + eps);
-    const __half* wn = head < Hq ? qw : kw;
-    float y[4];
-#pragma unroll
-    for (int e = 0; e < 4; ++e) y[e] = x[e] * inv * __half2float(wn[4 * lane + e]);
-    float o[4];
-#pragma unroll
-    for (int e = 0; e < 4; ++e) {
-        const float partner = __shfl_xor_sync(0xffffffffu, y[e], 16);
-        const int i = (4 * lane + e) & (kHeadDim / 2 - 1);  // frequency index
-        const float inv_freq = exp2f(-(2.f * (float)i / (float)kHeadDim) * log2_theta);
-        float sn, cs;
-        sincosf((float)p * inv_freq, &sn, &cs);
-        o[e] = lane < 16 ? y[e] * cs - partner * sn : y[e] * cs + partner * sn;
-    }
+    float cs[4], sn[4], o[4];
+    rope_angles(lane, p, log2_theta, cs, sn);
+    norm_rope4(x, head < Hq ? qw : kw, lane, cs, sn, eps, o);
     const __half2 lo = __floats2half2_rn(o[0], o[1]), hi = __floats2half2_rn(o[2], o[3]);
     uint2 outw;
     outw.x = *reinterpret_cast<const uint32_t*>(&lo);
@@ -205,6 +197,100 @@ __global__ void __launch_bounds__(128) qk_norm_rope_kernel(
         const int g = head - Hq;
         *reinterpret_cast<uint2*>(k_cache + (((size_t)m * Hkv + g) * L_max + p) * kHeadDim +
                                   4 * lane) = outw;
+    }
+}
+
+// The attention of one 64-token chunk whose K and V rows are staged in shared memory, for the
+// G q heads of a kv head (qs: [G][D] fp32, already scaled), written to the partial slots
+// part[j * nchunk * kPartial] (acc[D], max, sum) of head j.  Scores: a half-warp per token
+// (lane l & 15 holds q and k elements 8 (l & 15) .. +7; q in registers); probabilities stored
+// token-major (sc [kChunk][kMaxGroup]) so that one broadcast load gives every head's value of a
+// token; weighted V sum: warp w takes tokens w, w + 4, ..., lane l dimensions 4l .. 4l+3, then
+// the four warps' sums are added in warp order (red aliases the K rows, no longer needed).
+// Every thread of the CTA must call it.
+__device__ __forceinline__ void chunk_core(const __half (*ks)[kHeadDim],
+                                           const __half (*vs)[kHeadDim], const float* qs,
+                                           float* sc, float* mxs, float* sms, int nt, int G,
+                                           float* part, int nchunk) {
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, hl = lane & 15;
+    float qr[kMaxGroup][8];
+#pragma unroll
+    for (int j = 0; j < kMaxGroup; ++j)
+#pragma unroll
+        for (int e = 0; e < 8; ++e) qr[j][e] = j < G ? qs[j * kHeadDim + 8 * hl + e] : 0.f;
+    for (int base = 0; base < nt; base += 8) {
+        const int tt = base + 2 * warp + (lane >> 4);
+        float kv[8];
+        if (tt < nt) {
+            unpack8(*reinterpret_cast<const uint4*>(&ks[tt][8 * hl]), kv);
+        } else {
+#pragma unroll
+            for (int e = 0; e < 8; ++e) kv[e] = 0.f;
+        }
+#pragma unroll
+        for (int j = 0; j < kMaxGroup; ++j) {
+            if (j >= G) break;  // uniform
+            float s = 0.f;
+#pragma unroll
+            for (int e = 0; e < 8; ++e) s = fmaf(qr[j][e], kv[e], s);
+#pragma unroll
+            for (int o = 8; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+            if (hl == 0 && tt < nt) sc[tt * kMaxGroup + j] = s;
+        }
+    }
+    __syncthreads();
+    for (int j = warp; j < G; j += 4) {
+        const float a = lane < nt ? sc[lane * kMaxGroup + j] : -INFINITY;
+        const float b = lane + 32 < nt ? sc[(lane + 32) * kMaxGroup + j] : -INFINITY;
+        float v = fmaxf(a, b);
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+        const float pa = lane < nt ? expf(a - v) : 0.f;
+        const float pb = lane + 32 < nt ? expf(b - v) : 0.f;
+        if (lane < nt) sc[lane * kMaxGroup + j] = pa;
+        if (lane + 32 < nt) sc[(lane + 32) * kMaxGroup + j] = pb;
+        const float s = warp_sum(pa + pb);
+        if (lane == 0) {
+            mxs[j] = v;
+            sms[j] = s;
+        }
+    }
+    __syncthreads();
+    float acc[kMaxGroup][4];
+#pragma unroll
+    for (int j = 0; j < kMaxGroup; ++j)
+#pragma unroll
+        for (int e = 0; e < 4; ++e) acc[j][e] = 0.f;
+    for (int tt = warp; tt < nt; tt += 4) {
+        float vv[4];
+        load4(&vs[tt][4 * lane], vv);
+        const float4 p0 = *reinterpret_cast<const float4*>(sc + tt * kMaxGroup);
+        const float4 p1 = *reinterpret_cast<const float4*>(sc + tt * kMaxGroup + 4);
+        const float pj[8] = {p0.x, p0.y, p0.z, p0.w, p1.x, p1.y, p1.z, p1.w};
+#pragma unroll
+        for (int j = 0; j < kMaxGroup; ++j)
+            if (j < G)
+#pragma unroll
+                for (int e = 0; e < 4; ++e) acc[j][e] = fmaf(pj[j], vv[e], acc[j][e]);
+    }
+    float* red = reinterpret_cast<float*>(const_cast<__half*>(&ks[0][0]));  // [4][G][D]
+#pragma unroll
+    for (int j = 0; j < kMaxGroup; ++j)
+        if (j < G)
+            *reinterpret_cast<float4*>(red + ((size_t)warp * G + j) * kHeadDim + 4 * lane) =
+                make_float4(acc[j][0], acc[j][1], acc[j][2], acc[j][3]);
+    __syncthreads();
+    const int d = threadIdx.x;
+    for (int j = 0; j < G; ++j) {
+        float a = 0.f;
+#pragma unroll
+        for (int w = 0; w < 4; ++w) a += red[((size_t)w * G + j) * kHeadDim + d];
+        float* pp = part + (size_t)j * nchunk * kPartial;
+        pp[d] = a;
+        if (d == 0) {
+            pp[kHeadDim] = mxs[j];
+            pp[kHeadDim + 1] = sms[j];
+        }
     }
 }
 
@@ -222,8 +308,8 @@ __global__ void __launch_bounds__(128) attn_partial_kernel(
     pdl_wait();
     __shared__ __align__(16) __half ks[kChunk][kHeadDim];
     __shared__ __align__(16) __half vs[kChunk][kHeadDim];
-    __shared__ float qs[kMaxGroup][kHeadDim];
-    __shared__ float sc[kMaxGroup][kChunk];
+    __shared__ __align__(16) float qs[kMaxGroup * kHeadDim];
+    __shared__ __align__(16) float sc[kChunk * kMaxGroup];
     __shared__ float mx[kMaxGroup], sm[kMaxGroup];
     const int c = blockIdx.x, g = blockIdx.y, m = blockIdx.z;
     const int G = Hq / Hkv;
@@ -231,7 +317,6 @@ __global__ void __launch_bounds__(128) attn_partial_kernel(
     const int t0 = c * kChunk;
     if (t0 >= L) return;
     const int nt = min(kChunk, L - t0);
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const size_t kv0 = ((size_t)m * Hkv + g) * L_max + t0;  // row of token t0
     {
         const uint32_t kss = (uint32_t)__cvta_generic_to_shared(&ks[0][0]);
@@ -242,73 +327,12 @@ __global__ void __launch_bounds__(128) attn_partial_kernel(
         }
         cp_async_commit();
     }
-    for (int i = threadIdx.x; i < G * kHeadDim; i += blockDim.x) {
-        const int j = i / kHeadDim, d = i % kHeadDim;
-        qs[j][d] = scale * __half2float(q[((size_t)m * Hq + g * G + j) * kHeadDim + d]);
-    }
+    for (int i = threadIdx.x; i < G * kHeadDim; i += blockDim.x)
+        qs[i] = scale * __half2float(q[((size_t)m * Hq + g * G) * kHeadDim + i]);
     asm volatile("cp.async.wait_all;\n" ::: "memory");
     __syncthreads();
-    // Scores: a half-warp per token, lane l & 15 holding elements 8 (l & 15) .. +7.
-    const int hl = lane & 15;
-    for (int base = 0; base < nt; base += 8) {
-        const int tt = base + 2 * warp + (lane >> 4);
-        float kv[8];
-        if (tt < nt) {
-            unpack8(*reinterpret_cast<const uint4*>(&ks[tt][8 * hl]), kv);
-        } else {
-#pragma unroll
-            for (int e = 0; e < 8; ++e) kv[e] = 0.f;
-        }
-#pragma unroll
-        for (int j = 0; j < kMaxGroup; ++j) {
-            if (j >= G) break;  // uniform
-            float s = 0.f;
-#pragma unroll
-            for (int e = 0; e < 8; ++e) s = fmaf(qs[j][8 * hl + e], kv[e], s);
-#pragma unroll
-            for (int o = 8; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-            if (hl == 0 && tt < nt) sc[j][tt] = s;
-        }
-    }
-    __syncthreads();
-    for (int j = warp; j < G; j += 4) {
-        const float a = lane < nt ? sc[j][lane] : -INFINITY;
-        const float b = lane + 32 < nt ? sc[j][lane + 32] : -INFINITY;
-        float v = fmaxf(a, b);
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
-        const float pa = lane < nt ? expf(a - v) : 0.f;
-        const float pb = lane + 32 < nt ? expf(b - v) : 0.f;
-        if (lane < nt) sc[j][lane] = pa;
-        if (lane + 32 < nt) sc[j][lane + 32] = pb;
-        const float s = warp_sum(pa + pb);
-        if (lane == 0) {
-            mx[j] = v;
-            sm[j] = s;
-        }
-    }
-    __syncthreads();
-    // acc[j][d] = sum_t p[j][t] v[t][d]; thread d
-    const int d = threadIdx.x;
-    float acc[kMaxGroup];
-#pragma unroll
-    for (int j = 0; j < kMaxGroup; ++j) acc[j] = 0.f;
-    for (int tt = 0; tt < nt; ++tt) {
-        const float vv = __half2float(vs[tt][d]);
-#pragma unroll
-        for (int j = 0; j < kMaxGroup; ++j)
-            if (j < G) acc[j] = fmaf(sc[j][tt], vv, acc[j]);
-    }
-#pragma unroll
-    for (int j = 0; j < kMaxGroup; ++j) {
-        if (j >= G) break;
-        float* pp = part + (((size_t)m * Hq + g * G + j) * nchunk + c) * kPartial;
-        pp[d] = acc[j];
-        if (d == 0) {
-            pp[kHeadDim] = mx[j];
-            pp[kHeadDim + 1] = sm[j];
-        }
-    }
+    chunk_core(ks, vs, qs, sc, mx, sm, nt, G,
+               part + (((size_t)m * Hq + g * G) * nchunk + c) * kPartial, nchunk);
 }
 
 // ---- attention: combine the chunk partials in chunk order ----
@@ -382,13 +406,11 @@ __global__ void __launch_bounds__(128) attn_qkv_kernel(
     __half* k_cache, __half* v_cache, int64_t L_max, float scale, float* part, int nchunk) {
     pdl_launch_dependents();
     pdl_wait();
-    __shared__ __align__(16) float ksf[kChunk * kHeadDim / 2];  // K rows (fp16), later f_c
-    __shared__ __align__(16) float vsf[kChunk * kHeadDim / 2];  // V rows (fp16), later sum_c
-    __shared__ float qs[kMaxGroup][kHeadDim];
-    __shared__ float sc[kMaxGroup][kChunk];
+    __shared__ __align__(16) __half ks[kChunk][kHeadDim];
+    __shared__ __align__(16) __half vs[kChunk][kHeadDim];
+    __shared__ __align__(16) float qs[kMaxGroup * kHeadDim];
+    __shared__ __align__(16) float sc[kChunk * kMaxGroup];
     __shared__ float mx[kMaxGroup], sm[kMaxGroup];
-    __half(*ks)[kHeadDim] = reinterpret_cast<__half(*)[kHeadDim]>(ksf);
-    __half(*vs)[kHeadDim] = reinterpret_cast<__half(*)[kHeadDim]>(vsf);
     const int c = blockIdx.x, g = blockIdx.y, m = blockIdx.z;
     const int G = Hq / Hkv, nh = Hq + 2 * Hkv;
     const int64_t p = pos[m];
@@ -400,33 +422,33 @@ __global__ void __launch_bounds__(128) attn_qkv_kernel(
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const size_t kv0 = ((size_t)m * Hkv + g) * L_max + t0;
     {
-        const uint32_t kss = (uint32_t)__cvta_generic_to_shared(ksf);
-        const uint32_t vss = (uint32_t)__cvta_generic_to_shared(vsf);
+        const uint32_t kss = (uint32_t)__cvta_generic_to_shared(&ks[0][0]);
+        const uint32_t vss = (uint32_t)__cvta_generic_to_shared(&vs[0][0]);
         for (int u = threadIdx.x; u < nt * (kHeadDim / 8); u += blockDim.x) {
             cp_async16(kss + 16 * u, k_cache + kv0 * kHeadDim + 8 * u);
             cp_async16(vss + 16 * u, v_cache + kv0 * kHeadDim + 8 * u);
         }
         cp_async_commit();
     }
+    float cs[4], sn[4];
+    rope_angles(lane, p, log2_theta, cs, sn);
     const __half* row = qkv + (size_t)m * nh * kHeadDim;
     for (int j = warp; j < G; j += 4) {
         float x[4], o[4];
         load4(row + (size_t)(g * G + j) * kHeadDim + 4 * lane, x);
-        norm_rope4(x, qw, lane, p, log2_theta, eps, o);
-        const uint2 r = round4(o);  // the fp16 q of the separate path
-        const float2 a = __half22float2(*reinterpret_cast<const __half2*>(&r.x));
-        const float2 b = __half22float2(*reinterpret_cast<const __half2*>(&r.y));
-        qs[j][4 * lane] = scale * a.x;
-        qs[j][4 * lane + 1] = scale * a.y;
-        qs[j][4 * lane + 2] = scale * b.x;
-        qs[j][4 * lane + 3] = scale * b.y;
+        norm_rope4(x, qw, lane, cs, sn, eps, o);
+        const uint2 rq = round4(o);  // the fp16 q of the separate path
+        const float2 a = __half22float2(*reinterpret_cast<const __half2*>(&rq.x));
+        const float2 b = __half22float2(*reinterpret_cast<const __half2*>(&rq.y));
+        *reinterpret_cast<float4*>(qs + j * kHeadDim + 4 * lane) =
+            make_float4(scale * a.x, scale * a.y, scale * b.x, scale * b.y);
     }
     uint2 knew = make_uint2(0u, 0u), vnew = make_uint2(0u, 0u);
     if (holds_new && warp < 2) {
         if (warp == 0) {
             float x[4], o[4];
             load4(row + (size_t)(Hq + g) * kHeadDim + 4 * lane, x);
-            norm_rope4(x, kw, lane, p, log2_theta, eps, o);
+            norm_rope4(x, kw, lane, cs, sn, eps, o);
             knew = round4(o);
         } else {
             vnew = *reinterpret_cast<const uint2*>(row + (size_t)(Hq + Hkv + g) * kHeadDim +
@@ -443,67 +465,8 @@ __global__ void __launch_bounds__(128) attn_qkv_kernel(
         *reinterpret_cast<uint2*>(cache + (kv0 + tt) * kHeadDim + 4 * lane) = w;
     }
     __syncthreads();
-    const int hl = lane & 15;
-    for (int base = 0; base < nt; base += 8) {
-        const int tt = base + 2 * warp + (lane >> 4);
-        float kv[8];
-        if (tt < nt) {
-            unpack8(*reinterpret_cast<const uint4*>(&ks[tt][8 * hl]), kv);
-        } else {
-#pragma unroll
-            for (int e = 0; e < 8; ++e) kv[e] = 0.f;
-        }
-#pragma unroll
-        for (int j = 0; j < kMaxGroup; ++j) {
-            if (j >= G) break;  // uniform
-            float s = 0.f;
-#pragma unroll
-            for (int e = 0; e < 8; ++e) s = fmaf(qs[j][8 * hl + e], kv[e], s);
-#pragma unroll
-            for (int o = 8; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-            if (hl == 0 && tt < nt) sc[j][tt] = s;
-        }
-    }
-    __syncthreads();
-    for (int j = warp; j < G; j += 4) {
-        const float a = lane < nt ? sc[j][lane] : -INFINITY;
-        const float b = lane + 32 < nt ? sc[j][lane + 32] : -INFINITY;
-        float v = fmaxf(a, b);
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
-        const float pa = lane < nt ? expf(a - v) : 0.f;
-        const float pb = lane + 32 < nt ? expf(b - v) : 0.f;
-        if (lane < nt) sc[j][lane] = pa;
-        if (lane + 32 < nt) sc[j][lane + 32] = pb;
-        const float s = warp_sum(pa + pb);
-        if (lane == 0) {
-            mx[j] = v;
-            sm[j] = s;
-        }
-    }
-    __syncthreads();
-    const int d = threadIdx.x;
-    {
-        float acc[kMaxGroup];
-#pragma unroll
-        for (int j = 0; j < kMaxGroup; ++j) acc[j] = 0.f;
-        for (int tt = 0; tt < nt; ++tt) {
-            const float vv = __half2float(vs[tt][d]);
-#pragma unroll
-            for (int j = 0; j < kMaxGroup; ++j)
-                if (j < G) acc[j] = fmaf(sc[j][tt], vv, acc[j]);
-        }
-#pragma unroll
-        for (int j = 0; j < kMaxGroup; ++j) {
-            if (j >= G) break;
-            float* pp = part + (((size_t)m * Hq + g * G + j) * nchunk + c) * kPartial;
-            pp[d] = acc[j];
-            if (d == 0) {
-                pp[kHeadDim] = mx[j];
-                pp[kHeadDim + 1] = sm[j];
-            }
-        }
-    }
+    chunk_core(ks, vs, qs, sc, mx, sm, nt, G,
+               part + (((size_t)m * Hq + g * G) * nchunk + c) * kPartial, nchunk);
 }
 
 // ---- SiLU(gate) * up ----
