@@ -335,63 +335,85 @@ __global__ void __launch_bounds__(128) attn_partial_kernel(
                part + (((size_t)m * Hq + g * G) * nchunk + c) * kPartial, nchunk);
 }
 
-// ---- attention: combine the chunk partials in chunk order ----
+// ---- attention: combine the chunk partials ----
 // out[m][h][d] = sum_c e^(max_c - M) acc_c[d] / sum_c e^(max_c - M) sum_c, M = max_c max_c.
-// Each chunk's (max, sum) is read by one thread into shared memory (in parallel); the per-d
-// sums then read the acc values with 8 independent loads in flight, summing in chunk order.
-constexpr int kCombineMax = 1024;  // chunks held in shared memory per pass
-// `len` holds the token counts, or (len_is_pos) the new tokens' positions: count = pos + 1.
-__global__ void __launch_bounds__(128) attn_combine_kernel(const float* __restrict__ part,
-                                                           const int32_t* __restrict__ len,
-                                                           int len_is_pos, int Hq, int nchunk,
-                                                           __half* out) {
+// 512 threads: each chunk's (max, sum) is read once, by one thread, into shared memory; the
+// four 128-thread groups q take the chunks c = q mod 4 (8 independent loads in flight per
+// thread) and their sums are added in group order; the denominator by warp 0.  Fixed orders:
+// the result is deterministic.
+constexpr int kCombineMax = 2048;  // chunks held in shared memory per pass
+constexpr int kCombineThreads = 512;
+__global__ void __launch_bounds__(kCombineThreads) attn_combine_kernel(
+    const float* __restrict__ part, const int32_t* __restrict__ len, int len_is_pos, int Hq,
+    int nchunk, __half* out) {
     pdl_launch_dependents();
     pdl_wait();
     __shared__ float fs[kCombineMax], ss[kCombineMax];
-    __shared__ float red[4];
-    const int h = blockIdx.x, m = blockIdx.y, d = threadIdx.x;
+    __shared__ float red[kCombineThreads / 32];
+    __shared__ float nums[4][kHeadDim];
+    __shared__ float den_s;
+    const int h = blockIdx.x, m = blockIdx.y, tid = threadIdx.x;
+    const int d = tid & (kHeadDim - 1), q = tid >> 7;
     const int64_t n = (int64_t)len[m] + (len_is_pos ? 1 : 0);
     const int nc = (int)((min(max(n, (int64_t)0), (int64_t)nchunk * kChunk) + kChunk - 1) /
                          kChunk);
+    __half* o = out + ((size_t)m * Hq + h) * kHeadDim;
     if (nc == 0) {  // no cached token: zeros
-        out[((size_t)m * Hq + h) * kHeadDim + d] = __float2half_rn(0.f);
+        if (q == 0) o[d] = __float2half_rn(0.f);
         return;
     }
     const float* pp = part + ((size_t)m * Hq + h) * nchunk * kPartial;
-    // M = max over all chunks (in passes of kCombineMax; max is order-independent)
+    // M = max over all chunks (order-independent); the first pass's (max, sum) stay in smem
+    const int n0 = min(kCombineMax, nc);
     float lm = -INFINITY;
-    for (int cc = d; cc < nc; cc += blockDim.x) lm = fmaxf(lm, pp[(size_t)cc * kPartial + kHeadDim]);
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) lm = fmaxf(lm, __shfl_xor_sync(0xffffffffu, lm, o));
-    if ((d & 31) == 0) red[d >> 5] = lm;
-    __syncthreads();
-    const float M = fmaxf(fmaxf(red[0], red[1]), fmaxf(red[2], red[3]));
-    float num = 0.f, den = 0.f;
-    for (int c0 = 0; c0 < nc; c0 += kCombineMax) {
-        const int n = min(kCombineMax, nc - c0);
-        __syncthreads();  // the previous pass is done with fs / ss
-        for (int cc = d; cc < n; cc += blockDim.x) {
-            fs[cc] = expf(pp[(size_t)(c0 + cc) * kPartial + kHeadDim] - M);
-            ss[cc] = pp[(size_t)(c0 + cc) * kPartial + kHeadDim + 1];
-        }
-        __syncthreads();
-        int cc = 0;
-        for (; cc + 8 <= n; cc += 8) {
-            float a[8];
-#pragma unroll
-            for (int u = 0; u < 8; ++u) a[u] = pp[(size_t)(c0 + cc + u) * kPartial + d];
-#pragma unroll
-            for (int u = 0; u < 8; ++u) {
-                num = fmaf(fs[cc + u], a[u], num);
-                den = fmaf(fs[cc + u], ss[cc + u], den);
-            }
-        }
-        for (; cc < n; ++cc) {
-            num = fmaf(fs[cc], pp[(size_t)(c0 + cc) * kPartial + d], num);
-            den = fmaf(fs[cc], ss[cc], den);
+    for (int cc = tid; cc < nc; cc += kCombineThreads) {
+        const float mc = pp[(size_t)cc * kPartial + kHeadDim];
+        lm = fmaxf(lm, mc);
+        if (cc < n0) {
+            fs[cc] = mc;
+            ss[cc] = pp[(size_t)cc * kPartial + kHeadDim + 1];
         }
     }
-    out[((size_t)m * Hq + h) * kHeadDim + d] = __float2half_rn(num / den);
+#pragma unroll
+    for (int w = 16; w > 0; w >>= 1) lm = fmaxf(lm, __shfl_xor_sync(0xffffffffu, lm, w));
+    if ((tid & 31) == 0) red[tid >> 5] = lm;
+    __syncthreads();
+    float M = red[0];
+#pragma unroll
+    for (int k = 1; k < kCombineThreads / 32; ++k) M = fmaxf(M, red[k]);
+    float num = 0.f, dl = 0.f;  // dl: warp 0's share of the denominator
+    for (int c0 = 0; c0 < nc; c0 += kCombineMax) {
+        const int cnt = min(kCombineMax, nc - c0);
+        if (c0 > 0) {
+            __syncthreads();  // the previous pass is done with fs / ss
+            for (int cc = tid; cc < cnt; cc += kCombineThreads) {
+                fs[cc] = pp[(size_t)(c0 + cc) * kPartial + kHeadDim];
+                ss[cc] = pp[(size_t)(c0 + cc) * kPartial + kHeadDim + 1];
+            }
+        }
+        __syncthreads();
+        for (int cc = tid; cc < cnt; cc += kCombineThreads) fs[cc] = expf(fs[cc] - M);
+        __syncthreads();
+        if (tid < 32)
+            for (int cc = tid; cc < cnt; cc += 32) dl = fmaf(fs[cc], ss[cc], dl);
+        int cc = q;
+        for (; cc + 28 < cnt; cc += 32) {  // 8 chunks of this group per round
+            float a[8];
+#pragma unroll
+            for (int u = 0; u < 8; ++u) a[u] = pp[(size_t)(c0 + cc + 4 * u) * kPartial + d];
+#pragma unroll
+            for (int u = 0; u < 8; ++u) num = fmaf(fs[cc + 4 * u], a[u], num);
+        }
+        for (; cc < cnt; cc += 4) num = fmaf(fs[cc], pp[(size_t)(c0 + cc) * kPartial + d], num);
+    }
+    if (tid < 32) {
+        dl = warp_sum(dl);
+        if (tid == 0) den_s = dl;
+    }
+    nums[q][d] = num;
+    __syncthreads();
+    if (q == 0)
+        o[d] = __float2half_rn((nums[0][d] + nums[1][d] + nums[2][d] + nums[3][d]) / den_s);
 }
 
 // ---- attention partials with the q/k norm, rotation and cache append folded in ----
@@ -656,9 +678,9 @@ laq_status laq_attention_decode(const void* q, const void* k_cache, const void* 
                                static_cast<const __half*>(v_cache), len, (int)Hq, (int)Hkv, L_max,
                                scale, static_cast<float*>(workspace), (int)nchunk);
     if (st != LAQ_OK) return st;
-    return launch_pdl(attn_combine_kernel, dim3((unsigned)Hq, (unsigned)M), dim3(kHeadDim), s,
-                      static_cast<const float*>(workspace), len, 0, (int)Hq, (int)nchunk,
-                      static_cast<__half*>(out));
+    return launch_pdl(attn_combine_kernel, dim3((unsigned)Hq, (unsigned)M),
+                      dim3(kCombineThreads), s, static_cast<const float*>(workspace), len, 0,
+                      (int)Hq, (int)nchunk, static_cast<__half*>(out));
 }
 
 size_t laq_attention_qkv_workspace_bytes(int64_t M, int32_t Hq, int32_t Hkv, int64_t L_max) {
@@ -693,9 +715,9 @@ laq_status laq_attention_qkv(const void* qkv, const void* q_norm_w, const void* 
                                static_cast<__half*>(v_cache), L_max, scale,
                                static_cast<float*>(workspace), (int)nchunk);
     if (st != LAQ_OK) return st;
-    return launch_pdl(attn_combine_kernel, dim3((unsigned)Hq, (unsigned)M), dim3(kHeadDim), s,
-                      static_cast<const float*>(workspace), pos, 1, (int)Hq, (int)nchunk,
-                      static_cast<__half*>(out));
+    return launch_pdl(attn_combine_kernel, dim3((unsigned)Hq, (unsigned)M),
+                      dim3(kCombineThreads), s, static_cast<const float*>(workspace), pos, 1,
+                      (int)Hq, (int)nchunk, static_cast<__half*>(out));
 }
 
 laq_status laq_silu_mul(const void* gate_up, int64_t M, int64_t I, void* h, void* stream) {
