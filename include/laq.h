@@ -243,6 +243,42 @@ laq_status laq_gemm_chain(const laq_gemv *gemvs, int32_t count, void *workspace,
  */
 laq_status laq_gemm_chain_static(const laq_gemv *gemvs, int32_t count, void *stream);
 
+/*
+ * A prologue applied to X while laq_gemm_wxg128_prologue stages it, so that the operation
+ * before a projection costs no launch of its own.  The paper has no counterpart: this fuses two
+ * of the decoder operations declared below (laq_rmsnorm, laq_silu_mul) into the GEMV.
+ *   LAQ_PROLOGUE_RMSNORM: the GEMV's input is laq_rmsnorm's Y of (X [M][K], R, w, eps):
+ *     h = fp16(X + R) (h = X when R is NULL), input = fp16(h / sqrt(mean_k h^2 + eps) * w),
+ *     and when R_out is not NULL, R_out = h [M][K].  R_out must not alias X or R (CTAs read the
+ *     whole rows of X and R while one of them writes R_out): LAQ_ERR_SHAPE otherwise.
+ *   LAQ_PROLOGUE_SILU_MUL: X holds [M][2K] (gate | up); input = fp16(silu(gate) * up), as
+ *     laq_silu_mul.
+ * X, R, R_out and w 16-byte aligned.
+ */
+#define LAQ_PROLOGUE_NONE 0
+#define LAQ_PROLOGUE_RMSNORM 1
+#define LAQ_PROLOGUE_SILU_MUL 2
+typedef struct laq_gemm_prologue {
+    int32_t kind;
+    float eps;          /* RMSNORM */
+    const void *R;      /* RMSNORM: residual [M][K] or NULL */
+    void *R_out;        /* RMSNORM: receives fp16(X + R) [M][K], or NULL */
+    const void *w;      /* RMSNORM: weights [K] */
+} laq_gemm_prologue;
+
+/* laq_gemm_wxg128 with a prologue on X (pro NULL or kind NONE: plain) and an optional explicit
+ * configuration (cfg NULL: planned; laq_gemm_wxg128_config's rules otherwise).  All pointers are
+ * device pointers owned by the caller; Y [M][N] is overwritten.  Results equal those of the
+ * unfused sequence within fp16 rounding: the row's sum of squares is added in another order, and
+ * SILU_MUL uses the hardware exponential and reciprocal (relative error ~2^-21).  Errors: as
+ * laq_gemm_wxg128, plus LAQ_ERR_CONFIG for an unknown kind, LAQ_ERR_NULL for RMSNORM without
+ * w, LAQ_ERR_SHAPE for eps < 0 (or NaN) or R_out equal to X or R, LAQ_ERR_ALIGN for a
+ * misaligned X, R, R_out or w. */
+laq_status laq_gemm_wxg128_prologue(const void *X, int64_t M, int64_t K, int64_t N,
+                                    const void *packed, const void *s, const uint8_t *z, int bits,
+                                    void *Y, const laq_gemm_prologue *pro,
+                                    const laq_gemm_config *cfg, void *stream);
+
 /* ======================================================================================
  * Decoder operations around the projections: the rest of one decode step of a Qwen3-style
  * model (the models whose decoding speed Sec. 5.2 reports).  The paper defines none of them;

@@ -100,7 +100,8 @@ def silu_mul(gate_up):
     gu = _f64(gate_up)
     I = gu.shape[1] // 2
     g, u = gu[:, :I], gu[:, I:]
-    return _f16(g / (1.0 + np.exp(-g)) * u)
+    with np.errstate(over="ignore"):  # g << 0: e^-g = inf and g / inf = -0, silu's limit
+        return _f16(g / (1.0 + np.exp(-g)) * u)
 
 
 def embed(E, tokens):

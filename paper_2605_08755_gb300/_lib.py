@@ -20,6 +20,7 @@ STATUS = {0: "LAQ_OK", 1: "LAQ_ERR_NULL", 2: "LAQ_ERR_BITS", 3: "LAQ_ERR_GROUP",
 EXPORTS = ("laq_status_str", "laq_version", "laq_packed_bytes", "laq_quantize_rtn", "laq_pack",
            "laq_unpack", "laq_gemm_wxg128", "laq_gemm_plan", "laq_gemm_wxg128_config",
            "laq_chain_workspace_bytes", "laq_gemm_chain", "laq_gemm_chain_static",
+           "laq_gemm_wxg128_prologue",
            "laq_rmsnorm", "laq_qk_norm_rope", "laq_attention_workspace_bytes",
            "laq_attention_decode", "laq_attention_qkv_workspace_bytes", "laq_attention_qkv",
            "laq_silu_mul", "laq_embed", "laq_argmax")
@@ -44,6 +45,15 @@ class GemmConfig(ctypes.Structure):
     @classmethod
     def make(cls, tiles_per_cta, warps, cluster, stages, pdl=0):
         return cls(tiles_per_cta, warps, cluster, stages, pdl, (ctypes.c_int32 * 3)(0, 0, 0))
+
+
+class GemmPrologue(ctypes.Structure):
+    """struct laq_gemm_prologue."""
+    _fields_ = [("kind", ctypes.c_int32), ("eps", ctypes.c_float), ("R", ctypes.c_void_p),
+                ("R_out", ctypes.c_void_p), ("w", ctypes.c_void_p)]
+
+
+PROLOGUE_NONE, PROLOGUE_RMSNORM, PROLOGUE_SILU_MUL = 0, 1, 2
 
 
 class Gemv(ctypes.Structure):
@@ -74,6 +84,9 @@ def lib():
     L.laq_gemm_plan.argtypes = [I64, I64, I64, I, I, ctypes.POINTER(GemmConfig)]
     L.laq_gemm_wxg128_config.argtypes = [P, I64, I64, I64, P, P, P, I, P,
                                          ctypes.POINTER(GemmConfig), P]
+    L.laq_gemm_wxg128_prologue.argtypes = [P, I64, I64, I64, P, P, P, I, P,
+                                           ctypes.POINTER(GemmPrologue),
+                                           ctypes.POINTER(GemmConfig), P]
     L.laq_chain_workspace_bytes.argtypes = [ctypes.c_int32]
     L.laq_chain_workspace_bytes.restype = ctypes.c_size_t
     L.laq_gemm_chain.argtypes = [ctypes.POINTER(Gemv), ctypes.c_int32, P, ctypes.c_size_t, P]
@@ -94,6 +107,7 @@ def lib():
     for name in ("laq_quantize_rtn", "laq_pack", "laq_unpack", "laq_gemm_wxg128",
                  "laq_gemm_plan", "laq_gemm_wxg128_config", "laq_gemm_chain",
                  "laq_gemm_chain_static", "laq_rmsnorm", "laq_qk_norm_rope",
+                 "laq_gemm_wxg128_prologue",
                  "laq_attention_decode", "laq_attention_qkv_workspace_bytes", "laq_attention_qkv",
            "laq_silu_mul", "laq_embed", "laq_argmax"):
         getattr(L, name).restype = I
@@ -164,6 +178,26 @@ def laq_gemm_wxg128(X, packed, s, z, bits, Y=None, config=None, stream=None):
     else:
         _check(lib().laq_gemm_wxg128_config(*args, ctypes.byref(config), _stream(stream)),
                "laq_gemm_wxg128_config")
+    return Y
+
+
+def laq_gemm_wxg128_prologue(X, packed, s, z, bits, kind, Y=None, R=None, R_out=None, w=None,
+                             eps=0.0, config=None, stream=None):
+    """laq_gemm_wxg128 whose input is a prologue of X: PROLOGUE_RMSNORM (rmsnorm(X + R) * w,
+    R_out = fp16(X + R)) or PROLOGUE_SILU_MUL (X [M, 2K] = gate | up -> silu(gate) * up)."""
+    import torch
+    M = X.shape[0]
+    K = X.shape[1] // 2 if kind == PROLOGUE_SILU_MUL else X.shape[1]
+    N = s.shape[1]
+    if Y is None:
+        Y = torch.empty((M, N), dtype=torch.float16, device=X.device)
+    pro = GemmPrologue(kind, float(eps), None if R is None else R.data_ptr(),
+                       None if R_out is None else R_out.data_ptr(),
+                       None if w is None else w.data_ptr())
+    _check(lib().laq_gemm_wxg128_prologue(_ptr(X), M, K, N, _ptr(packed), _ptr(s), _ptr(z), bits,
+                                          _ptr(Y), ctypes.byref(pro),
+                                          None if config is None else ctypes.byref(config),
+                                          _stream(stream)), "laq_gemm_wxg128_prologue")
     return Y
 
 

@@ -15,7 +15,8 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD_DIR = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "liblaq.so")
-SOURCES = ("laq_api.cu", "laq_quant.cu", "laq_gemm.cu", "laq_chain.cu", "laq_decode.cu")
+SOURCES = ("laq_api.cu", "laq_quant.cu", "laq_gemm.cu", "laq_gemm_prologue.cu", "laq_chain.cu",
+           "laq_decode.cu")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

@@ -175,9 +175,22 @@ void plan(int64_t M, int64_t K, int64_t N, int bits, int sms, laq_gemm_config* o
 
 laq_status run_gemm(const void* X, int64_t M, int64_t K, int64_t N, const void* packed,
                     const void* s, const uint8_t* z, int bits, void* Y,
-                    const laq_gemm_config* cfg, void* stream) {
+                    const laq_gemm_config* cfg, void* stream,
+                    const laq_gemm_prologue* pro = nullptr) {
     laq_status st = check_gemm_args(X, M, K, N, packed, s, z, bits, Y);
     if (st != LAQ_OK) return st;
+    const int kind = pro ? pro->kind : LAQ_PROLOGUE_NONE;
+    if (kind != LAQ_PROLOGUE_NONE && kind != LAQ_PROLOGUE_RMSNORM && kind != LAQ_PROLOGUE_SILU_MUL)
+        return LAQ_ERR_CONFIG;
+    if (kind == LAQ_PROLOGUE_RMSNORM) {
+        if (!pro->w) return LAQ_ERR_NULL;
+        if (!(pro->eps >= 0.f)) return LAQ_ERR_SHAPE;
+        if (pro->R_out && (pro->R_out == X || pro->R_out == pro->R)) return LAQ_ERR_SHAPE;
+        if (((uintptr_t)pro->w & 15u) || ((uintptr_t)pro->R & 15u) ||
+            ((uintptr_t)pro->R_out & 15u))
+            return LAQ_ERR_ALIGN;
+    }
+    if (kind != LAQ_PROLOGUE_NONE && ((uintptr_t)X & 15u)) return LAQ_ERR_ALIGN;
     if (cfg) {
         st = check_config(cfg);
         if (st != LAQ_OK) return st;
@@ -209,6 +222,14 @@ laq_status run_gemm(const void* X, int64_t M, int64_t K, int64_t N, const void* 
     L.cluster = c.cluster;
     L.stages = c.stages;
     L.pdl = c.pdl;
+    L.pro = kind == LAQ_PROLOGUE_RMSNORM ? laq::kProRmsNorm
+            : kind == LAQ_PROLOGUE_SILU_MUL ? laq::kProSiluMul : laq::kProNone;
+    if (kind == LAQ_PROLOGUE_RMSNORM) {
+        L.eps = pro->eps;
+        L.R = static_cast<const uint16_t*>(pro->R);
+        L.R_out = static_cast<uint16_t*>(pro->R_out);
+        L.w = static_cast<const uint16_t*>(pro->w);
+    }
     return from_cuda(laq::launch_gemm(L, f.smem_optin, strm));
 }
 
@@ -437,6 +458,13 @@ laq_status laq_gemm_wxg128_config(const void* X, int64_t M, int64_t K, int64_t N
                                   void* Y, const laq_gemm_config* cfg, void* stream) {
     if (!cfg) return LAQ_ERR_NULL;
     return run_gemm(X, M, K, N, packed, s, z, bits, Y, cfg, stream);
+}
+
+laq_status laq_gemm_wxg128_prologue(const void* X, int64_t M, int64_t K, int64_t N,
+                                    const void* packed, const void* s, const uint8_t* z, int bits,
+                                    void* Y, const laq_gemm_prologue* pro,
+                                    const laq_gemm_config* cfg, void* stream) {
+    return run_gemm(X, M, K, N, packed, s, z, bits, Y, cfg, stream, pro);
 }
 
 size_t laq_chain_workspace_bytes(int32_t count) {

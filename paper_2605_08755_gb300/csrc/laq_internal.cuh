@@ -21,7 +21,14 @@ struct GemmLaunch {
     uint16_t* Y;
     int M, K, N, bits;
     int tiles_per_cta, warps, cluster, stages, pdl;
+    // X prologue (kPro*): the GEMV's input is RMSNorm(X + R) * w, or SiLU(gate) * up of X
+    int pro = 0;
+    float eps = 0.f;
+    const uint16_t* R = nullptr;
+    uint16_t* R_out = nullptr;
+    const uint16_t* w = nullptr;
 };
+constexpr int kProNone = 0, kProRmsNorm = 1, kProSiluMul = 2;
 
 // Dynamic shared memory the GEMM kernel needs for this launch (bytes), and the groups of X it
 // stages per phase.

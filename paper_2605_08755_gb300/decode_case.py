@@ -104,10 +104,11 @@ def main():
     ap.add_argument("--replays", type=int, default=50)
     ap.add_argument("--fp16", action="store_true")
     ap.add_argument("--separate-attention", action="store_true")
+    ap.add_argument("--separate-norms", action="store_true")
     a = ap.parse_args()
     torch.cuda.set_device(0)
     st = DecodeStep(model=a.model, bits=a.bits, M=a.M, layers=a.layers, context=a.context,
-                    fused_attention=not a.separate_attention)
+                    fused_attention=not a.separate_attention, fused_norms=not a.separate_norms)
     stream = torch.cuda.Stream()
     g = st.capture(stream=stream)
     us = time_graph(g, stream, a.replays)

@@ -25,10 +25,11 @@ from .weight_pass import QuantLinear, WeightPass
 
 class DecodeStep:
     def __init__(self, model="qwen3-4b", bits=3, M=1, layers=inputs.LAYERS, context=2048,
-                 vocab=None, seed=0, device="cuda", fused_attention=True):
+                 vocab=None, seed=0, device="cuda", fused_attention=True, fused_norms=True):
         dims = inputs.DECODER[model]
         self.model, self.bits, self.M, self.layers = model, bits, M, layers
         self.fused_attention = fused_attention
+        self.fused_norms = fused_norms  # the layers' RMSNorms folded into the next GEMV
         self.context, self.seed = context, seed
         self.H, self.Hq, self.Hkv, self.D, self.I = (dims[k] for k in ("H", "Hq", "Hkv", "D", "I"))
         self.V = vocab or dims["V"]
@@ -67,6 +68,7 @@ class DecodeStep:
         f16 = dict(dtype=torch.float16, device=dev)
         self.x = torch.empty((M, H), **f16)
         self.r = torch.empty((M, H), **f16)
+        self.r2 = torch.empty((M, H), **f16)  # the residual's other buffer (fused norms)
         self.h = torch.empty((M, H), **f16)
         self.qkv = torch.empty((M, (Hq + 2 * Hkv) * D), **f16)
         self.q = torch.empty((M, Hq, D), **f16)
@@ -88,6 +90,8 @@ class DecodeStep:
     def run(self, stream=None):
         """Launch one step on ``stream``: reads tokens, pos, the caches; writes the caches at pos,
         logits and next (the greedy tokens)."""
+        if self.fused_norms:
+            return self.run_fused(stream)
         L = _lib
         _lib.laq_embed(self.E, self.tokens, X=self.x, stream=stream)
         L.laq_rmsnorm(self.x, self.norms[0]["in_w"], self.eps, R_out=self.r, Y=self.h,
@@ -118,10 +122,48 @@ class DecodeStep:
         self.gemv(self.h, self.lm, self.logits, self.lm_cfg, stream)
         L.laq_argmax(self.logits, out=self.next, stream=stream)
 
+    def run_fused(self, stream=None):
+        """The same step with the two RMSNorms of each layer (and their residual adds) folded into
+        the X staging of the q|k|v and gate|up GEMVs (laq_gemm_wxg128_prologue); the residual
+        alternates between two buffers, since a prologue's residual output may not alias its
+        inputs.  SiLU*up and the final norm stay separate kernels: on GB300 their prologue forms
+        measured slower (every CTA of the down GEMV recomputes SiLU over its K range before its
+        first MMA; the LM head's ~1200 CTAs each redo the row norm)."""
+        L = _lib
+        RMS = _lib.PROLOGUE_RMSNORM
+        L.laq_embed(self.E, self.tokens, X=self.x, stream=stream)
+        res, nxt = self.r, self.r2
+        for l in range(self.layers):
+            nw, (qkv, o, gu, dn), cf = self.norms[l], self.proj[l], self.cfg[l]
+            if l == 0:  # r = x
+                L.laq_gemm_wxg128_prologue(self.x, qkv.packed, qkv.s, qkv.z, qkv.bits, RMS,
+                                           Y=self.qkv, R_out=res, w=nw["in_w"], eps=self.eps,
+                                           config=cf[0], stream=stream)
+            else:       # r += d
+                L.laq_gemm_wxg128_prologue(self.d, qkv.packed, qkv.s, qkv.z, qkv.bits, RMS,
+                                           Y=self.qkv, R=res, R_out=nxt, w=nw["in_w"],
+                                           eps=self.eps, config=cf[0], stream=stream)
+                res, nxt = nxt, res
+            L.laq_attention_qkv(self.qkv, nw["q_w"], nw["k_w"], self.pos, self.Hq, self.Hkv,
+                                self.theta, self.eps, self.kc[l], self.vc[l], self.scale, self.ws,
+                                out=self.att, stream=stream)
+            self.gemv(self.att, o, self.o, cf[1], stream)
+            L.laq_gemm_wxg128_prologue(self.o, gu.packed, gu.s, gu.z, gu.bits, RMS, Y=self.gu,
+                                       R=res, R_out=nxt, w=nw["post_w"], eps=self.eps,
+                                       config=cf[2], stream=stream)
+            res, nxt = nxt, res
+            L.laq_silu_mul(self.gu, h=self.act, stream=stream)
+            self.gemv(self.act, dn, self.d, cf[3], stream)
+        L.laq_rmsnorm(self.d, self.final_w, self.eps, R=res, Y=self.h, stream=stream)
+        self.gemv(self.h, self.lm, self.logits, self.lm_cfg, stream)
+        L.laq_argmax(self.logits, out=self.next, stream=stream)
+
     @property
     def launches(self):
         # embed, norm, per layer 4 GEMVs + 2 norms (1 in layer 0) + attention (2 fused, else
         # rope + 2) + silu, final norm, LM head, argmax
+        if self.fused_norms:  # embed, per layer 4 GEMVs + 2 attention + silu, norm, LM head, argmax
+            return 1 + self.layers * 7 + 3
         per_layer = 9 if self.fused_attention else 10
         return 2 + self.layers * per_layer - 1 + 3
 

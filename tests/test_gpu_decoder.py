@@ -199,13 +199,71 @@ def test_embed_and_argmax():
     assert list(host(_lib.laq_argmax(dev(odd)))) == list(dec.argmax(odd))
 
 
+# ---- GEMV with the RMSNorm or SiLU*up prologue ----
+
+def quantized(K, N, bits, seed):
+    from oracle import c_oracle
+    W = inputs.weights(K, N, seed=seed)
+    codes, s, z = c_oracle.quantize_rtn(W, bits)
+    packed = laq.laq_pack(dev(codes), bits)
+    return (codes, s, z), (packed, dev(s), dev(z))
+
+
+CFG = [None, laq.GemmConfig.make(2, 4, 8, 3, 1), laq.GemmConfig.make(1, 8, 1, 16, 0)]
+
+
+@pytest.mark.parametrize("M", [1, 3, 16])
+@pytest.mark.parametrize("ci", [0, 1, 2])
+@pytest.mark.parametrize("with_r", [False, True])
+def test_gemm_rmsnorm_prologue(M, ci, with_r):
+    K, N, bits = 2560, 272, 3
+    ref_q, (packed, s, z) = quantized(K, N, bits, seed=40 + M)
+    x = f16(RNG.standard_normal((M, K)))
+    r = f16(RNG.standard_normal((M, K)) * 2)
+    w = inputs.norm_weight(K, seed=5)
+    y_in, h = dec.rmsnorm(x, w, 1e-6, r if with_r else None)
+    ref = dec.linear(y_in, ref_q)
+    rd = dev(r)
+    r_out = torch.zeros((M, K), dtype=torch.float16, device=DEV)
+    Y = _lib.laq_gemm_wxg128_prologue(dev(x), packed, s, z, bits, _lib.PROLOGUE_RMSNORM,
+                                      R=rd if with_r else None, R_out=r_out, w=dev(w), eps=1e-6,
+                                      config=CFG[ci])
+    close(host(Y), ref, "rmsnorm prologue")
+    assert np.allclose(host(r_out).astype(np.float64), h.astype(np.float64), rtol=1e-3, atol=1e-7)
+
+
+@pytest.mark.parametrize("M", [1, 4])
+@pytest.mark.parametrize("ci", [0, 1])
+def test_gemm_silu_prologue(M, ci):
+    I, N, bits = 1280, 80, 4
+    ref_q, (packed, s, z) = quantized(I, N, bits, seed=60 + M)
+    gu = f16(RNG.standard_normal((M, 2 * I)) * 3)
+    # gates at the ends of the range: silu -> -0 (e^-g overflows) and silu(g) = g
+    gu[:, :8] = f16([-65504.0, -100.0, -88.0, -87.0, 60.0, 11.0, 0.0, -0.0])
+    ref = dec.linear(dec.silu_mul(gu), ref_q)
+    Y = _lib.laq_gemm_wxg128_prologue(dev(gu), packed, s, z, bits, _lib.PROLOGUE_SILU_MUL,
+                                      config=CFG[ci])
+    close(host(Y), ref, "silu prologue")
+
+
+def test_gemm_prologue_rejects_aliasing():
+    _, (packed, s, z) = quantized(256, 32, 3, seed=1)
+    x = torch.zeros((1, 256), dtype=torch.float16, device=DEV)
+    r = torch.zeros((1, 256), dtype=torch.float16, device=DEV)
+    w = torch.ones(256, dtype=torch.float16, device=DEV)
+    with pytest.raises(laq.LaqError) as e:
+        _lib.laq_gemm_wxg128_prologue(x, packed, s, z, 3, _lib.PROLOGUE_RMSNORM, R=r, R_out=r, w=w)
+    assert e.value.status == 4
+
+
 # ---- one whole decode step (2 layers, real Qwen3-4B widths, small vocabulary) ----
 
-@pytest.mark.parametrize("bits,M,fused", [(3, 1, True), (4, 2, True), (3, 2, False)])
-def test_decode_step(bits, M, fused):
+@pytest.mark.parametrize("bits,M,fused,norms", [(3, 1, True, True), (4, 2, True, True),
+                                                (3, 2, False, False), (4, 1, True, False)])
+def test_decode_step(bits, M, fused, norms):
     from paper_2605_08755_gb300.decode_step import DecodeStep
     st = DecodeStep(bits=bits, M=M, layers=2, context=96, vocab=4096, seed=3,
-                    fused_attention=fused)
+                    fused_attention=fused, fused_norms=norms)
     kc0 = [host(c).copy() for c in st.kc]
     vc0 = [host(c).copy() for c in st.vc]
     tokens = host(st.tokens)
