@@ -21,7 +21,7 @@ import re
 from .weight_pass import pass_plan
 from . import inputs
 
-SOURCES = ["laq_gemm.cu", "laq_device.cuh"]
+SOURCES = ["laq_gemm_kernel.cuh", "laq_gemm.cu", "laq_device.cuh"]
 CSRC = os.path.join(os.path.dirname(os.path.abspath(__file__)), "csrc")
 
 
@@ -43,8 +43,12 @@ def read_launches(path):
         m = re.search(r"gemm_kernel<([^>]*)>", row["Kernel Name"])
         if not m:
             continue
-        args = re.findall(r"\d+", re.sub(r"\([a-z ]+\)", "", m.group(1)))  # drop (int) casts
-        d = launches.setdefault(lid, {"kernel": "gemm_kernel<" + ", ".join(args) + ">"})
+        # <BITS, MP, NT, PRO>: ncu writes the ints as (int)3 and the flag as false/true or
+        # (bool)0/1; the prologue instances get their own name
+        targs = [t.strip() for t in re.sub(r"\([a-z ]+\)", "", m.group(1)).split(",")]
+        pro = len(targs) > 3 and targs[3] in ("true", "1")
+        name = "gemm_kernel<" + ", ".join(targs[:3]) + ">" + (" prologue" if pro else "")
+        d = launches.setdefault(lid, {"kernel": name})
         val = float(row["Metric Value"].replace(",", ""))
         unit = row["Metric Unit"]
         scale = {"byte": 1, "Kbyte": 1e3, "Mbyte": 1e6, "Gbyte": 1e9, "ns": 1e-3, "nsecond": 1e-3,

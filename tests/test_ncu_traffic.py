@@ -13,10 +13,11 @@ HEADER = ('"ID","Process ID","Process Name","Host Name","Kernel Name","Context",
           '"Metric Value"\n')
 
 
-def fake_csv(path, kernels, nbytes):
+def fake_csv(path, kernels, nbytes, flag="false"):
     rows = ["==PROF== Connected to process 1\n", HEADER]
     for i, (k, b) in enumerate(zip(kernels, nbytes)):
-        name = f"void laq::(anonymous namespace)::gemm_kernel<(int){k[0]}, (int){k[1]}, (int){k[2]}>(laq::(anonymous namespace)::Params)"
+        name = (f"void laq::(anonymous namespace)::gemm_kernel<(int){k[0]}, (int){k[1]}, "
+                f"(int){k[2]}, {flag}>(laq::(anonymous namespace)::Params)")
         for metric, unit, val in (("dram__bytes_read.sum", "Mbyte", f"{b / 1e6:.3f}"),
                                   ("dram__bytes_write.sum", "byte", "1,000"),
                                   ("gpu__time_duration.sum", "ns", "5000")):
@@ -25,12 +26,13 @@ def fake_csv(path, kernels, nbytes):
     path.write_text("".join(rows))
 
 
-def test_groups_launches_by_instance_and_projection_shapes(tmp_path):
+@pytest.mark.parametrize("flag", ["false", "(bool)0"])
+def test_groups_launches_by_instance_and_projection_shapes(tmp_path, flag):
     plan = pass_plan("qwen3-4b", True, 2)  # q|k|v, o, gate|up, down per layer
     kernels = [(3, 1, 2), (3, 1, 1), (3, 1, 4), (3, 1, 2)] * 2
     nbytes = [6.3e6, 4.2e6, 19.9e6, 9.9e6] * 2
     csvp = tmp_path / "l.csv"
-    fake_csv(csvp, kernels, nbytes)
+    fake_csv(csvp, kernels, nbytes, flag)
     launches = ncu_traffic.read_launches(str(csvp))
     assert [k for k, _, _ in launches] == [f"gemm_kernel<{a}, {b}, {c}>" for a, b, c in kernels]
     assert launches[0][1] == pytest.approx(6.3e6 + 1000)
@@ -54,3 +56,10 @@ def test_rejects_a_log_that_is_not_one_pass(tmp_path):
     r = subprocess.run([sys.executable, "-m", "paper_2605_08755_gb300.ncu_traffic", str(csvp),
                         "--variant", "graph_fused", "--layers", "1"], capture_output=True, text=True)
     assert r.returncode != 0 and "3 launches" in (r.stderr + r.stdout)
+
+
+@pytest.mark.parametrize("flag", ["true", "(bool)1"])
+def test_prologue_instances_are_named_apart(tmp_path, flag):
+    csvp = tmp_path / "l.csv"
+    fake_csv(csvp, [(3, 1, 2)], [1e6], flag)
+    assert ncu_traffic.read_launches(str(csvp))[0][0] == "gemm_kernel<3, 1, 2> prologue"
