@@ -8,4 +8,8 @@ CUDA library.
   quantizer, dequantizer, bit packing, and Y = X * W_hat.
 * ``oracle.ref_numpy`` -- an independent numpy (float64) restatement of the same definitions,
   used to cross-check the C oracle bit for bit.
+* ``oracle.decoder`` -- the operations of one decode step around the projections (RMSNorm,
+  rotary embedding, grouped-query attention, SiLU * up, embedding, argmax) and the step itself.
+* ``oracle.rotation`` -- the online pairwise rotation (channel scales, then rounds of Givens
+  rotations per 128-channel group) that rotation-based methods run before each projection.
 """

@@ -18,13 +18,16 @@ where the CUDA path stores fp16:
 * ``silu_mul``       -- SiLU(gate) * up, SiLU(x) = x / (1 + e^-x);
 * ``embed`` / ``argmax`` -- row gather; the first index of the maximum;
 * ``decode_step``    -- one token of a Qwen3-style decoder built from the above and the
-                        quantized projections (Eq. (1), dequantized by the C oracle).
+                        quantized projections (Eq. (1), dequantized by the C oracle),
+                        optionally with the online pairwise rotation of ``oracle.rotation`` on
+                        the input of every projection of a layer.
 """
 import math
 
 import numpy as np
 
 from . import c_oracle
+from . import rotation
 
 
 def _f64(a):
@@ -135,7 +138,9 @@ def decode_step(model, tokens, pos, k_caches, v_caches):
     ``model``: dict with ``E`` [V, H] (embedding), ``layers`` (each a dict of quantized
     projections ``qkv``, ``o``, ``gate_up``, ``down`` as (codes, s, z) and fp16 norm weights
     ``in_w``, ``post_w``, ``q_w``, ``k_w``), ``final_w``, ``lm`` (quantized [H, V]) and the
-    scalars ``Hq``, ``Hkv``, ``D``, ``I``, ``theta``, ``eps``.  ``k_caches`` / ``v_caches``:
+    scalars ``Hq``, ``Hkv``, ``D``, ``I``, ``theta``, ``eps``.  A layer may carry ``rot``: per
+    projection name a table (alpha, pairs, angles) of ``oracle.rotation`` applied to that
+    projection's input (fp16 in, fp16 out) before it.  ``k_caches`` / ``v_caches``:
     per layer fp16 [M, Hkv, L, D]; the new token's k and v are written at pos[m] (copies are
     returned with them).  Returns (logits fp16 [M, V], next tokens, new caches)."""
     Hq, Hkv, D = model["Hq"], model["Hkv"], model["D"]
@@ -148,18 +153,26 @@ def decode_step(model, tokens, pos, k_caches, v_caches):
     h, _ = rmsnorm(x, model["layers"][0]["in_w"], eps)
     lens = [p + 1 for p in pos]
     for li, Lw in enumerate(model["layers"]):
+        rot = Lw.get("rot", {})
+
+        def proj(name, x):
+            if name in rot:
+                alpha, pairs, angles = rot[name]
+                x = rotation.pairwise_rotate(x, alpha, pairs, angles)
+            return linear(x, Lw[name])
+
         if li > 0:
             h, r = rmsnorm(d, Lw["in_w"], eps, r)
-        qkv = linear(h, Lw["qkv"])
+        qkv = proj("qkv", h)
         q, k, v = qk_norm_rope(qkv, Lw["q_w"], Lw["k_w"], pos, Hq, Hkv, theta, eps, D)
         for m, p in enumerate(pos):
             kcs[li][m, :, p] = k[m]
             vcs[li][m, :, p] = v[m]
         a = attention(q, kcs[li], vcs[li], lens, scale).reshape(len(tokens), Hq * D)
-        o = linear(a, Lw["o"])
+        o = proj("o", a)
         h, r = rmsnorm(o, Lw["post_w"], eps, r)
-        gu = linear(h, Lw["gate_up"])
-        d = linear(silu_mul(gu), Lw["down"])
+        gu = proj("gate_up", h)
+        d = proj("down", silu_mul(gu))
     h, _ = rmsnorm(d, model["final_w"], eps, r)
     logits = linear(h, model["lm"])
     return logits, argmax(logits), kcs, vcs

@@ -114,3 +114,19 @@ def kv_cache_torch(M, Hkv, L, D, seed, device):
     g = torch.Generator(device=device)
     g.manual_seed(seed + 1_111_111)
     return torch.randn((M, Hkv, L, D), generator=g, device=device).to(torch.float16)
+
+
+# ---- the online pairwise rotation of a projection's input (the rotation-based comparison) ----
+
+def rotation(K, rounds, seed):
+    """Tables of a pairwise rotation of K channels: per 128-channel group and round, a random
+    perfect matching of the group's channels into 64 pairs (uint8 [K/128][rounds][64][2]), one
+    angle per pair (float32 [K/128][rounds][64], uniform in [-pi, pi)), and channel scales
+    (fp16 [K], 1 + N(0, 0.1^2))."""
+    rng = np.random.default_rng(seed + 4_444_444)
+    G = K // 128
+    pairs = np.stack([rng.permutation(128).astype(np.uint8).reshape(64, 2)
+                      for _ in range(G * rounds)]).reshape(G, rounds, 64, 2)
+    theta = rng.uniform(-np.pi, np.pi, size=(G, rounds, 64)).astype(np.float32)
+    alpha = (1.0 + NORM_STD * rng.standard_normal(K, dtype=np.float32)).astype(np.float16)
+    return pairs, theta, alpha

@@ -8,6 +8,7 @@ import pytest
 
 from oracle import c_oracle
 from oracle import decoder as dec
+from paper_2605_08755_gb300 import inputs
 
 RNG = np.random.default_rng(1234)
 
@@ -186,3 +187,30 @@ def test_decode_step_with_zero_attention_and_mlp_outputs():
         assert np.array_equal(kcs[0][m][:, mask], kc[0][m][:, mask])
         assert np.array_equal(vcs[0][m, :, p], v_new[m])
         assert np.array_equal(kcs[0][m, :, p], k_new[m])
+
+
+def test_decode_step_with_identity_rotations_is_unchanged():
+    # zero angles and unit scales: the rotated step equals the plain one bit for bit; one real
+    # rotation on the o input changes the logits
+    H, Hq, Hkv, D, I, V, L = 256, 2, 1, 128, 256, 32, 8
+    E = f16(RNG.standard_normal((V, H)))
+    q = lambda K, N: c_oracle.quantize_rtn(f16(RNG.standard_normal((K, N)) * 0.05), 3)
+    layer = {"qkv": q(H, (Hq + 2 * Hkv) * D), "o": q(Hq * D, H), "gate_up": q(H, 2 * I),
+             "down": q(I, H), "in_w": f16(np.ones(H)), "post_w": f16(np.ones(H)),
+             "q_w": f16(np.ones(D)), "k_w": f16(np.ones(D))}
+    model = {"E": E, "layers": [layer], "final_w": f16(np.ones(H)), "lm": q(H, V), "Hq": Hq,
+             "Hkv": Hkv, "D": D, "I": I, "theta": 1e6, "eps": 1e-6}
+    kc = [f16(RNG.standard_normal((1, Hkv, L, D)))]
+    vc = [f16(RNG.standard_normal((1, Hkv, L, D)))]
+    plain = dec.decode_step(model, [3], [4], kc, vc)[0]
+    ident = {}
+    for name, K in (("qkv", H), ("o", Hq * D), ("gate_up", H), ("down", I)):
+        pairs = inputs.rotation(K, 2, seed=K)[0]
+        ident[name] = (f16(np.ones(K)), pairs, np.zeros((K // 128, 2, 64), np.float32))
+    rotated = dec.decode_step({**model, "layers": [{**layer, "rot": ident}]}, [3], [4], kc, vc)[0]
+    assert np.array_equal(rotated, plain)
+    real = dict(ident)
+    real["o"] = inputs.rotation(Hq * D, 2, seed=9)
+    real["o"] = (real["o"][2], real["o"][0], real["o"][1])
+    moved = dec.decode_step({**model, "layers": [{**layer, "rot": real}]}, [3], [4], kc, vc)[0]
+    assert not np.array_equal(moved, plain)
