@@ -367,6 +367,39 @@ laq_status laq_embed(const void *E, const int32_t *tokens, int64_t M, int64_t V,
  * wins; a row of NaN or -inf gives 0). */
 laq_status laq_argmax(const void *logits, int64_t M, int64_t V, int32_t *out, void *stream);
 
+/* ======================================================================================
+ * The online pairwise rotation of rotation-based quantizers (the comparison of Sec. 5.2):
+ * ParoQuant-style methods turn each projection's input by a transform that cannot be folded
+ * into the weights and so runs before every projection at every token (Sec. 1, Sec. 2).  LAQuant
+ * has no such step; these two calls exist to measure what it costs beside the GEMV.  The paper
+ * does not define the transform; the one computed here:
+ *
+ *   per group of 128 channels (the quantization groups), v = x * alpha (per channel), then for
+ *   r = 0 .. rounds-1 and each of round r's 64 pairs (i, j) with angle t, in any order (a round's
+ *   pairs are disjoint): (v_i, v_j) <- (v_i cos t - v_j sin t, v_i sin t + v_j cos t);
+ *   Y = fp16(v), rounded once (fp32 arithmetic).
+ * ====================================================================================== */
+
+/* cs[2k] = cos(theta[k]), cs[2k + 1] = sin(theta[k]) for k < n (fp32; theta 4-byte aligned, cs
+ * 8-byte aligned, device pointers).  Run once per set of angles: the angles are parameters. */
+laq_status laq_rotation_tables(const float *theta, int64_t n, void *cs, void *stream);
+
+/* Y [M][K] fp16 = the rotation of X [M][K] fp16.
+ *   alpha  fp16 [K] channel scales, or NULL for none;
+ *   pairs  uint8 [K/128][rounds][64][2]: pair p of round r of group g is
+ *          (pairs[g][r][p][0], pairs[g][r][p][1]), channels within the group; each round's 64
+ *          pairs must partition 0..127 (not checked: indices are masked to 0..127, so other
+ *          tables give wrong values but no access outside the group);
+ *   cs     float [K/128][rounds][64][2] (cos, sin) of each pair's angle (laq_rotation_tables);
+ *   rounds 0..16 (0: the scales alone; pairs and cs may then be NULL).
+ * Device pointers, all 16-byte aligned (alpha too, when given); Y may equal X (in place).
+ * M = 0: nothing.  Errors: LAQ_ERR_NULL, LAQ_ERR_SHAPE (M > 65535, K not a positive multiple of
+ * 128, rounds outside 0..16), LAQ_ERR_ALIGN, LAQ_ERR_CUDA.  Launched with programmatic dependent
+ * launch: the tables are read before the preceding kernel on the stream has finished. */
+laq_status laq_pairwise_rotate(const void *X, int64_t M, int64_t K, const void *alpha,
+                               const uint8_t *pairs, const void *cs, int32_t rounds, void *Y,
+                               void *stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -23,7 +23,8 @@ EXPORTS = ("laq_status_str", "laq_version", "laq_packed_bytes", "laq_quantize_rt
            "laq_gemm_wxg128_prologue",
            "laq_rmsnorm", "laq_qk_norm_rope", "laq_attention_workspace_bytes",
            "laq_attention_decode", "laq_attention_qkv_workspace_bytes", "laq_attention_qkv",
-           "laq_silu_mul", "laq_embed", "laq_argmax")
+           "laq_silu_mul", "laq_embed", "laq_argmax", "laq_rotation_tables",
+           "laq_pairwise_rotate")
 CHAIN_MAX = 384  # LAQ_CHAIN_MAX
 
 
@@ -104,12 +105,14 @@ def lib():
     L.laq_silu_mul.argtypes = [P, I64, I64, P, P]
     L.laq_embed.argtypes = [P, P, I64, I64, I64, P, P]
     L.laq_argmax.argtypes = [P, I64, I64, P, P]
+    L.laq_rotation_tables.argtypes = [P, I64, P, P]
+    L.laq_pairwise_rotate.argtypes = [P, I64, I64, P, P, P, I32, P, P]
     for name in ("laq_quantize_rtn", "laq_pack", "laq_unpack", "laq_gemm_wxg128",
                  "laq_gemm_plan", "laq_gemm_wxg128_config", "laq_gemm_chain",
                  "laq_gemm_chain_static", "laq_rmsnorm", "laq_qk_norm_rope",
                  "laq_gemm_wxg128_prologue",
-                 "laq_attention_decode", "laq_attention_qkv_workspace_bytes", "laq_attention_qkv",
-           "laq_silu_mul", "laq_embed", "laq_argmax"):
+                 "laq_attention_decode", "laq_attention_qkv", "laq_silu_mul", "laq_embed",
+                 "laq_argmax", "laq_rotation_tables", "laq_pairwise_rotate"):
         getattr(L, name).restype = I
     return L
 
@@ -366,3 +369,27 @@ def laq_argmax(logits, out=None, stream=None):
         out = torch.empty((M,), dtype=torch.int32, device=logits.device)
     _check(lib().laq_argmax(_ptr(logits), M, V, _ptr(out), _stream(stream)), "laq_argmax")
     return out
+
+
+# ---- the online pairwise rotation (the rotation-based comparison) ----
+
+def laq_rotation_tables(theta, stream=None):
+    """(cos, sin) of every angle: float32 [..., 2] for float32 angles theta [...]."""
+    import torch
+    cs = torch.empty(tuple(theta.shape) + (2,), dtype=torch.float32, device=theta.device)
+    _check(lib().laq_rotation_tables(_ptr(theta), theta.numel(), _ptr(cs), _stream(stream)),
+           "laq_rotation_tables")
+    return cs
+
+
+def laq_pairwise_rotate(X, pairs, cs, alpha=None, Y=None, stream=None):
+    """Y [M, K] = the rotation of X: channel scales alpha [K] (or none), then the rounds of
+    pairs uint8 [K/128, R, 64, 2] with (cos, sin) cs [K/128, R, 64, 2]."""
+    import torch
+    M, K = X.shape
+    rounds = pairs.shape[1]
+    if Y is None:
+        Y = torch.empty((M, K), dtype=torch.float16, device=X.device)
+    _check(lib().laq_pairwise_rotate(_ptr(X), M, K, _ptr(alpha), _ptr(pairs), _ptr(cs), rounds,
+                                     _ptr(Y), _stream(stream)), "laq_pairwise_rotate")
+    return Y

@@ -1,13 +1,17 @@
 """Time one whole decode step (DecodeStep) and, for context, the same step in fp16 torch ops.
 
     python -m paper_2605_08755_gb300.decode_case --bits 3 --M 1 --context 2048 [--fp16]
+        [--rotation-rounds R]
 
 Prints one JSON line: microseconds per step (CUDA events around graph replays on the capture
 stream), tokens per second (M per step), the step's algorithmic bytes and GB/s, the weight pass
 alone (the fused projections graph), and with --fp16 the same decoder step as a CUDA graph of
 plain torch fp16 operations on the unquantized weights (F.rms_norm, matmul, rotary by hand,
 scaled_dot_product_attention with grouped kv heads, SiLU, matmul with the embedding): a context
-ratio like the paper's decode speed-up over FP16 (Sec. 5.2), measured here on one GB300.
+ratio like the paper's decode speed-up over FP16 (Sec. 5.2), measured here on one GB300.  With
+--rotation-rounds R the line also times the rotation-based variant of the same step (an online
+pairwise rotation of R rounds before every projection of a layer, norms unfused) and reports
+how much faster the step is without it, the comparison of Sec. 5.2 (LAQuant against ParoQuant).
 """
 import argparse
 import json
@@ -105,6 +109,7 @@ def main():
     ap.add_argument("--fp16", action="store_true")
     ap.add_argument("--separate-attention", action="store_true")
     ap.add_argument("--separate-norms", action="store_true")
+    ap.add_argument("--rotation-rounds", type=int, default=0)
     a = ap.parse_args()
     torch.cuda.set_device(0)
     st = DecodeStep(model=a.model, bits=a.bits, M=a.M, layers=a.layers, context=a.context,
@@ -119,8 +124,18 @@ def main():
            "context": a.context, "launches": st.launches, "us_per_step": us,
            "tokens_per_s": a.M / (us * 1e-6), "bytes_per_step": st.bytes_per_step(),
            "gbs": st.bytes_per_step() / (us * 1e-6) / 1e9, "weight_pass_us": us_w}
+    del g
+    if a.rotation_rounds:
+        rs = DecodeStep(model=a.model, bits=a.bits, M=a.M, layers=a.layers, context=a.context,
+                        fused_attention=not a.separate_attention,
+                        rotation_rounds=a.rotation_rounds)
+        gr = rs.capture(stream=stream)
+        us_rot = time_graph(gr, stream, a.replays)
+        out.update({"rotation_rounds": a.rotation_rounds, "rotated_launches": rs.launches,
+                    "rotated_us_per_step": us_rot,
+                    "speedup_without_rotation": us_rot / us - 1.0})
+        del gr, rs
     if a.fp16:
-        del g
         ref = Fp16Step(st)
         gr = ref.capture(stream)
         us16 = time_graph(gr, stream, a.replays)

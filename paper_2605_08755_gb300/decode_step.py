@@ -10,7 +10,11 @@ per layer
     d = down GEMV(silu(gate) * up),  gate|up = gate|up GEMV(h);  r += d  (in the next norm)
 
 then the final rmsnorm, the LM head (the embedding, tied as in Qwen3-4B, quantized like the
-projections) and the greedy argmax.  Every step of it runs in the library's kernels
+projections) and the greedy argmax.  With ``rotation_rounds`` > 0 the step is that of a
+rotation-based quantizer instead: the input of every projection of a layer first goes through
+the online pairwise rotation (``laq_pairwise_rotate``: channel scales and that many rounds of
+Givens rotations per 128-channel group, synthetic tables), the per-token work LAQuant removes
+(Sec. 5.2 measures decoding with and without it).  Every step of it runs in the library's kernels
 (``laq_gemm_wxg128`` and the decoder operations of include/laq.h), launched in stream order
 with programmatic dependent launch and captured into one CUDA graph.  The KV cache holds
 ``context - 1`` synthetic tokens before the new one, so attention reads ``context`` tokens.
@@ -25,11 +29,14 @@ from .weight_pass import QuantLinear, WeightPass
 
 class DecodeStep:
     def __init__(self, model="qwen3-4b", bits=3, M=1, layers=inputs.LAYERS, context=2048,
-                 vocab=None, seed=0, device="cuda", fused_attention=True, fused_norms=True):
+                 vocab=None, seed=0, device="cuda", fused_attention=True, fused_norms=True,
+                 rotation_rounds=0):
         dims = inputs.DECODER[model]
         self.model, self.bits, self.M, self.layers = model, bits, M, layers
         self.fused_attention = fused_attention
-        self.fused_norms = fused_norms  # the layers' RMSNorms folded into the next GEMV
+        # the layers' RMSNorms folded into the next GEMV (not with a rotation between them)
+        self.fused_norms = fused_norms and not rotation_rounds
+        self.rotation_rounds = rotation_rounds
         self.context, self.seed = context, seed
         self.H, self.Hq, self.Hkv, self.D, self.I = (dims[k] for k in ("H", "Hq", "Hkv", "D", "I"))
         self.V = vocab or dims["V"]
@@ -83,9 +90,31 @@ class DecodeStep:
                    else _lib.attention_workspace(M, Hq, context, dev))
         self.scale = 1.0 / math.sqrt(D)
 
-    def gemv(self, X, q, Y, cfg, stream):
-        _lib.laq_gemm_wxg128(X.view(self.M, -1), q.packed, q.s, q.z, q.bits, Y=Y.view(self.M, -1),
-                             config=cfg, stream=stream)
+        # the rotation-based variant: per layer, tables for the inputs of q|k|v, o, gate|up, down
+        self.rot = []
+        if rotation_rounds:
+            for l in range(layers):
+                tabs = {}
+                for j, (name, K) in enumerate((("qkv", H), ("o", Hq * D), ("gate_up", H),
+                                               ("down", I))):
+                    pairs, theta, alpha = inputs.rotation(K, rotation_rounds,
+                                                          inputs.proj_seed(seed, l, 30 + j))
+                    th = torch.from_numpy(theta).to(dev)
+                    tabs[name] = dict(pairs=torch.from_numpy(pairs).to(dev), theta=th,
+                                      cs=_lib.laq_rotation_tables(th),
+                                      alpha=torch.from_numpy(alpha).to(dev))
+                self.rot.append(tabs)
+            self.xr = {K: torch.empty((M, K), **f16) for K in {H, Hq * D, I}}
+
+    def gemv(self, X, q, Y, cfg, stream, rot=None):
+        X = X.view(self.M, -1)
+        if rot is not None:  # the rotation-based variant: turn the input first
+            Xr = self.xr[X.shape[1]]
+            _lib.laq_pairwise_rotate(X, rot["pairs"], rot["cs"], alpha=rot["alpha"], Y=Xr,
+                                     stream=stream)
+            X = Xr
+        _lib.laq_gemm_wxg128(X, q.packed, q.s, q.z, q.bits, Y=Y.view(self.M, -1), config=cfg,
+                             stream=stream)
 
     def run(self, stream=None):
         """Launch one step on ``stream``: reads tokens, pos, the caches; writes the caches at pos,
@@ -98,10 +127,11 @@ class DecodeStep:
                       stream=stream)
         for l in range(self.layers):
             nw, (qkv, o, gu, dn), cf = self.norms[l], self.proj[l], self.cfg[l]
+            rt = self.rot[l] if self.rot else {}
             if l > 0:
                 L.laq_rmsnorm(self.d, nw["in_w"], self.eps, R=self.r, R_out=self.r, Y=self.h,
                               stream=stream)
-            self.gemv(self.h, qkv, self.qkv, cf[0], stream)
+            self.gemv(self.h, qkv, self.qkv, cf[0], stream, rt.get("qkv"))
             if self.fused_attention:  # norm, rotation, cache append and attention: two launches
                 L.laq_attention_qkv(self.qkv, nw["q_w"], nw["k_w"], self.pos, self.Hq, self.Hkv,
                                     self.theta, self.eps, self.kc[l], self.vc[l], self.scale,
@@ -112,12 +142,12 @@ class DecodeStep:
                                    stream=stream)
                 L.laq_attention_decode(self.q, self.kc[l], self.vc[l], self.lens, self.scale,
                                        self.ws, out=self.att, stream=stream)
-            self.gemv(self.att, o, self.o, cf[1], stream)
+            self.gemv(self.att, o, self.o, cf[1], stream, rt.get("o"))
             L.laq_rmsnorm(self.o, nw["post_w"], self.eps, R=self.r, R_out=self.r, Y=self.h,
                           stream=stream)
-            self.gemv(self.h, gu, self.gu, cf[2], stream)
+            self.gemv(self.h, gu, self.gu, cf[2], stream, rt.get("gate_up"))
             L.laq_silu_mul(self.gu, h=self.act, stream=stream)
-            self.gemv(self.act, dn, self.d, cf[3], stream)
+            self.gemv(self.act, dn, self.d, cf[3], stream, rt.get("down"))
         L.laq_rmsnorm(self.d, self.final_w, self.eps, R=self.r, Y=self.h, stream=stream)
         self.gemv(self.h, self.lm, self.logits, self.lm_cfg, stream)
         L.laq_argmax(self.logits, out=self.next, stream=stream)
@@ -164,7 +194,7 @@ class DecodeStep:
         # rope + 2) + silu, final norm, LM head, argmax
         if self.fused_norms:  # embed, per layer 4 GEMVs + 2 attention + silu, norm, LM head, argmax
             return 1 + self.layers * 7 + 3
-        per_layer = 9 if self.fused_attention else 10
+        per_layer = (9 if self.fused_attention else 10) + (4 if self.rotation_rounds else 0)
         return 2 + self.layers * per_layer - 1 + 3
 
     def capture(self, stream=None):
@@ -198,6 +228,10 @@ class DecodeStep:
                 ws.append(c_oracle.quantize_rtn(W, self.bits))
             nw = {k: v.cpu().numpy() for k, v in self.norms[l].items()}
             layers.append(dict(qkv=ws[0], o=ws[1], gate_up=ws[2], down=ws[3], **nw))
+            if self.rot:
+                layers[-1]["rot"] = {name: (t["alpha"].cpu().numpy(), t["pairs"].cpu().numpy(),
+                                            t["theta"].cpu().numpy())
+                                     for name, t in self.rot[l].items()}
         E = self.E.cpu().numpy()
         return {"E": E, "layers": layers, "final_w": self.final_w.cpu().numpy(),
                 "lm": c_oracle.quantize_rtn(E.T.copy(), self.bits), "Hq": self.Hq,

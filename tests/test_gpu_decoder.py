@@ -258,12 +258,14 @@ def test_gemm_prologue_rejects_aliasing():
 
 # ---- one whole decode step (2 layers, real Qwen3-4B widths, small vocabulary) ----
 
-@pytest.mark.parametrize("bits,M,fused,norms", [(3, 1, True, True), (4, 2, True, True),
-                                                (3, 2, False, False), (4, 1, True, False)])
-def test_decode_step(bits, M, fused, norms):
+@pytest.mark.parametrize("bits,M,fused,norms,rot", [
+    (3, 1, True, True, 0), (4, 2, True, True, 0), (3, 2, False, False, 0), (4, 1, True, False, 0),
+    # the rotation-based variant: a pairwise rotation before every projection of a layer
+    (3, 1, True, True, 4), (4, 2, False, False, 2)])
+def test_decode_step(bits, M, fused, norms, rot):
     from paper_2605_08755_gb300.decode_step import DecodeStep
     st = DecodeStep(bits=bits, M=M, layers=2, context=96, vocab=4096, seed=3,
-                    fused_attention=fused, fused_norms=norms)
+                    fused_attention=fused, fused_norms=norms, rotation_rounds=rot)
     kc0 = [host(c).copy() for c in st.kc]
     vc0 = [host(c).copy() for c in st.vc]
     tokens = host(st.tokens)
