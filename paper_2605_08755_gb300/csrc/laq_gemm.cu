@@ -26,16 +26,18 @@ size_t gemm_smem_bytes(const GemmLaunch& L, int* groups_per_phase) {
     const size_t ring = (size_t)L.warps * L.stages * rec;
     const int G = L.K / 128;
     const int gc = (G + L.cluster - 1) / L.cluster;
-    // raw X and (S, P) of one group
-    const size_t per_group = (size_t)L.M * (256 + 8);
+    // staged X (xs_row_chunks) and (S, P) of one group, and the zero block of the unpadded form
+    const int mp = mp_class(L.M);
+    const size_t per_group = (size_t)L.M * (xs_group_chunks(mp) * 16 + 8);
     int gpp = (int)(kXsBudget / per_group);
     if (gpp > gc) gpp = gc;
     if (gpp < 1) gpp = 1;
     if (groups_per_phase) *groups_per_phase = gpp;
-    const int mp = mp_class(L.M);
+    const size_t xs = (size_t)L.M * xs_row_chunks(gpp, mp) * 16 + (size_t)L.M * gpp * 8 +
+                      (xs_padded(mp) ? 0 : 64);
     const size_t sz = (size_t)(gc > 0 ? gc : 1) * L.tiles_per_cta * 48;  // s (32 B) + z (16 B)
     const size_t pro = L.pro != kProNone ? 64 : 0;  // inv_rms [16] fp32 of the prologue
-    return ring + (size_t)gpp * per_group + 64 + sz + (size_t)L.tiles_per_cta * mp * 16 * 4 + pro;
+    return ring + xs + sz + (size_t)L.tiles_per_cta * mp * 16 * 4 + pro;
 }
 
 cudaError_t launch_gemm(const GemmLaunch& L, size_t smem_limit, cudaStream_t stream) {

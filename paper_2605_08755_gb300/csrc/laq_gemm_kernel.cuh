@@ -243,18 +243,22 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 2) gemm_kernel(const Params p)
     const int g0 = (int)((long long)p.G * rank / C);
     const int g1 = (int)((long long)p.G * (rank + 1) / C);
 
-    // shared memory: ring [W][S][record] | x [M][GP][128] fp16 | zero block (64 B)
-    //                | s [gc][NT][16] fp16 | z [gc][NT][16] u8 | (S, P) [M][GP] float2
+    // shared memory: ring [W][S][record] | x [M][xs_row_chunks(GP, MP)] 16-byte chunks
+    //                | zero block (64 B, MP <= 2) | s [gc][NT][16] fp16 | z [gc][NT][16] u8
+    //                | (S, P) [M][GP] float2
     //                | part [NT][MP][16] fp32 | inv_rms [16] fp32
     uint8_t* ring = smem;
     uint4* xs = reinterpret_cast<uint4*>(smem + (size_t)W * S * F::kBytes);
-    uint4* zblk = xs + (size_t)M * GP * 16;
-    uint16_t* s_sm = reinterpret_cast<uint16_t*>(zblk + 4);
+    constexpr bool kPad = xs_padded(MP);
+    constexpr int GC = xs_group_chunks(MP);     // chunks per group of staged X
+    const int RS = xs_row_chunks(GP, MP);       // chunks per batch row of staged X
+    uint4* zblk = xs + (size_t)M * RS;          // zeros for B columns of other records
+    uint16_t* s_sm = reinterpret_cast<uint16_t*>(zblk + (kPad ? 0 : 4));
     uint8_t* z_sm = reinterpret_cast<uint8_t*>(s_sm + (size_t)p.gc * NT * 16);
     float2* ps = reinterpret_cast<float2*>(z_sm + (size_t)p.gc * NT * 16);
     float* part = reinterpret_cast<float*>(ps + (size_t)M * GP);
     float* inv_rms = part + NT * MP * 16;  // RMSNorm prologue: 1 / rms of each row (16)
-    if (threadIdx.x < 4) zblk[threadIdx.x] = make_uint4(0u, 0u, 0u, 0u);
+    if (!kPad && threadIdx.x < 4) zblk[threadIdx.x] = make_uint4(0u, 0u, 0u, 0u);
 
     const uint32_t ring_s = (uint32_t)__cvta_generic_to_shared(ring) +
                             (uint32_t)(warp * S * F::kBytes);
@@ -351,7 +355,7 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 2) gemm_kernel(const Params p)
                             v[r][0] = ld_cg16(src);
                             v[r][1] = ld_cg16(src + 64);
                         }
-                        xo[r] = b * GP * 16 + q;
+                        xo[r] = b * RS + (uu >> 3) * GC + (uu & 7);
                         po[r] = b * GP + (uu >> 3);
                     } else {
                         v[r][0] = v[r][1] = make_uint4(0u, 0u, 0u, 0u);
@@ -381,7 +385,7 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 2) gemm_kernel(const Params p)
                     }
                     if (xo[r] >= 0) {
                         xs[xo[r]] = v[r][0];
-                        xs[xo[r] + 8] = v[r][1];
+                        xs[xo[r] + (kPad ? 9 : 8)] = v[r][1];  // chunk h + 8 (past the pad)
                         if ((lane & 7) == 0) ps[po[r]] = make_float2(sx, px);  // unit h = 0
                     }
                 }
@@ -397,11 +401,13 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 2) gemm_kernel(const Params p)
         // Batch row and group column of this lane's B fragment (MMA column R).
         const int bl = MP <= 8 ? R / GPA : R;
         const int gil = MP <= 8 ? R % GPA : 0;
-        // X of the lane's B column for the warp's record i: uint4 offset xo0[h] + i * xstep.
-        const int xstep = WT * 16;
+        // X of the lane's B column for the warp's record i: uint4 offset xo0[h] + i * xstep
+        // (chunks 4c .. 4c+3 of the group; rows past M are never read, and clamped anyway).
+        const int xstep = WT * GC;
         int xo0[NH];
 #pragma unroll
-        for (int h = 0; h < NH; ++h) xo0[h] = ((bl + 8 * h) * GP + team) * 16 + c * 4;
+        for (int h = 0; h < NH; ++h)
+            xo0[h] = min(bl + 8 * h, M - 1) * RS + team * GC + c * 4 + (kPad ? c >> 1 : 0);
 
         int rslot = 0;
         float D[2][NH][4];  // two independent accumulator chains (even / odd k16 steps)
@@ -419,14 +425,24 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 2) gemm_kernel(const Params p)
             uint32_t B[NH][8][2];
 #pragma unroll
             for (int h = 0; h < NH; ++h) {
-                const uint4* src = gil == gi && bl + 8 * h < M ? xm[h] : zblk;
+                uint4 v[4];
+                if (!kPad) {  // every lane loads: X of its record, or the zero block
+                    const uint4* src = gil == gi && bl + 8 * h < M ? xm[h] : zblk;
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) v[q] = src[q];
+                } else if (gil == gi && bl + 8 * h < M) {  // others take zeros, reading nothing
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) v[q] = xm[h][q];
+                } else {
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) v[q] = make_uint4(0u, 0u, 0u, 0u);
+                }
 #pragma unroll
                 for (int q = 0; q < 4; ++q) {
-                    const uint4 v = src[q];
-                    B[h][2 * q][0] = v.x;
-                    B[h][2 * q][1] = v.y;
-                    B[h][2 * q + 1][0] = v.z;
-                    B[h][2 * q + 1][1] = v.w;
+                    B[h][2 * q][0] = v[q].x;
+                    B[h][2 * q][1] = v[q].y;
+                    B[h][2 * q + 1][0] = v[q].z;
+                    B[h][2 * q + 1][1] = v[q].w;
                 }
             }
             LAQ_TRACE_LOOP(2, i);

@@ -30,6 +30,17 @@ struct GemmLaunch {
 };
 constexpr int kProNone = 0, kProRmsNorm = 1, kProSiluMul = 2;
 
+// Staged X in the GEMM's shared memory, in 16-byte chunks (chunk j holds x[8j .. 8j+7]).  For
+// M <= 2 (MP <= 2) chunk j of group lg of batch row b sits at b * 16 gpp + 16 lg + j; at most 4
+// lanes of a load phase read X then.  For MP >= 4, where 8 lanes of a phase read 4 chunk columns
+// of 2 batch rows, the chunk sits at b * xs_row_chunks + 17 lg + j + j / 8: the pad between a
+// group's halves and a row stride of 2 mod 8 chunks put those 8 lanes on 8 different bank slots.
+__host__ __device__ constexpr bool xs_padded(int mp) { return mp >= 4; }
+__host__ __device__ constexpr int xs_group_chunks(int mp) { return xs_padded(mp) ? 17 : 16; }
+__host__ __device__ constexpr int xs_row_chunks(int gpp, int mp) {
+    return xs_padded(mp) ? gpp * 17 + (((2 - gpp * 17) % 8) + 8) % 8 : gpp * 16;
+}
+
 // Dynamic shared memory the GEMM kernel needs for this launch (bytes), and the groups of X it
 // stages per phase.
 size_t gemm_smem_bytes(const GemmLaunch& L, int* groups_per_phase);

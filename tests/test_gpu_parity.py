@@ -133,14 +133,18 @@ SMEM_OPTIN = 232448   # bytes of dynamic shared memory a CTA may opt into on sm_
 
 def smem_needed(M, K, bits, cfg):
     """Mirror of the library's shared-memory budget: per-warp cp.async rings, staged X with its
-    group sums (up to 64 KB per phase), zero block, scales and zeros, per-CTA partial sums."""
+    group sums (about 64 KB per phase; padded rows from M = 3), the zero block (M <= 2), scales
+    and zeros, per-CTA partial sums."""
     rec = 1024 if bits == 4 else 768
     gc = -(-(K // 128) // cfg.cluster)
-    per_group = M * 264
-    gpp = max(1, min(gc, 64 * 1024 // per_group))
     mp = 1 if M <= 1 else 2 if M <= 2 else 4 if M <= 4 else 8 if M <= 8 else 16
-    return (cfg.warps * cfg.stages * rec + gpp * per_group + 64 + gc * cfg.tiles_per_cta * 48
-            + cfg.tiles_per_cta * mp * 64)
+    padded = mp >= 4
+    per_group = M * ((17 if padded else 16) * 16 + 8)
+    gpp = max(1, min(gc, 64 * 1024 // per_group))
+    # X rows in 16-byte chunks (padded: 17 per group, row stride 2 mod 8), zero block if not
+    row_chunks = gpp * 17 + (2 - gpp * 17) % 8 if padded else gpp * 16
+    return (cfg.warps * cfg.stages * rec + M * row_chunks * 16 + M * gpp * 8
+            + (0 if padded else 64) + gc * cfg.tiles_per_cta * 48 + cfg.tiles_per_cta * mp * 64)
 
 
 @pytest.mark.parametrize("bits", [3, 4])
