@@ -133,8 +133,8 @@ laq_status laq_gemm_wxg128(const void *X, int64_t M, int64_t K, int64_t N, const
 /*
  * Launch configuration of laq_gemm_wxg128 (a tuning interface; the library picks one itself).
  *   tiles_per_cta  16-column tiles per CTA: 1, 2, 4 or 8.
- *   warps          warps per CTA, 1..8, a multiple of tiles_per_cta; each tile gets
- *                  warps / tiles_per_cta warps, which split the CTA's K range.
+ *   warps          warps per CTA, 1..16 (1..8 for M <= 2), a multiple of tiles_per_cta;
+ *                  each tile gets warps / tiles_per_cta warps, which split the CTA's K range.
  *   cluster        CTAs per thread-block cluster, 1, 2, 4 or 8; the CTAs of a cluster split
  *                  K and reduce their partial sums through distributed shared memory.
  *   stages         depth of each warp's cp.async ring of weight records, 2..16; with

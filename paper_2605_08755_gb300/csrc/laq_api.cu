@@ -87,7 +87,7 @@ laq_status check_config(const laq_gemm_config* c) {
     if (c->tiles_per_cta != 1 && c->tiles_per_cta != 2 && c->tiles_per_cta != 4 &&
         c->tiles_per_cta != 8)
         return LAQ_ERR_CONFIG;
-    if (c->warps < 1 || c->warps > 8) return LAQ_ERR_CONFIG;
+    if (c->warps < 1 || c->warps > 16) return LAQ_ERR_CONFIG;
     if (c->warps % c->tiles_per_cta) return LAQ_ERR_CONFIG;  // whole warps per tile
     if (c->cluster != 1 && c->cluster != 2 && c->cluster != 4 && c->cluster != 8)
         return LAQ_ERR_CONFIG;
@@ -112,6 +112,8 @@ int ceil_div(int64_t a, int64_t b) { return (int)((a + b - 1) / b); }
 //    doubles until a warp holds at most 5 records and the grid covers every SM (down: 640
 //    CTAs, 5 records per warp; measured on GB300 in the Qwen3-4B pass, W3 and W4: 1.6 us less
 //    per down launch).  Shorter K (o, q, k, v) measured best with the rule above.
+//  * M > 4: 16 warps per CTA where the plan above leaves one 8-warp CTA per SM (wide outputs;
+//    the long-K down projection at M > 8, with half the cluster).
 //  * Eight warps otherwise (fewer when a CTA owns fewer groups), and a cp.async ring deep
 //    enough to hold all of a warp's records (at most 16) within 100 KB.
 void plan(int64_t M, int64_t K, int64_t N, int bits, int sms, laq_gemm_config* out) {
@@ -126,6 +128,17 @@ void plan(int64_t M, int64_t K, int64_t N, int bits, int sms, laq_gemm_config* o
         while (cl < 8 && cl * 2 <= G && (int64_t)ceil_div(T, nt) * cl < sms) cl *= 2;
         best_nt = nt;
         best_cl = cl;
+        // M > 4: one 8-warp CTA per SM leaves each scheduler two warps, too few to hide the
+        // MMA and shared-memory latency of the wider batch.  16-warp CTAs (two warps per tile)
+        // where the output alone fills the SMs, and for the long K of the down projection at
+        // M > 8 with half the cluster (measured on GB300, Qwen3-4B W3 pass: gate|up -140 us at
+        // M = 8 and -196 us at M = 16, down -266 us at M = 16; q|k|v, o and M <= 4 within 2%).
+        if (M > 8 && G >= 64 && best_cl >= 2) {
+            warps_max = 16;
+            best_cl /= 2;
+        } else if (M > 4 && best_cl == 1 && (int64_t)ceil_div(T, best_nt) >= sms) {
+            warps_max = 16;
+        }
     } else {
         double best_cost = 1e300;
         int64_t best_ctas = INT64_MAX;
@@ -194,6 +207,7 @@ laq_status run_gemm(const void* X, int64_t M, int64_t K, int64_t N, const void* 
     if (cfg) {
         st = check_config(cfg);
         if (st != LAQ_OK) return st;
+        if (cfg->warps > 8 && M < 3) return LAQ_ERR_CONFIG;  // 16-warp CTAs from M = 3
     }
     if (M == 0 || N == 0) return LAQ_OK;
     cudaStream_t strm = static_cast<cudaStream_t>(stream);

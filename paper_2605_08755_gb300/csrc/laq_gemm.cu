@@ -36,7 +36,7 @@ size_t gemm_smem_bytes(const GemmLaunch& L, int* groups_per_phase) {
     const size_t xs = (size_t)L.M * xs_row_chunks(gpp, mp) * 16 + (size_t)L.M * gpp * 8 +
                       (xs_padded(mp) ? 0 : 64);
     const size_t sz = (size_t)(gc > 0 ? gc : 1) * L.tiles_per_cta * 48;  // s (32 B) + z (16 B)
-    const size_t pro = L.pro != kProNone ? 64 : 0;  // inv_rms [16] fp32 of the prologue
+    const size_t pro = L.pro != kProNone ? 128 : 0;  // inv_rms [16] + warp sums [16], fp32
     return ring + xs + sz + (size_t)L.tiles_per_cta * mp * 16 * 4 + pro;
 }
 

@@ -67,7 +67,10 @@ namespace laq {
 
 namespace {
 
-constexpr int kMaxWarps = 8;
+// Warps per CTA: up to 8 for M <= 2 (two CTAs per SM), up to 16 from M = 3, where a CTA
+// shares staged X over 4 or 8 tiles and two warps per tile hide the MMA and shared-memory
+// latency that one CTA per SM leaves exposed.
+__host__ __device__ constexpr int max_warps(int mp) { return mp >= 4 ? 16 : 8; }
 
 struct Params {
     const uint16_t* X;
@@ -183,11 +186,11 @@ __device__ void rms_rows(const Params& p, float* inv_rms) {
         }
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
-        if (lane == 0) inv_rms[8 + warp] = ss;  // (W <= 8)
+        if (lane == 0) inv_rms[16 + warp] = ss;  // (W <= 16)
         __syncthreads();
         if (threadIdx.x == 0) {
             float tot = 0.f;
-            for (int k = 0; k < W; ++k) tot += inv_rms[8 + k];
+            for (int k = 0; k < W; ++k) tot += inv_rms[16 + k];
             inv_rms[0] = rsqrtf(tot / (float)p.K + p.eps);
         }
         __syncthreads();
@@ -215,7 +218,8 @@ __device__ void rms_rows(const Params& p, float* inv_rms) {
 }
 
 template <int BITS, int MP, int NT, bool PRO>
-__global__ void __launch_bounds__(kMaxWarps * 32, 2) gemm_kernel(const Params p) {
+__global__ void __launch_bounds__(max_warps(MP) * 32, 16 / max_warps(MP))
+gemm_kernel(const Params p) {
     using F = RecordFmt<BITS>;
     constexpr int WPL = BITS == 4 ? 8 : 6;
     constexpr int GPA = MP >= 8 ? 1 : 8 / MP;  // groups sharing one accumulator (columns)
@@ -257,7 +261,7 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 2) gemm_kernel(const Params p)
     uint8_t* z_sm = reinterpret_cast<uint8_t*>(s_sm + (size_t)p.gc * NT * 16);
     float2* ps = reinterpret_cast<float2*>(z_sm + (size_t)p.gc * NT * 16);
     float* part = reinterpret_cast<float*>(ps + (size_t)M * GP);
-    float* inv_rms = part + NT * MP * 16;  // RMSNorm prologue: 1 / rms of each row (16)
+    float* inv_rms = part + NT * MP * 16;  // RMSNorm prologue: 1 / rms per row, warp sums
     if (!kPad && threadIdx.x < 4) zblk[threadIdx.x] = make_uint4(0u, 0u, 0u, 0u);
 
     const uint32_t ring_s = (uint32_t)__cvta_generic_to_shared(ring) +

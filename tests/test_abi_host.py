@@ -95,7 +95,8 @@ def test_gemm_config_validation(L):
     assert run(tiles_per_cta=3) == 9
     assert run(tiles_per_cta=16) == 9
     assert run(warps=0) == 9
-    assert run(warps=9) == 9
+    assert run(warps=17) == 9
+    assert run(warps=16) == 9  # more than 8 warps only from M = 3 (this call has M = 1)
     assert run(cluster=3) == 9
     assert run(cluster=16) == 9
     assert run(stages=1) == 9
@@ -134,7 +135,7 @@ def test_plan_is_valid_for_every_workload_shape(L, bits, M):
         for sms in (152, 148, 1):
             c = laq.laq_gemm_plan(M, K, N, bits, sms)
             assert c.tiles_per_cta in (1, 2, 4, 8)
-            assert 1 <= c.warps <= 8
+            assert 1 <= c.warps <= 16 and c.warps % c.tiles_per_cta == 0
             assert c.cluster in (1, 2, 4, 8) and c.cluster <= max(1, K // 128)
             assert 2 <= c.stages <= 16
             assert c.pdl == 0
@@ -210,10 +211,22 @@ def test_plan_shares_x_across_tiles_at_m_above_one(L):
     # M > 1: 4 (M <= 4) or 8 tiles per CTA, and a cluster K split towards one CTA per SM
     c = laq.laq_gemm_plan(4, 9728, 2560, 3, 152)
     assert (c.tiles_per_cta, c.cluster) == (4, 4)
+    c = laq.laq_gemm_plan(4, 2560, 19456, 3, 152)
+    assert (c.tiles_per_cta, c.warps, c.cluster) == (4, 8, 1)
+    c = laq.laq_gemm_plan(8, 9728, 2560, 3, 152)
+    assert (c.tiles_per_cta, c.warps, c.cluster) == (8, 8, 8)
+    # M > 4 where that leaves one 8-warp CTA per SM: 16-warp CTAs (two warps per tile); the
+    # long-K down projection at M > 8 with half the cluster
+    c = laq.laq_gemm_plan(8, 2560, 19456, 3, 152)
+    assert (c.tiles_per_cta, c.warps, c.cluster) == (8, 16, 1)
     c = laq.laq_gemm_plan(16, 2560, 19456, 3, 152)
-    assert (c.tiles_per_cta, c.cluster) == (8, 1)
+    assert (c.tiles_per_cta, c.warps, c.cluster) == (8, 16, 1)
     c = laq.laq_gemm_plan(16, 9728, 2560, 3, 152)
-    assert (c.tiles_per_cta, c.cluster) == (8, 8)
+    assert (c.tiles_per_cta, c.warps, c.cluster) == (8, 16, 4)
+    # 16 warps only from M = 3 (the M <= 2 kernels are built for at most 8)
+    for M in (1, 2):
+        for K, N in ((2560, 19456), (9728, 2560), (4096, 24576)):
+            assert laq.laq_gemm_plan(M, K, N, 3, 152).warps <= 8
     # M = 1: the fused Qwen3-4B projections
     assert laq.laq_gemm_plan(1, 2560, 19456, 3, 152).tiles_per_cta == 4
     assert laq.laq_gemm_plan(1, 2560, 6144, 3, 152).tiles_per_cta == 2
