@@ -111,7 +111,7 @@ def test_qwen3_4b_pass_batch_sweep(bits, M):
     _sampled(wp, layers={5, 30})
 
 
-@pytest.mark.parametrize("bits,M", [(3, 1), (4, 1), (3, 16)])
+@pytest.mark.parametrize("bits,M", [(3, 1), (4, 1), (3, 8), (3, 16)])
 def test_qwen3_4b_fused_pass(bits, M):
     """q|k|v and gate|up as single GEMVs over concatenated columns (4 launches per layer)."""
     wp = WeightPass(model="qwen3-4b", bits=bits, M=M, fuse=True)
