@@ -381,7 +381,8 @@ laq_status laq_argmax(const void *logits, int64_t M, int64_t V, int32_t *out, vo
  * ====================================================================================== */
 
 /* cs[2k] = cos(theta[k]), cs[2k + 1] = sin(theta[k]) for k < n (fp32; theta 4-byte aligned, cs
- * 8-byte aligned, device pointers).  Run once per set of angles: the angles are parameters. */
+ * 8-byte aligned, device pointers; 0 <= n <= 2^31, LAQ_ERR_SHAPE otherwise).  Run once per set of
+ * angles: the angles are parameters. */
 laq_status laq_rotation_tables(const float *theta, int64_t n, void *cs, void *stream);
 
 /* Y [M][K] fp16 = the rotation of X [M][K] fp16.

@@ -115,7 +115,7 @@ extern "C" {
 laq_status laq_rotation_tables(const float* theta, int64_t n, void* cs, void* stream) {
     if (n == 0) return LAQ_OK;
     if (!theta || !cs) return LAQ_ERR_NULL;
-    if (n < 0 || n > ((int64_t)1 << 40)) return LAQ_ERR_SHAPE;
+    if (n < 0 || n > ((int64_t)1 << 31)) return LAQ_ERR_SHAPE;  // grid.x limit x 256 threads
     if (((uintptr_t)theta & 3u) || ((uintptr_t)cs & 7u)) return LAQ_ERR_ALIGN;
     rotation_tables_kernel<<<(unsigned)((n + 255) / 256), 256, 0,
                              static_cast<cudaStream_t>(stream)>>>(theta, n,

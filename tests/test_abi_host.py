@@ -246,3 +246,49 @@ def test_plan_splits_k_of_narrow_outputs_at_m_one(L, bits):
     # shorter K (o, q, k, v of Qwen3-4B) and wide outputs keep 8-warp CTAs
     for K, N in ((4096, 2560), (2560, 4096), (2560, 1024), (2560, 19456), (2560, 6144)):
         assert laq.laq_gemm_plan(1, K, N, bits, 152).warps >= 5, (K, N)
+
+
+def test_gemm_prologue_argument_validation(L):
+    def run(kind=1, eps=1e-6, R=None, R_out=None, w=FAKE, X=FAKE):
+        pro = _lib.GemmPrologue(kind, eps, R, R_out, w)
+        return L.laq_gemm_wxg128_prologue(X, 1, 256, 32, FAKE, FAKE, FAKE, 3, FAKE,
+                                          ctypes.byref(pro), None, None)
+    assert run(kind=3) == 9             # unknown kind: LAQ_ERR_CONFIG
+    assert run(kind=-1) == 9
+    assert run(w=None) == 1             # RMSNorm without weights
+    assert run(eps=-1.0) == 4
+    assert run(eps=float("nan")) == 4
+    assert run(R=FAKE, R_out=FAKE) == 4          # R_out may not alias R ...
+    assert run(R_out=FAKE) == 4                  # ... nor X (both FAKE here)
+    assert run(w=ODD) == 5
+    assert run(R=ODD) == 5
+    assert run(R_out=ctypes.c_void_p(0x20008)) == 5
+    assert run(kind=2, X=ODD) == 5
+
+
+def test_rotation_argument_validation(L):
+    def rot(X=FAKE, M=1, K=256, alpha=None, pairs=FAKE, cs=FAKE, rounds=4, Y=FAKE):
+        return L.laq_pairwise_rotate(X, M, K, alpha, pairs, cs, rounds, Y, None)
+    assert rot(M=0) == 0                # nothing to do, no launch
+    assert rot(X=None) == 1
+    assert rot(Y=None) == 1
+    assert rot(pairs=None) == 1
+    assert rot(cs=None) == 1
+    assert rot(K=200) == 4
+    assert rot(K=0) == 4
+    assert rot(M=65536) == 4
+    assert rot(M=-1) == 4
+    assert rot(rounds=17) == 4
+    assert rot(rounds=-1) == 4
+    assert rot(X=ODD) == 5
+    assert rot(Y=ctypes.c_void_p(0x10008)) == 5
+    assert rot(alpha=ODD) == 5
+    assert rot(pairs=ctypes.c_void_p(0x10008)) == 5
+    tables = L.laq_rotation_tables
+    assert tables(None, 0, None, None) == 0
+    assert tables(None, 5, FAKE, None) == 1
+    assert tables(FAKE, 5, None, None) == 1
+    assert tables(FAKE, -1, FAKE, None) == 4
+    assert tables(FAKE, (1 << 31) + 1, FAKE, None) == 4
+    assert tables(ctypes.c_void_p(0x10002), 5, FAKE, None) == 5
+    assert tables(FAKE, 5, ctypes.c_void_p(0x10004), None) == 5
