@@ -1,6 +1,6 @@
 """Per-instance DRAM traffic of a decode-step pass from an ncu launch list.
 
-    python -m paper_2605_08755_gb300.ncu_traffic gpurun_out/traffic_graph_fused.csv \\
+    python -m paper_2605_08755_gb300.ncu_traffic launches_graph_fused.csv \\
         --variant graph_fused [--model qwen3-4b --bits 3 --M 1] [--write profiles/traffic.json]
 
 The CSV is ncu's ``--csv`` log of ``--metrics dram__bytes_read.sum,dram__bytes_write.sum,
