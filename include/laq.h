@@ -244,6 +244,69 @@ laq_status laq_gemm_chain(const laq_gemv *gemvs, int32_t count, void *workspace,
 laq_status laq_gemm_chain_static(const laq_gemv *gemvs, int32_t count, void *stream);
 
 /*
+ * ======================================================================================
+ * The planned pass: the chain of laq_gemm_chain (same laq_gemv entries and stage rules), with
+ * the walk over its weights done once on the host.  A plan deals each stage's 16-column tiles
+ * to the SMs as whole tiles (balanced by records of 16 columns x 128 rows), cuts every SM's
+ * records into 16 warp shares, and orders them into one contiguous stream per SM, each record's
+ * 16 scales and 16 zeros beside its packed codes.  laq_pass_prepare writes those streams into a
+ * caller-owned device buffer once; laq_pass_run then streams them with bulk copies into a ring
+ * of shared memory that runs ahead across the stage boundaries (the weights never depend on the
+ * activations), while the stages wait for their inputs.  It serves the decode-step weight pass
+ * (Sec. 5.2, "Inference": a decode step streams every projection's weights once), and each
+ * entry's Y is that of laq_gemm_wxg128 (fp32 sums of Eq. (1) products, one fp16 rounding; the
+ * summation orders differ).  M = 1 only.
+ *
+ * Usage: laq_pass_plan_sizes -> allocate the host plan (plan_bytes) and the device buffer
+ * (device_bytes, 256-byte aligned) -> laq_pass_plan_build -> laq_pass_prepare -> a zeroed
+ * workspace of laq_pass_workspace_bytes -> laq_pass_run, any number of times.
+ * ====================================================================================== */
+
+/* Host bytes of the plan and device bytes of the streams and tables for `count` entries
+ * (HOST array, read during the call) on a device with `num_sms` SMs.  Host work only (no CUDA
+ * call).  Entries as laq_gemm_chain's, with M = 1, one `bits` for all, K <= 24576 (an entry's X
+ * must fit the kernel's staging area), N % 16 == 0, K, N > 0.  The device buffer holds every
+ * packed record once more (K * N * bits / 8 + 3 * N * K / 128 bytes per entry) plus tables.
+ * Errors: LAQ_ERR_NULL, LAQ_ERR_BITS (invalid or mixed bits), LAQ_ERR_M_RANGE (M != 1),
+ * LAQ_ERR_SHAPE (count outside 0..LAQ_CHAIN_MAX, num_sms outside 1..1024, a bad K or N, or an
+ * SM's share of one stage above 255 warp segments), LAQ_ERR_ALIGN (a pointer not 16-byte
+ * aligned). */
+laq_status laq_pass_plan_sizes(const laq_gemv *gemvs, int32_t count, int32_t num_sms,
+                               size_t *plan_bytes, size_t *device_bytes);
+
+/* Write the plan into the HOST buffer `plan` (plan_bytes from laq_pass_plan_sizes; smaller:
+ * LAQ_ERR_WORKSPACE).  Host work only.  The plan records the entries' X and Y addresses, which
+ * every laq_pass_run uses; packed, s and z are read only by laq_pass_prepare. */
+laq_status laq_pass_plan_build(const laq_gemv *gemvs, int32_t count, int32_t num_sms,
+                               void *plan, size_t plan_bytes);
+
+/* Workspace bytes laq_pass_run needs for this plan (status word, a finished-CTA count and one
+ * counter per stage; 0 if `plan` is not a plan). */
+size_t laq_pass_workspace_bytes(const void *plan);
+
+/* Lay the plan's weights out in the DEVICE buffer `device` (256-byte aligned, device_bytes from
+ * laq_pass_plan_sizes): copies the plan's tables (a host-to-device copy from pageable memory,
+ * which waits for the stream's earlier work; not for stream capture) and enqueues the gather
+ * kernel on `stream`.  The entries' packed codes, scales and zeros must stay valid until that
+ * kernel has run; afterwards the pass reads only `device`.  Errors: LAQ_ERR_CONFIG (not a
+ * plan), LAQ_ERR_NULL, LAQ_ERR_ALIGN, LAQ_ERR_WORKSPACE (device buffer too small),
+ * LAQ_ERR_CUDA. */
+laq_status laq_pass_prepare(const void *plan, void *device, size_t device_bytes, void *stream);
+
+/* Run the planned pass on `stream`: one cooperative launch of one CTA per SM.  `plan` is the
+ * HOST plan, `device` the prepared buffer, `workspace` a DEVICE buffer of at least
+ * laq_pass_workspace_bytes(plan) bytes, 16-byte aligned, zero before its first use (a completed
+ * call leaves it zero again); word 0 (uint32) is the device-side status: 0, or LAQ_ERR_TIMEOUT
+ * if a wait gave up after about a second (Y undefined; zero the workspace before the next
+ * call).  Calls sharing one workspace must not overlap in time.  The device must have the SM
+ * count the plan was built for (LAQ_ERR_CONFIG otherwise).  Errors: LAQ_ERR_CONFIG (not a plan,
+ * another SM count, the launch does not fit), LAQ_ERR_NULL, LAQ_ERR_ALIGN (device buffer),
+ * LAQ_ERR_WORKSPACE, LAQ_ERR_SHAPE (the staging area and a ring of two slots exceed shared
+ * memory), LAQ_ERR_CUDA. */
+laq_status laq_pass_run(const void *plan, const void *device, void *workspace,
+                        size_t workspace_bytes, void *stream);
+
+/*
  * A prologue applied to X while laq_gemm_wxg128_prologue stages it, so that the operation
  * before a projection costs no launch of its own.  The paper has no counterpart: this fuses two
  * of the decoder operations declared below (laq_rmsnorm, laq_silu_mul) into the GEMV.

@@ -24,7 +24,8 @@ EXPORTS = ("laq_status_str", "laq_version", "laq_packed_bytes", "laq_quantize_rt
            "laq_rmsnorm", "laq_qk_norm_rope", "laq_attention_workspace_bytes",
            "laq_attention_decode", "laq_attention_qkv_workspace_bytes", "laq_attention_qkv",
            "laq_silu_mul", "laq_embed", "laq_argmax", "laq_rotation_tables",
-           "laq_pairwise_rotate")
+           "laq_pairwise_rotate", "laq_pass_plan_sizes", "laq_pass_plan_build",
+           "laq_pass_workspace_bytes", "laq_pass_prepare", "laq_pass_run")
 CHAIN_MAX = 384  # LAQ_CHAIN_MAX
 
 
@@ -107,12 +108,21 @@ def lib():
     L.laq_argmax.argtypes = [P, I64, I64, P, P]
     L.laq_rotation_tables.argtypes = [P, I64, P, P]
     L.laq_pairwise_rotate.argtypes = [P, I64, I64, P, P, P, I32, P, P]
+    L.laq_pass_plan_sizes.argtypes = [ctypes.POINTER(Gemv), I32, I32, ctypes.POINTER(SZ),
+                                      ctypes.POINTER(SZ)]
+    L.laq_pass_plan_build.argtypes = [ctypes.POINTER(Gemv), I32, I32, P, SZ]
+    L.laq_pass_workspace_bytes.argtypes = [P]
+    L.laq_pass_workspace_bytes.restype = SZ
+    L.laq_pass_prepare.argtypes = [P, P, SZ, P]
+    L.laq_pass_run.argtypes = [P, P, P, SZ, P]
     for name in ("laq_quantize_rtn", "laq_pack", "laq_unpack", "laq_gemm_wxg128",
                  "laq_gemm_plan", "laq_gemm_wxg128_config", "laq_gemm_chain",
                  "laq_gemm_chain_static", "laq_rmsnorm", "laq_qk_norm_rope",
                  "laq_gemm_wxg128_prologue",
                  "laq_attention_decode", "laq_attention_qkv", "laq_silu_mul", "laq_embed",
-                 "laq_argmax", "laq_rotation_tables", "laq_pairwise_rotate"):
+                 "laq_argmax", "laq_rotation_tables", "laq_pairwise_rotate",
+                 "laq_pass_plan_sizes", "laq_pass_plan_build", "laq_pass_prepare",
+                 "laq_pass_run"):
         getattr(L, name).restype = I
     return L
 
@@ -259,6 +269,45 @@ def chain_status(workspace):
     import torch
     torch.cuda.synchronize(workspace.device)
     return int(workspace[:4].view(torch.int32)[0].item())
+
+
+def pass_plan(gemvs, count, num_sms):
+    """Host work only: the laq_pass plan of ``count`` laq_gemv entries (a ctypes Gemv array) for
+    ``num_sms`` SMs, as a ctypes byte buffer, and the device bytes it needs."""
+    pb, db = ctypes.c_size_t(0), ctypes.c_size_t(0)
+    _check(lib().laq_pass_plan_sizes(gemvs, count, num_sms, ctypes.byref(pb), ctypes.byref(db)),
+           "laq_pass_plan_sizes")
+    plan = (ctypes.c_uint8 * pb.value)()
+    _check(lib().laq_pass_plan_build(gemvs, count, num_sms, plan, pb.value),
+           "laq_pass_plan_build")
+    return plan, db.value
+
+
+class PassPlan:
+    """The entries of a ``Chain`` planned for laq_pass_run on ``device``: the host plan, the
+    prepared device buffer (per-SM weight streams and tables) and a zeroed workspace.  The
+    entries' X and Y tensors are kept alive; their packed weights are no longer read once
+    ``prepare`` has run on the stream."""
+
+    def __init__(self, entries, device, stream=None):
+        import torch
+        self.chain = Chain(entries)
+        self.device = torch.device(device)
+        sms = torch.cuda.get_device_properties(self.device).multi_processor_count
+        self.plan, dev_bytes = pass_plan(self.chain.array, self.chain.count, sms)
+        self.buffer = torch.empty((max(dev_bytes, 256),), dtype=torch.uint8, device=self.device)
+        self.ws = torch.zeros((max(256, int(lib().laq_pass_workspace_bytes(self.plan))),),
+                              dtype=torch.uint8, device=self.device)
+        _check(lib().laq_pass_prepare(self.plan, _ptr(self.buffer), self.buffer.numel(),
+                                      _stream(stream)), "laq_pass_prepare")
+
+    def run(self, stream=None):
+        _check(lib().laq_pass_run(self.plan, _ptr(self.buffer), _ptr(self.ws), self.ws.numel(),
+                                  _stream(stream)), "laq_pass_run")
+
+    def status(self):
+        """The device-side status word (synchronizes the device)."""
+        return chain_status(self.ws)
 
 
 # ---- decoder operations around the projections (one decode step) ----

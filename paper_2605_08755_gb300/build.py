@@ -16,7 +16,7 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD_DIR = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "liblaq.so")
 SOURCES = ("laq_api.cu", "laq_quant.cu", "laq_gemm.cu", "laq_gemm_prologue.cu", "laq_chain.cu",
-           "laq_decode.cu", "laq_rotate.cu")
+           "laq_decode.cu", "laq_rotate.cu", "laq_pass.cu")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

@@ -1,0 +1,1007 @@
+// laq_pass.cu -- the decode-step weight pass (Sec. 5.2, "Inference": every projection's
+// weights streamed once per token) as a planned persistent launch over per-SM weight streams.
+//
+// laq_gemm_chain runs the same chain of WbG128 GEMVs (Eq. (1) weights) in one launch, but each
+// of its warps walks the packed weights, scales and zeros of its shares itself (a cursor over
+// entries, tiles and groups, and three source arrays per record).  Here that walk happens once,
+// on the host, when the chain is planned:
+//
+//  * Plan (host only).  The chain is cut into stages at the entries that wait for their
+//    predecessors.  Each stage's 16-column tiles are dealt to the SMs in order as whole tiles,
+//    balanced by records (tile x group of 128 rows), so no output tile is split between SMs and
+//    no cross-SM reduction sits on the critical path.  An SM's records of a stage are cut into
+//    16 contiguous warp shares that differ by at most one record.  The SM's records, all
+//    stages in order, form its stream, laid out in rounds: round r holds the r-th record of
+//    every warp that has one, warp w's at position w.
+//
+//  * Prepare (once).  A gather kernel writes every SM's stream into one device buffer: each
+//    record's packed codes followed by its 16 scales and 16 zeros, so an SM's whole pass is
+//    one contiguous byte range.
+//
+//  * Run.  One cooperative CTA per SM: 16 consumer warps and one producer warp.  The producer
+//    copies the SM's stream round by round with cp.async.bulk into a ring of shared-memory
+//    slots (one mbarrier pair per slot), with no knowledge of stages: weights never depend on
+//    activations, so the ring runs ahead across stage boundaries while the consumers wait for
+//    a stage's input.  Per stage the consumers wait for every SM to have finished the previous
+//    stage (a release/acquire counter per stage in the workspace), stage the stage's X in
+//    shared memory with the group sums S_g = sum_k x_k and P_g = sum_k c_k x_k, take their
+//    records from the ring (one per round and warp), and reduce their partial tiles in warp
+//    order (deterministic, no atomics on Y).
+//
+//  * The record arithmetic is that of laq_gemm_wxg128 at M = 1: one mask-and-or per pair of
+//    codes gives fp16 values c + q, the m16n8k16 MMA contracts them with raw x, the eight groups
+//    of a block share one accumulator (one MMA column each), and the block epilogue applies
+//    Eq. (1) as y += s * (D - P - z S).
+//
+//  * Every wait is bounded (about a second): a timed-out wait records LAQ_ERR_TIMEOUT in the
+//    workspace, the CTA's warps leave together (barrier reductions decide it), the producer
+//    first waits for its copies in flight, and the call's results are undefined.
+#include <cuda_fp16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <atomic>
+#include <climits>
+#include <cstring>
+#include <vector>
+
+#include "laq.h"
+#include "laq_device.cuh"
+
+namespace laq {
+namespace {
+
+constexpr uint32_t kPassMagic = 0x5051414cu;  // "LAQP"
+constexpr int32_t kPassVersion = 1;
+constexpr int kPW = 16;                        // consumer warps
+constexpr int kPThreads = (kPW + 1) * 32;      // and the producer warp
+constexpr int kPRec = 16;                      // records per round (one per consumer warp)
+constexpr int kSZ = 48;                        // a record's 16 fp16 scales and 16 uint8 zeros
+constexpr int kMaxSegs = 255;                  // warp segments per (SM, stage)
+constexpr int kMaxXsBytes = 48 * 1024;         // staged X per (SM, stage)
+constexpr int kMaxRing = 16;                   // ring slots
+constexpr int kMaxSms = 1024;
+constexpr unsigned long long kWaitNs = 1000000000ull;  // wait limit (1 s)
+constexpr int kWaitSpins = 1 << 24;                    // and an iteration limit besides
+
+// ---- plan tables: the same bytes in the host plan and in the device buffer -------------------
+
+struct SmDesc {        // one per SM
+    int64_t rec0;      // the SM's first record in the stream buffer (records, all of rb bytes)
+    int32_t round0;    // its first entry of the round table
+    int32_t nrounds;
+};
+struct StageDesc {     // one per (SM, stage), SM-major
+    int32_t n;         // records of the SM in the stage
+    int32_t nr;        // rounds: ceil(n / 16)
+    int32_t seg0;      // first segment (index into the segment table)
+    int32_t tile0;     // first local tile
+    int32_t x0;        // first staged X
+    int16_t nseg, nt, nx, pad;
+    uint8_t wseg[kPW + 1];  // warp w's segments: [seg0 + wseg[w], seg0 + wseg[w + 1])
+    uint8_t pad2[3];
+};
+struct Seg {           // groups [g0, g0 + ng) of tile t of entry e, as one warp runs them
+    int32_t e, t;
+    int16_t g0, ng;
+    int16_t xg;        // the entry's first group in the stage's X area
+    int16_t lt;        // local tile (index into the stage's local tiles)
+};
+struct LTile {         // a tile of the SM's stage share: its 16 outputs, its segments' slots
+    uint16_t* y;       // Y + 16 t of its entry
+    int32_t slot0, nslot;
+};
+struct XItem {         // one entry's X staged for the SM's stage share
+    const uint16_t* x;
+    int32_t K;
+    int32_t xg;        // first group in the X area (a group is 256 bytes of X)
+};
+struct PrepEntry {     // what the gather kernel reads of an entry
+    const uint8_t* packed;
+    const uint16_t* s;
+    const uint8_t* z;
+    int32_t N, G;
+};
+struct GatherRec {     // stream record i is record rid = t * G + g of entry e
+    int32_t e, rid;
+};
+static_assert(sizeof(SmDesc) == 16 && sizeof(StageDesc) == 48 && sizeof(Seg) == 16 &&
+                  sizeof(LTile) == 16 && sizeof(XItem) == 16 && sizeof(PrepEntry) == 32 &&
+                  sizeof(GatherRec) == 8,
+              "plan table layout");
+
+struct PlanHeader {
+    uint32_t magic;
+    int32_t version;
+    int32_t count, nstages, sms, bits;
+    int32_t rb;        // stream bytes of a record (packed codes + scales + zeros)
+    int32_t xs_bytes;  // largest staged X of an (SM, stage)
+    int32_t max_segs;  // most segments of an (SM, stage)
+    int32_t max_nx;    // most staged X items of an (SM, stage)
+    int64_t records, rounds, segs, ltiles, xitems;
+    int64_t tables_h;      // offset of the table region in the plan buffer
+    int64_t tables_bytes;  // its size (the same region follows the streams on the device)
+    int64_t stream_bytes;  // bytes of the streams at the start of the device buffer
+    // offsets of the tables within the table region
+    int64_t o_sm, o_rounds, o_stage, o_seg, o_tile, o_x, o_prep, o_gather;
+    int64_t plan_bytes, device_bytes;
+};
+static_assert(sizeof(PlanHeader) <= 256, "plan header");
+
+constexpr int64_t align_up(int64_t v, int64_t a) { return (v + a - 1) / a * a; }
+
+int record_bytes(int bits) { return (bits == 4 ? 1024 : 768) + kSZ; }
+
+// ---- host planner ------------------------------------------------------------------------------
+
+struct HostPlan {
+    int count = 0, nstages = 0, sms = 0, bits = 3;
+    int xs_bytes = 0, max_segs = 0, max_nx = 0;
+    std::vector<SmDesc> sm;
+    std::vector<uint8_t> rounds;
+    std::vector<StageDesc> stage;
+    std::vector<Seg> seg;
+    std::vector<LTile> tile;
+    std::vector<XItem> xi;
+    std::vector<PrepEntry> prep;
+    std::vector<GatherRec> gather;
+};
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+laq_status plan_pass(const laq_gemv* g, int32_t count, int32_t P, HostPlan& H) {
+    if (count < 0 || count > LAQ_CHAIN_MAX) return LAQ_ERR_SHAPE;
+    if (P < 1 || P > kMaxSms) return LAQ_ERR_SHAPE;
+    if (count > 0 && !g) return LAQ_ERR_NULL;
+    H = HostPlan();
+    H.count = count;
+    H.sms = P;
+    std::vector<int> start;  // first entry of each stage
+    for (int i = 0; i < count; ++i) {
+        const laq_gemv& e = g[i];
+        if (e.bits != 3 && e.bits != 4) return LAQ_ERR_BITS;
+        if (i == 0) H.bits = e.bits;
+        if (e.bits != H.bits) return LAQ_ERR_BITS;
+        if (e.M != 1) return LAQ_ERR_M_RANGE;
+        if (e.K <= 0 || e.N <= 0 || e.K % 128 != 0 || e.N % 16 != 0) return LAQ_ERR_SHAPE;
+        if (e.K * 2 > kMaxXsBytes || e.N / 16 > ((int64_t)1 << 24)) return LAQ_ERR_SHAPE;
+        if (!e.X || !e.packed || !e.s || !e.z || !e.Y) return LAQ_ERR_NULL;
+        if (!aligned16(e.X) || !aligned16(e.packed) || !aligned16(e.s) || !aligned16(e.z) ||
+            !aligned16(e.Y))
+            return LAQ_ERR_ALIGN;
+        if (i == 0 || e.wait_prev != 0) start.push_back(i);
+        H.prep.push_back(PrepEntry{static_cast<const uint8_t*>(e.packed),
+                                   static_cast<const uint16_t*>(e.s), e.z, (int32_t)e.N,
+                                   (int32_t)(e.K / 128)});
+    }
+    const int S = (int)start.size();
+    H.nstages = S;
+    start.push_back(count);
+
+    // Whole tiles to SMs, in order: a tile goes to the SM whose equal share of the stage's
+    // records holds the tile's middle record, so SM shares are contiguous tile ranges and
+    // differ from the mean by less than one tile.  first[s][j] = SM j's first stage tile.
+    std::vector<std::vector<int64_t>> first(S);
+    for (int s = 0; s < S; ++s) {
+        int64_t tiles = 0, W = 0;
+        for (int e = start[s]; e < start[s + 1]; ++e) {
+            tiles += g[e].N / 16;
+            W += (g[e].N / 16) * (g[e].K / 128);
+        }
+        std::vector<int64_t>& f = first[s];
+        f.assign((size_t)P + 1, tiles);
+        int64_t c = 0, tix = 0;
+        int jp = -1;
+        for (int e = start[s]; e < start[s + 1]; ++e) {
+            const int64_t T = g[e].N / 16, G = g[e].K / 128;
+            for (int64_t t = 0; t < T; ++t, ++tix, c += G) {
+                int64_t j = (2 * c + G) * P / (2 * W);
+                if (j > P - 1) j = P - 1;
+                while (jp < j) f[(size_t)(++jp)] = tix;
+            }
+        }
+        while (jp < P) f[(size_t)(++jp)] = tiles;
+    }
+
+    struct TileRef {
+        int e;
+        int64_t t;
+        int G;
+    };
+    for (int j = 0; j < P; ++j) {
+        SmDesc sd;
+        sd.rec0 = (int64_t)H.gather.size();
+        sd.round0 = (int32_t)H.rounds.size();
+        for (int s = 0; s < S; ++s) {
+            // the SM's tiles of the stage
+            std::vector<TileRef> tl;
+            {
+                int64_t ta = first[s][(size_t)j], tb = first[s][(size_t)j + 1], base = 0;
+                for (int e = start[s]; e < start[s + 1] && ta < tb; ++e) {
+                    const int64_t T = g[e].N / 16;
+                    for (; ta < tb && ta < base + T; ++ta)
+                        tl.push_back(TileRef{e, ta - base, (int)(g[e].K / 128)});
+                    base += T;
+                }
+            }
+            StageDesc d;
+            std::memset(&d, 0, sizeof(d));
+            d.seg0 = (int32_t)H.seg.size();
+            d.tile0 = (int32_t)H.tile.size();
+            d.x0 = (int32_t)H.xi.size();
+            int64_t n = 0;
+            for (const TileRef& r : tl) n += r.G;
+            if (n > INT_MAX / 2) return LAQ_ERR_SHAPE;
+            d.n = (int32_t)n;
+            d.nr = (int32_t)((n + kPRec - 1) / kPRec);
+            if (n == 0) {
+                H.stage.push_back(d);
+                continue;
+            }
+            if ((int64_t)tl.size() > kMaxSegs) return LAQ_ERR_SHAPE;
+            // X of every entry the share touches, one after another, whole groups
+            std::vector<int> xg_of(tl.size());
+            int xg = 0, last_e = -1;
+            for (size_t k = 0; k < tl.size(); ++k) {
+                if (tl[k].e != last_e) {
+                    last_e = tl[k].e;
+                    H.xi.push_back(XItem{static_cast<const uint16_t*>(g[last_e].X),
+                                         (int32_t)g[last_e].K, (int32_t)xg});
+                    xg += (int)(g[last_e].K / 128);
+                    ++d.nx;
+                }
+                xg_of[k] = H.xi.back().xg;
+            }
+            if (xg * 256 > kMaxXsBytes) return LAQ_ERR_SHAPE;
+            if (xg * 256 > H.xs_bytes) H.xs_bytes = xg * 256;
+            if (d.nx > H.max_nx) H.max_nx = d.nx;
+            // record offset of each local tile
+            std::vector<int64_t> toff(tl.size() + 1, 0);
+            for (size_t k = 0; k < tl.size(); ++k) toff[k + 1] = toff[k] + tl[k].G;
+            // warp shares and their segments
+            const int64_t q = n / kPW, rem = n % kPW;
+            size_t lt = 0;
+            int nseg = 0;
+            for (int w = 0; w < kPW; ++w) {
+                int64_t a = w * q + (w < rem ? w : rem);
+                const int64_t b = a + q + (w < rem ? 1 : 0);
+                if (nseg > kMaxSegs) return LAQ_ERR_SHAPE;
+                d.wseg[w] = (uint8_t)nseg;
+                while (a < b) {
+                    while (toff[lt + 1] <= a) ++lt;
+                    const int64_t end = b < toff[lt + 1] ? b : toff[lt + 1];
+                    H.seg.push_back(Seg{tl[lt].e, (int32_t)tl[lt].t, (int16_t)(a - toff[lt]),
+                                        (int16_t)(end - a), (int16_t)xg_of[lt], (int16_t)lt});
+                    ++nseg;
+                    a = end;
+                }
+            }
+            if (nseg > kMaxSegs) return LAQ_ERR_SHAPE;
+            d.wseg[kPW] = (uint8_t)nseg;
+            d.nseg = (int16_t)nseg;
+            d.nt = (int16_t)tl.size();
+            if (nseg > H.max_segs) H.max_segs = nseg;
+            // local tiles: the consecutive segments that cover each
+            for (size_t k = 0; k < tl.size(); ++k) {
+                LTile t;
+                t.y = static_cast<uint16_t*>(g[tl[k].e].Y) + tl[k].t * 16;
+                t.slot0 = -1;
+                t.nslot = 0;
+                H.tile.push_back(t);
+            }
+            for (int k = 0; k < nseg; ++k) {
+                LTile& t = H.tile[(size_t)d.tile0 + (size_t)H.seg[(size_t)d.seg0 + k].lt];
+                if (t.slot0 < 0) t.slot0 = k;
+                ++t.nslot;
+            }
+            // rounds, and the stream records in round order
+            int cur_k[kPW], cur_i[kPW];
+            for (int w = 0; w < kPW; ++w) {
+                cur_k[w] = d.wseg[w];
+                cur_i[w] = 0;
+            }
+            for (int64_t r = 0; r < d.nr; ++r) {
+                const int cnt = r < q ? kPRec : (int)rem;
+                H.rounds.push_back((uint8_t)cnt);
+                for (int w = 0; w < cnt; ++w) {
+                    const Seg& sg = H.seg[(size_t)d.seg0 + cur_k[w]];
+                    const int64_t G = g[sg.e].K / 128;
+                    H.gather.push_back(GatherRec{sg.e, (int32_t)(sg.t * G + sg.g0 + cur_i[w])});
+                    if (++cur_i[w] == sg.ng) {
+                        ++cur_k[w];
+                        cur_i[w] = 0;
+                    }
+                }
+            }
+            H.stage.push_back(d);
+        }
+        const int64_t nr = (int64_t)H.rounds.size() - sd.round0;
+        if ((int64_t)H.rounds.size() > INT_MAX / 2) return LAQ_ERR_SHAPE;
+        sd.nrounds = (int32_t)nr;
+        H.sm.push_back(sd);
+    }
+    return LAQ_OK;
+}
+
+// Layout of the serialized plan and of the device buffer.
+void layout(const HostPlan& H, PlanHeader& h) {
+    std::memset(&h, 0, sizeof(h));
+    h.magic = kPassMagic;
+    h.version = kPassVersion;
+    h.count = H.count;
+    h.nstages = H.nstages;
+    h.sms = H.sms;
+    h.bits = H.bits;
+    h.rb = record_bytes(H.bits);
+    h.xs_bytes = H.xs_bytes;
+    h.max_segs = H.max_segs;
+    h.max_nx = H.max_nx;
+    h.records = (int64_t)H.gather.size();
+    h.rounds = (int64_t)H.rounds.size();
+    h.segs = (int64_t)H.seg.size();
+    h.ltiles = (int64_t)H.tile.size();
+    h.xitems = (int64_t)H.xi.size();
+    int64_t o = 0;
+    h.o_sm = o;      o = align_up(o + (int64_t)H.sm.size() * (int64_t)sizeof(SmDesc), 256);
+    h.o_rounds = o;  o = align_up(o + (int64_t)H.rounds.size(), 256);
+    h.o_stage = o;   o = align_up(o + (int64_t)H.stage.size() * (int64_t)sizeof(StageDesc), 256);
+    h.o_seg = o;     o = align_up(o + (int64_t)H.seg.size() * (int64_t)sizeof(Seg), 256);
+    h.o_tile = o;    o = align_up(o + (int64_t)H.tile.size() * (int64_t)sizeof(LTile), 256);
+    h.o_x = o;       o = align_up(o + (int64_t)H.xi.size() * (int64_t)sizeof(XItem), 256);
+    h.o_prep = o;    o = align_up(o + (int64_t)H.prep.size() * (int64_t)sizeof(PrepEntry), 256);
+    h.o_gather = o;  o = align_up(o + (int64_t)H.gather.size() * (int64_t)sizeof(GatherRec), 256);
+    h.tables_bytes = o;
+    h.tables_h = align_up(256 + (int64_t)H.count * (int64_t)sizeof(laq_gemv), 256);
+    h.plan_bytes = h.tables_h + h.tables_bytes;
+    h.stream_bytes = align_up(h.records * h.rb, 256);
+    h.device_bytes = h.stream_bytes + h.tables_bytes;
+}
+
+template <class T>
+void put(uint8_t* region, int64_t off, const std::vector<T>& v) {
+    if (!v.empty()) std::memcpy(region + off, v.data(), v.size() * sizeof(T));
+}
+
+// A plan buffer from laq_pass_plan_build, or nullptr.
+const PlanHeader* as_plan(const void* plan) {
+    if (!plan) return nullptr;
+    const PlanHeader* h = static_cast<const PlanHeader*>(plan);
+    if (h->magic != kPassMagic || h->version != kPassVersion) return nullptr;
+    if (h->sms < 1 || h->sms > kMaxSms || h->nstages < 0 || h->nstages > LAQ_CHAIN_MAX ||
+        (h->bits != 3 && h->bits != 4) || h->rb != record_bytes(h->bits) ||
+        h->xs_bytes < 0 || h->xs_bytes > kMaxXsBytes || h->max_segs < 0 ||
+        h->max_segs > kMaxSegs || h->max_nx < 0 || h->max_nx > kMaxSegs)
+        return nullptr;
+    return h;
+}
+
+size_t pass_workspace(const PlanHeader& h) {
+    return (size_t)align_up(4 * (2 + (int64_t)h.nstages), 256);
+}
+
+// ---- shared memory layout of the pass kernel (host and device) -------------------------------
+
+struct PassSmem {
+    int xs, sp, seg, tile, xi, slot, zero, bar, flag, total;
+};
+__host__ __device__ inline PassSmem pass_smem(int rb, int ns, int xs_bytes, int max_segs,
+                                              int max_nx) {
+    PassSmem m;
+    m.xs = (ns * kPRec * rb + 127) / 128 * 128;
+    m.sp = m.xs + xs_bytes;
+    m.seg = (m.sp + xs_bytes / 256 * 8 + 15) / 16 * 16;
+    m.tile = m.seg + max_segs * (int)sizeof(Seg);
+    m.xi = m.tile + max_segs * (int)sizeof(LTile);
+    m.slot = m.xi + max_nx * (int)sizeof(XItem);
+    m.zero = m.slot + max_segs * 16 * 4;
+    m.bar = m.zero + 64;
+    m.flag = m.bar + 2 * kMaxRing * 8;
+    m.total = m.flag + 16;
+    return m;
+}
+
+// ---- device helpers ----------------------------------------------------------------------------
+
+__device__ __forceinline__ unsigned long long gtimer() {
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+__device__ __forceinline__ uint32_t ld_acq(const uint32_t* p) {
+    uint32_t v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+__device__ __forceinline__ uint32_t ld_rlx(const uint32_t* p) {
+    uint32_t v;
+    asm volatile("ld.relaxed.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+__device__ __forceinline__ void red_rel_add(uint32_t* p, uint32_t v) {
+    asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+__device__ __forceinline__ uint32_t atom_acq_rel_add(uint32_t* p, uint32_t v) {
+    uint32_t old;
+    asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], %2;"
+                 : "=r"(old)
+                 : "l"(p), "r"(v)
+                 : "memory");
+    return old;
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar),
+                 "r"(bytes)
+                 : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ bool mbar_try(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n"
+        ".reg .pred p;\n"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+        "selp.u32 %0, 1, 0, p;\n"
+        "}\n"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0u;
+}
+// Copy `bytes` (a multiple of 16) from global memory into this CTA's shared memory; the copy
+// counts its bytes against the transaction count of mbarrier `bar`.
+__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t bytes,
+                                         uint32_t bar) {
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+        ::"r"(dst), "l"(src), "r"(bytes), "r"(bar)
+        : "memory");
+}
+
+// Named barrier of the 16 consumer warps, returning whether any of them passed `v` true (the
+// same answer in every thread, so decisions taken on it keep the warps together).
+__device__ __forceinline__ bool cbar_any(bool v) {
+    uint32_t r;
+    asm volatile(
+        "{\n"
+        ".reg .pred p, q;\n"
+        "setp.ne.u32 q, %1, 0;\n"
+        "bar.red.or.pred p, 1, 512, q;\n"
+        "selp.u32 %0, 1, 0, p;\n"
+        "}\n"
+        : "=r"(r)
+        : "r"((uint32_t)v)
+        : "memory");
+    return r != 0u;
+}
+__device__ __forceinline__ void cbar() { asm volatile("bar.sync 1, 512;" ::: "memory"); }
+
+// Record a device-side timeout in the workspace status word (the first error stays).
+__device__ __forceinline__ void record_timeout(uint32_t* status) {
+    atomicCAS(status, 0u, (uint32_t)LAQ_ERR_TIMEOUT);
+}
+
+// Wait for phase `parity` of mbarrier `bar`.  False when the CTA is aborting (the flag is read
+// every 64 polls) or after about a second (then the flag and the status word are set).
+__device__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag,
+                          uint32_t* status) {
+    if (mbar_try(bar, parity)) return true;
+    const unsigned long long t0 = gtimer();
+    for (int spin = 0; spin < kWaitSpins; ++spin) {
+        if (mbar_try(bar, parity)) return true;
+        if ((spin & 63) == 63) {
+            if (abort_flag && *abort_flag) return false;
+            if (gtimer() - t0 > kWaitNs) break;
+        }
+    }
+    if (abort_flag) {
+        *abort_flag = 1;
+        record_timeout(status);
+    }
+    return false;
+}
+
+// Wait until *cnt >= target (acquire).  False when the status word already holds an error or
+// after about a second (then LAQ_ERR_TIMEOUT is recorded).
+__device__ bool wait_ge(const uint32_t* cnt, uint32_t target, uint32_t* status) {
+    if (ld_rlx(status) != 0u) return false;
+    if (ld_acq(cnt) >= target) return true;
+    const unsigned long long t0 = gtimer();
+    for (int spin = 0; spin < kWaitSpins; ++spin) {
+        if (ld_acq(cnt) >= target) return true;
+        if ((spin & 31) == 31) {
+            if (ld_rlx(status) != 0u) return false;
+            if (gtimer() - t0 > kWaitNs) break;
+        }
+    }
+    record_timeout(status);
+    return false;
+}
+
+struct PassParams {
+    const uint8_t* stream;
+    const SmDesc* sm;
+    const uint8_t* rounds;
+    const StageDesc* stage;
+    const Seg* seg;
+    const LTile* tile;
+    const XItem* xi;
+    uint32_t* ws;  // [0] status, [1] finished CTAs, [2 + s] CTAs done with stage s
+    int nstages, ns, xs_bytes, max_segs, max_nx;
+    Exps exps;
+};
+
+// ---- the producer warp -------------------------------------------------------------------------
+
+template <int BITS>
+__device__ void pass_producer(const PassParams& p, const SmDesc& sd, uint32_t ring_s,
+                              uint32_t full_s, uint32_t empty_s, volatile int* abort_flag,
+                              int lane) {
+    constexpr int RB = RecordFmt<BITS>::kBytes + kSZ;
+    constexpr uint32_t SLOT = (uint32_t)(kPRec * RB);
+    const int NS = p.ns, NR = sd.nrounds;
+    const uint8_t* src = p.stream + sd.rec0 * RB;
+    const uint8_t* rt = p.rounds + sd.round0;
+    int issued = 0;
+    bool ok = true;
+    for (int r0 = 0; r0 < NR && ok; r0 += 32) {
+        const int mine = r0 + lane < NR ? (int)rt[r0 + lane] : 0;
+        const int lim = NR - r0 < 32 ? NR - r0 : 32;
+        for (int i = 0; i < lim; ++i) {
+            const int cnt = __shfl_sync(0xffffffffu, mine, i);
+            const int r = r0 + i, slot = r % NS, k = r / NS;
+            // slot reuse: every consumer warp has released the round that used it last
+            if (k > 0 && !__all_sync(0xffffffffu,
+                                     mbar_wait(empty_s + 8u * slot, (uint32_t)((k - 1) & 1),
+                                               abort_flag, p.ws))) {
+                ok = false;
+                break;
+            }
+            if (lane == 0) {
+                const uint32_t bytes = (uint32_t)(cnt * RB);
+                mbar_expect_tx(full_s + 8u * slot, bytes);
+                bulk_g2s(ring_s + SLOT * (uint32_t)slot, src, bytes, full_s + 8u * slot);
+            }
+            __syncwarp();
+            src += (size_t)cnt * RB;
+            issued = r + 1;
+        }
+    }
+    // No copy may still be landing in shared memory when the CTA exits: wait for the last
+    // round issued into each slot (immediate when the consumers took every round).
+    for (int r = issued > NS ? issued - NS : 0; r < issued; ++r)
+        mbar_wait(full_s + 8u * (r % NS), (uint32_t)((r / NS) & 1), nullptr, p.ws);
+}
+
+// ---- the consumer warps ------------------------------------------------------------------------
+
+// Stage one entry's X (K fp16) at group xg of the X area: 16-byte chunk ci of the entry lands
+// at xs[16 xg + ci]; the 16 lanes holding a group's chunks sum S_g = sum_k x_k and
+// P_g = sum_k c_k x_k (chunk q of a group holds pairs 4 (q % 4) + w, w < 4, of the record
+// layout) into sp[xg + group].
+template <int BITS>
+__device__ void pass_stage_x(const XItem& X, uint4* xs, float2* sp, int tid) {
+    const int nch = X.K >> 3;  // a multiple of 16
+    for (int c0 = 0; c0 < nch; c0 += 4 * 512) {
+        uint4 v[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int ci = c0 + u * 512 + tid;
+            v[u] = ci < nch ? ld_cg16(X.x + 8 * (size_t)ci) : make_uint4(0u, 0u, 0u, 0u);
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int wfirst = c0 + u * 512 + (tid & ~31);  // the warp's first chunk
+            if (wfirst >= nch) break;                       // warp-uniform
+            const int ci = wfirst + (tid & 31);
+            const uint32_t w4[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
+            float sx = 0.f, px = 0.f;
+#pragma unroll
+            for (int w = 0; w < 4; ++w) {
+                const float2 f = __half22float2(*reinterpret_cast<const __half2*>(&w4[w]));
+                const float pair = f.x + f.y;
+                sx += pair;
+                px = fmaf(row_offset<BITS>((ci & 3) * 4 + w), pair, px);
+            }
+#pragma unroll
+            for (int o = 1; o < 16; o <<= 1) {
+                sx += __shfl_xor_sync(0xffffffffu, sx, o);
+                px += __shfl_xor_sync(0xffffffffu, px, o);
+            }
+            if (ci < nch) {
+                xs[16 * X.xg + ci] = v[u];
+                if ((ci & 15) == 0) sp[X.xg + (ci >> 4)] = make_float2(sx, px);
+            }
+        }
+    }
+}
+
+template <int BITS>
+__device__ void pass_consumer(const PassParams& p, uint8_t* smem, const PassSmem& L,
+                              uint32_t full_s, uint32_t empty_s, volatile int* abort_flag,
+                              int warp, int lane) {
+    constexpr int RBC = RecordFmt<BITS>::kBytes;
+    constexpr int RB = RBC + kSZ;
+    constexpr int SLOT = kPRec * RB;
+    constexpr int WPL = BITS == 4 ? 8 : 6;
+    const int tid = warp * 32 + lane;
+    const int c = lane & 3, R = lane >> 2;
+    const int NS = p.ns;
+    uint4* xs = reinterpret_cast<uint4*>(smem + L.xs);
+    float2* sp = reinterpret_cast<float2*>(smem + L.sp);
+    Seg* segs = reinterpret_cast<Seg*>(smem + L.seg);
+    LTile* tiles = reinterpret_cast<LTile*>(smem + L.tile);
+    XItem* xitems = reinterpret_cast<XItem*>(smem + L.xi);
+    float* slots = reinterpret_cast<float*>(smem + L.slot);
+    const uint4* zblk = reinterpret_cast<const uint4*>(smem + L.zero);
+    const uint8_t* ring = smem;
+    int round = 0;  // rounds of this SM taken so far (the ring position)
+
+    for (int s = 0; s < p.nstages; ++s) {
+        const StageDesc* dp = p.stage + (size_t)blockIdx.x * p.nstages + s;
+        const int n = dp->n, nr = dp->nr, nseg = dp->nseg, nt = dp->nt, nx = dp->nx;
+        // The stage's tables (constants) into shared memory: every consumer has passed the
+        // previous stage's last barrier, so nothing reads the old ones any more.
+        for (int i = tid; i < nseg; i += 512) segs[i] = p.seg[dp->seg0 + i];
+        for (int i = tid; i < nt; i += 512) tiles[i] = p.tile[dp->tile0 + i];
+        for (int i = tid; i < nx; i += 512) xitems[i] = p.xi[dp->x0 + i];
+        const int k0 = dp->wseg[warp], k1 = dp->wseg[warp + 1];
+        // Stage s reads what earlier stages wrote: wait until every CTA has finished stage
+        // s - 1 (and, by induction, all before it).
+        bool bad = false;
+        if (tid == 0 && s > 0 && n > 0)
+            bad = !wait_ge(p.ws + 2 + (s - 1), gridDim.x, p.ws);
+        if (tid == 0 && bad) *abort_flag = 1;
+        if (cbar_any(bad || *abort_flag)) return;
+        if (n > 0) {
+            for (int i = 0; i < nx; ++i) pass_stage_x<BITS>(xitems[i], xs, sp, tid);
+            cbar();
+
+            // This warp's records: the first q + (warp < rem) of the stage's rounds, at
+            // position `warp` of each round's slot.
+            const int len = (n >> 4) + (warp < (n & 15) ? 1 : 0);
+            int k = k0, i = 0, gi = 0;
+            Seg sg = k < k1 ? segs[k] : Seg{0, 0, 0, 0, 0, 0};
+            float D[2][4], y[4], sv[2][2], zv[2][2];
+#pragma unroll
+            for (int v = 0; v < 4; ++v) {
+                D[0][v] = D[1][v] = y[v] = 0.f;
+                sv[v >> 1][v & 1] = zv[v >> 1][v & 1] = 0.f;
+            }
+            bool aborted = false;
+            for (int r = 0; r < nr; ++r) {
+                const int slot = round % NS;
+                const uint32_t par = (uint32_t)((round / NS) & 1);
+                ++round;
+                // (every lane polls; the answer is made warp-wide before the aligned MMAs)
+                if (!__all_sync(0xffffffffu, mbar_wait(full_s + 8u * slot, par, abort_flag, p.ws))) {
+                    aborted = true;
+                    break;
+                }
+                if (r < len) {
+                    const uint8_t* rec = ring + (size_t)slot * SLOT + (size_t)warp * RB;
+                    const int g = sg.g0 + i;
+                    // B fragments: x of the record's group for the lanes of MMA column gi
+                    // (rows 32c .. 32c + 31 of the group), zeros for the other columns.
+                    const uint4* xsrc = R == gi ? xs + 16 * (sg.xg + g) + 4 * c : zblk;
+                    uint32_t B[8][2];
+#pragma unroll
+                    for (int qq = 0; qq < 4; ++qq) {
+                        const uint4 v = xsrc[qq];
+                        B[2 * qq][0] = v.x;
+                        B[2 * qq][1] = v.y;
+                        B[2 * qq + 1][0] = v.z;
+                        B[2 * qq + 1][1] = v.w;
+                    }
+                    uint32_t wd[WPL];
+                    const uint4 c0 = *reinterpret_cast<const uint4*>(rec + lane * 16);
+                    wd[0] = c0.x; wd[1] = c0.y; wd[2] = c0.z; wd[3] = c0.w;
+                    if constexpr (BITS == 4) {
+                        const uint4 c1 = *reinterpret_cast<const uint4*>(rec + 512 + lane * 16);
+                        wd[4] = c1.x; wd[5] = c1.y; wd[6] = c1.z; wd[7] = c1.w;
+                    } else {
+                        const uint2 c1 = *reinterpret_cast<const uint2*>(rec + 512 + lane * 8);
+                        wd[4] = c1.x; wd[5] = c1.y;
+                    }
+                    uint32_t a[8][4];
+                    extract<BITS>(wd, p.exps, a);
+#pragma unroll
+                    for (int j = 0; j < 8; ++j)
+                        mma16816(D[j & 1], a[j][0], a[j][1], a[j][2], a[j][3], B[j][0], B[j][1]);
+                    // The lanes whose accumulator columns include gi keep the record's scales
+                    // and zeros of their two output rows.
+                    if (c == (gi >> 1)) {
+                        const uint16_t* ss = reinterpret_cast<const uint16_t*>(rec + RBC);
+                        const uint8_t* zz = rec + RBC + 32;
+                        const float s0 = __half2float(__ushort_as_half(ss[R]));
+                        const float s1 = __half2float(__ushort_as_half(ss[R + 8]));
+                        const float z0 = (float)zz[R], z1 = (float)zz[R + 8];
+                        if (gi & 1) {
+                            sv[1][0] = s0; sv[1][1] = s1; zv[1][0] = z0; zv[1][1] = z1;
+                        } else {
+                            sv[0][0] = s0; sv[0][1] = s1; zv[0][0] = z0; zv[0][1] = z1;
+                        }
+                    }
+                    ++i;
+                    if (gi == 7 || i == sg.ng) {
+                        // Block epilogue (Eq. (1)): value v is output row R + 8 (v >> 1) and
+                        // MMA column 2c + (v & 1), the block's record of that index.
+                        const int gb = sg.xg + sg.g0 + i - 1 - gi;  // the block's first group
+#pragma unroll
+                        for (int v = 0; v < 4; ++v) {
+                            const int col = 2 * c + (v & 1);
+                            if (col <= gi) {
+                                const float2 spv = sp[gb + col];  // (S, P)
+                                const float dv = D[0][v] + D[1][v];
+                                const float sc = sv[v & 1][v >> 1], zc = zv[v & 1][v >> 1];
+                                y[v] = fmaf(sc, dv - spv.y - zc * spv.x, y[v]);
+                            }
+                            D[0][v] = D[1][v] = 0.f;
+                        }
+                        gi = 0;
+                    } else {
+                        ++gi;
+                    }
+                    if (i == sg.ng) {
+                        // Segment end: the four lanes of an output row hold its two columns'
+                        // partial sums; the slot of segment k gets the 16 outputs.
+                        float lo = y[0] + y[1], hi = y[2] + y[3];
+                        lo += __shfl_xor_sync(0xffffffffu, lo, 1);
+                        hi += __shfl_xor_sync(0xffffffffu, hi, 1);
+                        lo += __shfl_xor_sync(0xffffffffu, lo, 2);
+                        hi += __shfl_xor_sync(0xffffffffu, hi, 2);
+                        if (c == 0) {
+                            slots[16 * k + R] = lo;
+                            slots[16 * k + R + 8] = hi;
+                        }
+#pragma unroll
+                        for (int v = 0; v < 4; ++v) y[v] = 0.f;
+                        ++k;
+                        i = 0;
+                        if (k < k1) sg = segs[k];
+                    }
+                }
+                __syncwarp();
+                if (lane == 0) mbar_arrive(empty_s + 8u * slot);
+            }
+            if (cbar_any(aborted || *abort_flag)) return;
+
+            // The SM's tiles of the stage: each output is its segments' slots summed in order.
+            for (int idx = tid; idx < nt * 16; idx += 512) {
+                const LTile t = tiles[idx >> 4];
+                const int col = idx & 15;
+                float acc = 0.f;
+                for (int q = 0; q < t.nslot; ++q) acc += slots[16 * (t.slot0 + q) + col];
+                t.y[col] = __half_as_ushort(__float2half_rn(acc));
+            }
+            cbar();
+        }
+        if (tid == 0) red_rel_add(p.ws + 2 + s, 1u);
+    }
+}
+
+template <int BITS>
+__global__ void __launch_bounds__(kPThreads, 1) pass_kernel(const PassParams p) {
+    extern __shared__ __align__(128) uint8_t smem[];
+    constexpr int RB = RecordFmt<BITS>::kBytes + kSZ;
+    const PassSmem L = pass_smem(RB, p.ns, p.xs_bytes, p.max_segs, p.max_nx);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const uint32_t base = (uint32_t)__cvta_generic_to_shared(smem);
+    const uint32_t full_s = base + (uint32_t)L.bar;
+    const uint32_t empty_s = full_s + 8u * kMaxRing;
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L.flag);
+
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < p.ns; ++i) {
+            mbar_init(full_s + 8u * i, 1u);
+            mbar_init(empty_s + 8u * i, (uint32_t)kPW);
+        }
+        *abort_flag = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    if (threadIdx.x < 4)
+        reinterpret_cast<uint4*>(smem + L.zero)[threadIdx.x] = make_uint4(0u, 0u, 0u, 0u);
+    __syncthreads();
+
+    const SmDesc sd = p.sm[blockIdx.x];
+    if (warp == kPW)
+        pass_producer<BITS>(p, sd, base, full_s, empty_s, abort_flag, lane);
+    else
+        pass_consumer<BITS>(p, smem, L, full_s, empty_s, abort_flag, warp, lane);
+    __syncthreads();
+
+    // The last CTA to finish zeroes the stage counters for the next call on the stream.
+    if (threadIdx.x == 0 && *abort_flag == 0) {
+        const uint32_t done = atom_acq_rel_add(p.ws + 1, 1u);
+        if (done == gridDim.x - 1) {
+            for (int s = 0; s < p.nstages; ++s) p.ws[2 + s] = 0u;
+            p.ws[1] = 0u;
+        }
+    }
+}
+
+// ---- the gather kernel of laq_pass_prepare -----------------------------------------------------
+
+// One warp per stream record: its packed codes (rbc bytes), then the 16 scales and 16 zeros of
+// its (group, tile).
+__global__ void pass_gather_kernel(const GatherRec* __restrict__ gt,
+                                   const PrepEntry* __restrict__ pe, uint8_t* __restrict__ out,
+                                   int64_t records, int rbc, int rb) {
+    const int lane = threadIdx.x & 31;
+    const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    for (int64_t i = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5; i < records;
+         i += nw) {
+        const GatherRec g = gt[i];
+        const PrepEntry E = pe[g.e];
+        const int t = g.rid / E.G, grp = g.rid - t * E.G;
+        const uint4* src = reinterpret_cast<const uint4*>(E.packed + (int64_t)g.rid * rbc);
+        uint4* dst = reinterpret_cast<uint4*>(out + i * rb);
+        for (int ch = lane; ch < rbc / 16; ch += 32) dst[ch] = src[ch];
+        const size_t so = (size_t)grp * (size_t)E.N + (size_t)t * 16;
+        if (lane < 2)
+            dst[rbc / 16 + lane] = reinterpret_cast<const uint4*>(E.s + so)[lane];
+        else if (lane == 2)
+            dst[rbc / 16 + 2] = *reinterpret_cast<const uint4*>(E.z + so);
+    }
+}
+
+std::atomic<int> g_pass_attr[2];  // dynamic shared memory granted to pass_kernel<3>, <4>
+
+int device_sms(int* sms, int* smem_optin) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return -1;
+    if (cudaDeviceGetAttribute(sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+        return -1;
+    if (cudaDeviceGetAttribute(smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) !=
+        cudaSuccess)
+        return -1;
+    return 0;
+}
+
+}  // namespace
+}  // namespace laq
+
+using namespace laq;
+
+extern "C" {
+
+laq_status laq_pass_plan_sizes(const laq_gemv* gemvs, int32_t count, int32_t num_sms,
+                               size_t* plan_bytes, size_t* device_bytes) {
+    if (!plan_bytes || !device_bytes) return LAQ_ERR_NULL;
+    HostPlan H;
+    const laq_status st = plan_pass(gemvs, count, num_sms, H);
+    if (st != LAQ_OK) return st;
+    PlanHeader h;
+    layout(H, h);
+    *plan_bytes = (size_t)h.plan_bytes;
+    *device_bytes = (size_t)h.device_bytes;
+    return LAQ_OK;
+}
+
+laq_status laq_pass_plan_build(const laq_gemv* gemvs, int32_t count, int32_t num_sms,
+                               void* plan, size_t plan_bytes) {
+    if (!plan) return LAQ_ERR_NULL;
+    HostPlan H;
+    const laq_status st = plan_pass(gemvs, count, num_sms, H);
+    if (st != LAQ_OK) return st;
+    PlanHeader h;
+    layout(H, h);
+    if (plan_bytes < (size_t)h.plan_bytes) return LAQ_ERR_WORKSPACE;
+    uint8_t* out = static_cast<uint8_t*>(plan);
+    std::memset(out, 0, (size_t)h.plan_bytes);
+    std::memcpy(out, &h, sizeof(h));
+    if (count > 0) std::memcpy(out + 256, gemvs, (size_t)count * sizeof(laq_gemv));
+    uint8_t* t = out + h.tables_h;
+    put(t, h.o_sm, H.sm);
+    put(t, h.o_rounds, H.rounds);
+    put(t, h.o_stage, H.stage);
+    put(t, h.o_seg, H.seg);
+    put(t, h.o_tile, H.tile);
+    put(t, h.o_x, H.xi);
+    put(t, h.o_prep, H.prep);
+    put(t, h.o_gather, H.gather);
+    return LAQ_OK;
+}
+
+size_t laq_pass_workspace_bytes(const void* plan) {
+    const PlanHeader* h = as_plan(plan);
+    return h ? pass_workspace(*h) : 0;
+}
+
+laq_status laq_pass_prepare(const void* plan, void* device, size_t device_bytes, void* stream) {
+    const PlanHeader* h = as_plan(plan);
+    if (!h) return LAQ_ERR_CONFIG;
+    if (!device) return LAQ_ERR_NULL;
+    if (reinterpret_cast<uintptr_t>(device) & 255u) return LAQ_ERR_ALIGN;
+    if (device_bytes < (size_t)h->device_bytes) return LAQ_ERR_WORKSPACE;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    uint8_t* dev = static_cast<uint8_t*>(device);
+    const uint8_t* host = static_cast<const uint8_t*>(plan);
+    if (h->tables_bytes > 0 &&
+        cudaMemcpyAsync(dev + h->stream_bytes, host + h->tables_h, (size_t)h->tables_bytes,
+                        cudaMemcpyHostToDevice, st) != cudaSuccess)
+        return LAQ_ERR_CUDA;
+    if (h->records == 0) return LAQ_OK;
+    const uint8_t* tables = dev + h->stream_bytes;
+    const int64_t blocks64 = (h->records + 7) / 8;
+    const unsigned blocks = (unsigned)(blocks64 < 8192 ? blocks64 : 8192);
+    pass_gather_kernel<<<blocks, 256, 0, st>>>(
+        reinterpret_cast<const GatherRec*>(tables + h->o_gather),
+        reinterpret_cast<const PrepEntry*>(tables + h->o_prep), dev, h->records,
+        h->rb - kSZ, h->rb);
+    return cudaGetLastError() == cudaSuccess ? LAQ_OK : LAQ_ERR_CUDA;
+}
+
+laq_status laq_pass_run(const void* plan, const void* device, void* workspace,
+                        size_t workspace_bytes, void* stream) {
+    const PlanHeader* h = as_plan(plan);
+    if (!h) return LAQ_ERR_CONFIG;
+    if (!device || !workspace) return LAQ_ERR_NULL;
+    if (reinterpret_cast<uintptr_t>(device) & 255u) return LAQ_ERR_ALIGN;
+    if ((reinterpret_cast<uintptr_t>(workspace) & 15u) || workspace_bytes < pass_workspace(*h))
+        return LAQ_ERR_WORKSPACE;
+    if (h->nstages == 0) return LAQ_OK;
+    int sms = 0, optin = 0;
+    if (device_sms(&sms, &optin) != 0) return LAQ_ERR_CUDA;
+    if (sms != h->sms) return LAQ_ERR_CONFIG;  // planned for another SM count
+    // ring depth: as many 16-record slots as the shared memory left over holds
+    int ns = kMaxRing;
+    while (ns >= 2 && pass_smem(h->rb, ns, h->xs_bytes, h->max_segs, h->max_nx).total > optin)
+        --ns;
+    if (ns < 2) return LAQ_ERR_SHAPE;
+    const PassSmem L = pass_smem(h->rb, ns, h->xs_bytes, h->max_segs, h->max_nx);
+
+    const uint8_t* dev = static_cast<const uint8_t*>(device);
+    const uint8_t* t = dev + h->stream_bytes;
+    PassParams P;
+    P.stream = dev;
+    P.sm = reinterpret_cast<const SmDesc*>(t + h->o_sm);
+    P.rounds = t + h->o_rounds;
+    P.stage = reinterpret_cast<const StageDesc*>(t + h->o_stage);
+    P.seg = reinterpret_cast<const Seg*>(t + h->o_seg);
+    P.tile = reinterpret_cast<const LTile*>(t + h->o_tile);
+    P.xi = reinterpret_cast<const XItem*>(t + h->o_x);
+    P.ws = static_cast<uint32_t*>(workspace);
+    P.nstages = h->nstages;
+    P.ns = ns;
+    P.xs_bytes = h->xs_bytes;
+    P.max_segs = h->max_segs;
+    P.max_nx = h->max_nx;
+    P.exps = exps_for(h->bits);
+
+    const void* fn = h->bits == 4 ? (const void*)pass_kernel<4> : (const void*)pass_kernel<3>;
+    std::atomic<int>& granted = g_pass_attr[h->bits == 4];
+    if (granted.load() < L.total) {
+        if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, L.total) !=
+            cudaSuccess)
+            return LAQ_ERR_CUDA;
+        granted.store(L.total);
+    }
+    int per_sm = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, kPThreads, L.total) !=
+            cudaSuccess ||
+        per_sm < 1)
+        return LAQ_ERR_CONFIG;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)h->sms);
+    cfg.blockDim = dim3(kPThreads);
+    cfg.dynamicSmemBytes = (size_t)L.total;
+    cfg.stream = static_cast<cudaStream_t>(stream);
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeCooperative;
+    attr[0].val.cooperative = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    void* args[] = {&P};
+    const cudaError_t err = cudaLaunchKernelExC(&cfg, fn, args);
+    if (err == cudaErrorInvalidConfiguration || err == cudaErrorCooperativeLaunchTooLarge)
+        return LAQ_ERR_CONFIG;
+    return err == cudaSuccess ? LAQ_OK : LAQ_ERR_CUDA;
+}
+
+}  // extern "C"
