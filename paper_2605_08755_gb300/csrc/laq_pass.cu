@@ -453,13 +453,21 @@ __device__ __forceinline__ bool mbar_try(uint32_t bar, uint32_t parity) {
         : "memory");
     return ok != 0u;
 }
-// Copy `bytes` (a multiple of 16) from global memory into this CTA's shared memory; the copy
-// counts its bytes against the transaction count of mbarrier `bar`.
+// An L2 policy that evicts first what it tags: the weight stream is read exactly once per pass,
+// so it should not push X, Y and the plan's tables out of L2.
+__device__ __forceinline__ uint64_t evict_first_policy() {
+    uint64_t pol;
+    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
+    return pol;
+}
+// Copy `bytes` (a multiple of 16) from global memory into this CTA's shared memory under L2
+// policy `pol`; the copy counts its bytes against the transaction count of mbarrier `bar`.
 __device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t bytes,
-                                         uint32_t bar) {
+                                         uint32_t bar, uint64_t pol) {
     asm volatile(
-        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
-        ::"r"(dst), "l"(src), "r"(bytes), "r"(bar)
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
+        " [%0], [%1], %2, [%3], %4;"
+        ::"r"(dst), "l"(src), "r"(bytes), "r"(bar), "l"(pol)
         : "memory");
 }
 
@@ -547,6 +555,7 @@ __device__ void pass_producer(const PassParams& p, const SmDesc& sd, uint32_t ri
     const int NS = p.ns, NR = sd.nrounds;
     const uint8_t* src = p.stream + sd.rec0 * RB;
     const uint8_t* rt = p.rounds + sd.round0;
+    const uint64_t pol = evict_first_policy();
     int issued = 0;
     bool ok = true;
     for (int r0 = 0; r0 < NR && ok; r0 += 32) {
@@ -565,7 +574,7 @@ __device__ void pass_producer(const PassParams& p, const SmDesc& sd, uint32_t ri
             if (lane == 0) {
                 const uint32_t bytes = (uint32_t)(cnt * RB);
                 mbar_expect_tx(full_s + 8u * slot, bytes);
-                bulk_g2s(ring_s + SLOT * (uint32_t)slot, src, bytes, full_s + 8u * slot);
+                bulk_g2s(ring_s + SLOT * (uint32_t)slot, src, bytes, full_s + 8u * slot, pol);
             }
             __syncwarp();
             src += (size_t)cnt * RB;
@@ -644,20 +653,24 @@ __device__ void pass_consumer(const PassParams& p, uint8_t* smem, const PassSmem
 
     for (int s = 0; s < p.nstages; ++s) {
         const StageDesc* dp = p.stage + (size_t)blockIdx.x * p.nstages + s;
-        const int n = dp->n, nr = dp->nr, nseg = dp->nseg, nt = dp->nt, nx = dp->nx;
-        // The stage's tables (constants) into shared memory: every consumer has passed the
-        // previous stage's last barrier, so nothing reads the old ones any more.
-        for (int i = tid; i < nseg; i += 512) segs[i] = p.seg[dp->seg0 + i];
-        for (int i = tid; i < nt; i += 512) tiles[i] = p.tile[dp->tile0 + i];
-        for (int i = tid; i < nx; i += 512) xitems[i] = p.xi[dp->x0 + i];
-        const int k0 = dp->wseg[warp], k1 = dp->wseg[warp + 1];
-        // Stage s reads what earlier stages wrote: wait until every CTA has finished stage
-        // s - 1 (and, by induction, all before it).
+        // Stage s reads what earlier stages wrote: thread 0 waits until every CTA has finished
+        // stage s - 1 (and, by induction, all before it), at once, so that the wait is not
+        // queued behind a table load; a CTA without work in the stage waits too, long before
+        // the stage as a whole can finish.  Meanwhile warps 1-15 copy the stage's tables
+        // (constants) into shared memory: every consumer has passed the previous stage's last
+        // barrier, so nothing reads the old ones any more.
         bool bad = false;
-        if (tid == 0 && s > 0 && n > 0)
-            bad = !wait_ge(p.ws + 2 + (s - 1), gridDim.x, p.ws);
+        if (tid == 0 && s > 0) bad = !wait_ge(p.ws + 2 + (s - 1), gridDim.x, p.ws);
         if (tid == 0 && bad) *abort_flag = 1;
+        if (warp > 0) {
+            const int nseg = dp->nseg, nt = dp->nt, nx = dp->nx;
+            for (int i = tid - 32; i < nseg; i += 480) segs[i] = p.seg[dp->seg0 + i];
+            for (int i = tid - 32; i < nt; i += 480) tiles[i] = p.tile[dp->tile0 + i];
+            for (int i = tid - 32; i < nx; i += 480) xitems[i] = p.xi[dp->x0 + i];
+        }
         if (cbar_any(bad || *abort_flag)) return;
+        const int n = dp->n, nr = dp->nr, nt = dp->nt, nx = dp->nx;
+        const int k0 = dp->wseg[warp], k1 = dp->wseg[warp + 1];
         if (n > 0) {
             for (int i = 0; i < nx; ++i) pass_stage_x<BITS>(xitems[i], xs, sp, tid);
             cbar();
