@@ -15,8 +15,9 @@
 //    every warp that has one, warp w's at position w.
 //
 //  * Prepare (once).  A gather kernel writes every SM's stream into one device buffer: each
-//    record's packed codes followed by its 16 scales and 16 zeros, so an SM's whole pass is
-//    one contiguous byte range.
+//    record's packed codes followed by its 16 scales and 16 zeros (as pairs of output rows
+//    r, r + 8, the two rows one lane of the MMA holds), so an SM's whole pass is one contiguous
+//    byte range.
 //
 //  * Run.  One cooperative CTA per SM: 16 consumer warps and one producer warp.  The producer
 //    copies the SM's stream round by round with cp.async.bulk into a ring of shared-memory
@@ -649,7 +650,8 @@ __device__ void pass_consumer(const PassParams& p, uint8_t* smem, const PassSmem
     float* slots = reinterpret_cast<float*>(smem + L.slot);
     const uint4* zblk = reinterpret_cast<const uint4*>(smem + L.zero);
     const uint8_t* ring = smem;
-    int round = 0;  // rounds of this SM taken so far (the ring position)
+    int slot = 0;        // ring position of the SM's next round
+    uint32_t par = 0u;   // and the phase parity of its slot
 
     for (int s = 0; s < p.nstages; ++s) {
         const StageDesc* dp = p.stage + (size_t)blockIdx.x * p.nstages + s;
@@ -680,17 +682,12 @@ __device__ void pass_consumer(const PassParams& p, uint8_t* smem, const PassSmem
             const int len = (n >> 4) + (warp < (n & 15) ? 1 : 0);
             int k = k0, i = 0, gi = 0;
             Seg sg = k < k1 ? segs[k] : Seg{0, 0, 0, 0, 0, 0};
-            float D[2][4], y[4], sv[2][2], zv[2][2];
+            float D[2][4], y[4];
+            uint32_t sw[2] = {0u, 0u}, zw[2] = {0u, 0u};  // scale / zero row pairs, columns 2c, 2c + 1
 #pragma unroll
-            for (int v = 0; v < 4; ++v) {
-                D[0][v] = D[1][v] = y[v] = 0.f;
-                sv[v >> 1][v & 1] = zv[v >> 1][v & 1] = 0.f;
-            }
+            for (int v = 0; v < 4; ++v) D[0][v] = D[1][v] = y[v] = 0.f;
             bool aborted = false;
             for (int r = 0; r < nr; ++r) {
-                const int slot = round % NS;
-                const uint32_t par = (uint32_t)((round / NS) & 1);
-                ++round;
                 // (every lane polls; the answer is made warp-wide before the aligned MMAs)
                 if (!__all_sync(0xffffffffu, mbar_wait(full_s + 8u * slot, par, abort_flag, p.ws))) {
                     aborted = true;
@@ -726,18 +723,17 @@ __device__ void pass_consumer(const PassParams& p, uint8_t* smem, const PassSmem
 #pragma unroll
                     for (int j = 0; j < 8; ++j)
                         mma16816(D[j & 1], a[j][0], a[j][1], a[j][2], a[j][3], B[j][0], B[j][1]);
-                    // The lanes whose accumulator columns include gi keep the record's scales
-                    // and zeros of their two output rows.
+                    // The lanes whose accumulator columns include gi keep the record's scale
+                    // and zero pairs of their output rows R, R + 8 (converted in the epilogue).
                     if (c == (gi >> 1)) {
-                        const uint16_t* ss = reinterpret_cast<const uint16_t*>(rec + RBC);
-                        const uint8_t* zz = rec + RBC + 32;
-                        const float s0 = __half2float(__ushort_as_half(ss[R]));
-                        const float s1 = __half2float(__ushort_as_half(ss[R + 8]));
-                        const float z0 = (float)zz[R], z1 = (float)zz[R + 8];
+                        const uint32_t sr = reinterpret_cast<const uint32_t*>(rec + RBC)[R];
+                        const uint32_t zr = reinterpret_cast<const uint16_t*>(rec + RBC + 32)[R];
                         if (gi & 1) {
-                            sv[1][0] = s0; sv[1][1] = s1; zv[1][0] = z0; zv[1][1] = z1;
+                            sw[1] = sr;
+                            zw[1] = zr;
                         } else {
-                            sv[0][0] = s0; sv[0][1] = s1; zv[0][0] = z0; zv[0][1] = z1;
+                            sw[0] = sr;
+                            zw[0] = zr;
                         }
                     }
                     ++i;
@@ -751,7 +747,9 @@ __device__ void pass_consumer(const PassParams& p, uint8_t* smem, const PassSmem
                             if (col <= gi) {
                                 const float2 spv = sp[gb + col];  // (S, P)
                                 const float dv = D[0][v] + D[1][v];
-                                const float sc = sv[v & 1][v >> 1], zc = zv[v & 1][v >> 1];
+                                const float sc = __half2float(__ushort_as_half(
+                                    (uint16_t)(sw[v & 1] >> (16 * (v >> 1)))));
+                                const float zc = (float)((zw[v & 1] >> (8 * (v >> 1))) & 0xffu);
                                 y[v] = fmaf(sc, dv - spv.y - zc * spv.x, y[v]);
                             }
                             D[0][v] = D[1][v] = 0.f;
@@ -781,6 +779,10 @@ __device__ void pass_consumer(const PassParams& p, uint8_t* smem, const PassSmem
                 }
                 __syncwarp();
                 if (lane == 0) mbar_arrive(empty_s + 8u * slot);
+                if (++slot == NS) {
+                    slot = 0;
+                    par ^= 1u;
+                }
             }
             if (cbar_any(aborted || *abort_flag)) return;
 
@@ -840,8 +842,10 @@ __global__ void __launch_bounds__(kPThreads, 1) pass_kernel(const PassParams p) 
 
 // ---- the gather kernel of laq_pass_prepare -----------------------------------------------------
 
-// One warp per stream record: its packed codes (rbc bytes), then the 16 scales and 16 zeros of
-// its (group, tile).
+// One warp per stream record: its packed codes (rbc bytes), then the scales and zeros of its
+// (group, tile) as row pairs: 32-bit word r (r < 8) holds the fp16 scales of tile columns r
+// (low half) and r + 8 (high half), then 16-bit word r the zeros of columns r (low byte) and
+// r + 8, so the lane of output rows r and r + 8 reads one word and one half-word.
 __global__ void pass_gather_kernel(const GatherRec* __restrict__ gt,
                                    const PrepEntry* __restrict__ pe, uint8_t* __restrict__ out,
                                    int64_t records, int rbc, int rb) {
@@ -856,10 +860,13 @@ __global__ void pass_gather_kernel(const GatherRec* __restrict__ gt,
         uint4* dst = reinterpret_cast<uint4*>(out + i * rb);
         for (int ch = lane; ch < rbc / 16; ch += 32) dst[ch] = src[ch];
         const size_t so = (size_t)grp * (size_t)E.N + (size_t)t * 16;
-        if (lane < 2)
-            dst[rbc / 16 + lane] = reinterpret_cast<const uint4*>(E.s + so)[lane];
-        else if (lane == 2)
-            dst[rbc / 16 + 2] = *reinterpret_cast<const uint4*>(E.z + so);
+        if (lane < 8) {
+            uint8_t* sz = out + i * rb + rbc;
+            reinterpret_cast<uint32_t*>(sz)[lane] =
+                (uint32_t)E.s[so + lane] | ((uint32_t)E.s[so + lane + 8] << 16);
+            reinterpret_cast<uint16_t*>(sz + 32)[lane] =
+                (uint16_t)((uint32_t)E.z[so + lane] | ((uint32_t)E.z[so + lane + 8] << 8));
+        }
     }
 }
 
