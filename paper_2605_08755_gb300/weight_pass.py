@@ -68,12 +68,19 @@ class WeightPass:
     With ``chain``, the whole pass is one ``laq_gemm_chain`` launch (M <= 4) whose stages follow
     the decoder's data flow: an entry waits for every earlier one unless it reads the input of
     the projection before it (k and v after q, up after gate), so each layer has the four
-    dependency points q|k|v -> o -> gate|up -> down -> next layer."""
+    dependency points q|k|v -> o -> gate|up -> down -> next layer.
+
+    With ``planned`` (M = 1), the same entries run through ``laq_pass_run`` after
+    ``laq_pass_prepare`` has laid their weights out as per-SM streams (``_lib.PassPlan``)."""
 
     def __init__(self, model="qwen3-4b", bits=3, M=1, layers=inputs.LAYERS, seed=0,
-                 outliers=False, device="cuda", pdl=True, fuse=False, chain=False):
+                 outliers=False, device="cuda", pdl=True, fuse=False, chain=False,
+                 planned=False):
+        if planned and M != 1:
+            raise ValueError("the planned pass runs M = 1 only")
         self.model, self.bits, self.M, self.layers = model, bits, M, layers
         self.seed, self.outliers, self.fuse, self.chain = seed, outliers, fuse, chain
+        self.planned = planned
         self.device = torch.device(device)
         plan = pass_plan(model, fuse, layers)
         xs = sum(M * K for *_, K, N in plan)
@@ -102,13 +109,17 @@ class WeightPass:
             c = _lib.laq_gemm_plan(M, q.K, q.N, bits, sms)
             c.pdl = 1 if pdl else 0
             self.configs.append(c)
-        if chain:
+        if chain or planned:
             entries = []
             for i, (_, members, name, q) in enumerate(self.linears):
                 wait = not (name in SHARES_INPUT and i > 0)
                 entries.append((self.X[i], q.packed, q.s, q.z, bits, self.Y[i], wait))
-            self.chain_spec = _lib.Chain(entries)
-            self.ws = _lib.chain_workspace(len(entries), self.device)
+            if planned:
+                self.plan = _lib.PassPlan(entries, self.device)
+                self.ws = self.plan.ws
+            else:
+                self.chain_spec = _lib.Chain(entries)
+                self.ws = _lib.chain_workspace(len(entries), self.device)
         torch.cuda.synchronize(self.device)
 
     def weight(self, layer, members):
@@ -125,7 +136,7 @@ class WeightPass:
 
     @property
     def launches(self):
-        return 1 if self.chain else len(self.linears)
+        return 1 if self.chain or self.planned else len(self.linears)
 
     def bytes_per_pass(self):
         return sum(q.bytes_per_call(self.M) for *_, q in self.linears)
@@ -136,10 +147,13 @@ class WeightPass:
     def run(self, stream=None, events=None):
         """Launch the pass; with ``events`` (launches + 1 CUDA events) record one before each
         launch and one after the last."""
-        if self.chain:
+        if self.chain or self.planned:
             if events is not None:
                 events[0].record(stream)
-            self.chain_spec.run(self.ws, stream)
+            if self.planned:
+                self.plan.run(stream)
+            else:
+                self.chain_spec.run(self.ws, stream)
             if events is not None:
                 events[-1].record(stream)
             return
