@@ -2,13 +2,14 @@
 
     python -m paper_2605_08755_gb300.pass_case --variant graph_fused --bits 3 --M 1 --replays 3
 
-Builds the Qwen3-4B-shaped pass (36 layers, synthetic weights) in one of its four forms
-(``graph_252``, ``graph_fused``, ``chain_252``, ``chain_fused``), captures it into a CUDA graph
+Builds the Qwen3-4B-shaped pass (36 layers, synthetic weights) in one of its forms
+(``graph_252``, ``graph_fused``, ``chain_252``, ``chain_fused``, and the planned pass over
+per-SM weight streams, ``planned_252`` and ``planned_fused``, M = 1), captures it into a CUDA graph
 (the capture is preceded by one eager run of the pass), replays the graph ``replays`` times and
 prints the mean device time per replay.  Under a profiler, the first replay's kernels follow the
 eager run's: for a graph form, ``-k regex:gemm_kernel -s L -c L`` with L = the printed
 ``launches`` selects exactly the first replay; for a chain form, ``-k regex:chain_kernel -s 1
--c 1`` does.
+-c 1`` does, and ``-k regex:pass_kernel -s 1 -c 1`` for a planned form.
 """
 import argparse
 import json
@@ -17,8 +18,9 @@ import torch
 
 from .weight_pass import WeightPass
 
-VARIANTS = {"graph_252": (False, False), "graph_fused": (True, False),
-            "chain_252": (False, True), "chain_fused": (True, True)}
+VARIANTS = {"graph_252": (False, False, False), "graph_fused": (True, False, False),
+            "chain_252": (False, True, False), "chain_fused": (True, True, False),
+            "planned_252": (False, False, True), "planned_fused": (True, False, True)}
 
 
 def main():
@@ -30,11 +32,12 @@ def main():
     ap.add_argument("--layers", type=int, default=36)
     ap.add_argument("--replays", type=int, default=3)
     a = ap.parse_args()
-    fuse, chain = VARIANTS[a.variant]
+    fuse, chain, planned = VARIANTS[a.variant]
     dev = torch.device("cuda", 0)
     torch.cuda.set_device(dev)
     wp = WeightPass(model=a.model, bits=a.bits, M=a.M, layers=a.layers, device=dev,
-                    outliers=(a.model == "qwen3-8b"), fuse=fuse, chain=chain)
+                    outliers=(a.model == "qwen3-8b"), fuse=fuse, chain=chain,
+                    planned=planned)
     stream = torch.cuda.Stream(dev)
     g = wp.capture(stream=stream)
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
