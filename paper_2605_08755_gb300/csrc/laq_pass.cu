@@ -683,13 +683,15 @@ __device__ void pass_consumer(const PassParams& p, uint8_t* smem, const PassSmem
             int k = k0, i = 0, gi = 0;
             Seg sg = k < k1 ? segs[k] : Seg{0, 0, 0, 0, 0, 0};
             float D[2][4], y[4];
-            uint32_t sw[2] = {0u, 0u}, zw[2] = {0u, 0u};  // scale / zero row pairs, columns 2c, 2c + 1
+            // scale and zero row pairs of the lane's block columns 2c, 2c + 1
+            uint32_t sw[2] = {0u, 0u}, zw[2] = {0u, 0u};
 #pragma unroll
             for (int v = 0; v < 4; ++v) D[0][v] = D[1][v] = y[v] = 0.f;
             bool aborted = false;
             for (int r = 0; r < nr; ++r) {
                 // (every lane polls; the answer is made warp-wide before the aligned MMAs)
-                if (!__all_sync(0xffffffffu, mbar_wait(full_s + 8u * slot, par, abort_flag, p.ws))) {
+                if (!__all_sync(0xffffffffu,
+                                mbar_wait(full_s + 8u * slot, par, abort_flag, p.ws))) {
                     aborted = true;
                     break;
                 }

@@ -255,7 +255,8 @@ def emulate(tb, shapes, bits, data):
                 e = next(e for e in range(len(shapes))
                          if addr(e, "Y") <= int(ti["y"]) < addr(e, "Y") + 2 * shapes[e][1])
                 t = (int(ti["y"]) - addr(e, "Y")) // 32
-                Y[e][16 * t:16 * t + 16] = slots[int(ti["slot0"]):int(ti["slot0"] + ti["nslot"])].sum(0)
+                k0, nk = int(ti["slot0"]), int(ti["nslot"])
+                Y[e][16 * t:16 * t + 16] = slots[k0:k0 + nk].sum(0)
             base += n
     return Y
 
