@@ -6,10 +6,10 @@ Builds the Qwen3-4B-shaped pass (36 layers, synthetic weights) in one of its for
 (``graph_252``, ``graph_fused``, ``chain_252``, ``chain_fused``, and the planned pass over
 per-SM weight streams, ``planned_252`` and ``planned_fused``, M = 1), captures it into a CUDA
 graph (the capture is preceded by one eager run of the pass), replays the graph ``replays``
-times and prints the mean device time per replay.  Under a profiler, the first replay's kernels follow the
-eager run's: for a graph form, ``-k regex:gemm_kernel -s L -c L`` with L = the printed
-``launches`` selects exactly the first replay; for a chain form, ``-k regex:chain_kernel -s 1
--c 1`` does, and ``-k regex:pass_kernel -s 1 -c 1`` for a planned form.
+times and prints the mean device time per replay.  Under a profiler, the first replay's kernels
+follow the eager run's: for a graph form, ``-k regex:gemm_kernel -s L -c L`` with L = the
+printed ``launches`` selects exactly the first replay; for a chain form, ``-k
+regex:chain_kernel -s 1 -c 1`` does, and ``-k regex:pass_kernel -s 1 -c 1`` for a planned form.
 """
 import argparse
 import json
