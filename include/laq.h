@@ -299,7 +299,9 @@ laq_status laq_pass_prepare(const void *plan, void *device, size_t device_bytes,
  * call leaves it zero again); word 0 (uint32) is the device-side status: 0, or LAQ_ERR_TIMEOUT
  * if a wait gave up after about a second (Y undefined; zero the workspace before the next
  * call).  Calls sharing one workspace must not overlap in time.  The device must have the SM
- * count the plan was built for (LAQ_ERR_CONFIG otherwise).  Errors: LAQ_ERR_CONFIG (not a plan,
+ * count the plan was built for (LAQ_ERR_CONFIG otherwise).  The first call for each bit width
+ * and shared-memory size sets the kernel's limit: make it before any stream capture, which may
+ * then record later calls.  Errors: LAQ_ERR_CONFIG (not a plan,
  * another SM count, the launch does not fit), LAQ_ERR_NULL, LAQ_ERR_ALIGN (device buffer),
  * LAQ_ERR_WORKSPACE, LAQ_ERR_SHAPE (the staging area and a ring of two slots exceed shared
  * memory), LAQ_ERR_CUDA. */

@@ -997,18 +997,20 @@ laq_status laq_pass_run(const void* plan, const void* device, void* workspace,
     P.exps = exps_for(h->bits);
 
     const void* fn = h->bits == 4 ? (const void*)pass_kernel<4> : (const void*)pass_kernel<3>;
+    // First call with this much shared memory (before any stream capture): raise the kernel's
+    // limit and check that a CTA fits an SM, as the cooperative launch requires.
     std::atomic<int>& granted = g_pass_attr[h->bits == 4];
     if (granted.load() < L.total) {
         if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, L.total) !=
             cudaSuccess)
             return LAQ_ERR_CUDA;
+        int per_sm = 0;
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, kPThreads, L.total) !=
+                cudaSuccess ||
+            per_sm < 1)
+            return LAQ_ERR_CONFIG;
         granted.store(L.total);
     }
-    int per_sm = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, kPThreads, L.total) !=
-            cudaSuccess ||
-        per_sm < 1)
-        return LAQ_ERR_CONFIG;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)h->sms);
     cfg.blockDim = dim3(kPThreads);
