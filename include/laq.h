@@ -281,7 +281,7 @@ laq_status laq_pass_plan_build(const laq_gemv *gemvs, int32_t count, int32_t num
                                void *plan, size_t plan_bytes);
 
 /* Workspace bytes laq_pass_run needs for this plan (status word, a finished-CTA count and one
- * counter per stage; 0 if `plan` is not a plan). */
+ * completed-stage flag per SM; 0 if `plan` is not a plan). */
 size_t laq_pass_workspace_bytes(const void *plan);
 
 /* Lay the plan's weights out in the DEVICE buffer `device` (256-byte aligned, device_bytes from

@@ -24,10 +24,10 @@
 //    slots (one mbarrier pair per slot), with no knowledge of stages: weights never depend on
 //    activations, so the ring runs ahead across stage boundaries while the consumers wait for
 //    a stage's input.  Per stage the consumers wait for every SM to have finished the previous
-//    stage (a release/acquire counter per stage in the workspace), stage the stage's X in
-//    shared memory with the group sums S_g = sum_k x_k and P_g = sum_k c_k x_k, take their
-//    records from the ring (one per round and warp), and reduce their partial tiles in warp
-//    order (deterministic, no atomics on Y).
+//    stage (a release flag per CTA in the workspace: the stages it has completed), stage the
+//    stage's X in shared memory with the group sums S_g = sum_k x_k and P_g = sum_k c_k x_k,
+//    take their records from the ring (one per round and warp), and reduce their partial tiles
+//    in warp order (deterministic, no atomics on Y).
 //
 //  * The record arithmetic is that of laq_gemm_wxg128 at M = 1: one mask-and-or per pair of
 //    codes gives fp16 values c + q, the m16n8k16 MMA contracts them with raw x, the eight groups
@@ -376,8 +376,9 @@ const PlanHeader* as_plan(const void* plan) {
     return h;
 }
 
+// Workspace: [0] status, [1] finished CTAs, [2 + j] the stages CTA j has completed.
 size_t pass_workspace(const PlanHeader& h) {
-    return (size_t)align_up(4 * (2 + (int64_t)h.nstages), 256);
+    return (size_t)align_up(4 * (2 + (int64_t)h.sms), 256);
 }
 
 // ---- shared memory layout of the pass kernel (host and device) -------------------------------
@@ -418,8 +419,8 @@ __device__ __forceinline__ uint32_t ld_rlx(const uint32_t* p) {
     asm volatile("ld.relaxed.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
     return v;
 }
-__device__ __forceinline__ void red_rel_add(uint32_t* p, uint32_t v) {
-    asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+__device__ __forceinline__ void st_rel(uint32_t* p, uint32_t v) {
+    asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
 }
 __device__ __forceinline__ uint32_t atom_acq_rel_add(uint32_t* p, uint32_t v) {
     uint32_t old;
@@ -515,20 +516,25 @@ __device__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort_fla
     return false;
 }
 
-// Wait until *cnt >= target (acquire).  False when the status word already holds an error or
-// after about a second (then LAQ_ERR_TIMEOUT is recorded).
-__device__ bool wait_ge(const uint32_t* cnt, uint32_t target, uint32_t* status) {
-    if (ld_rlx(status) != 0u) return false;
-    if (ld_acq(cnt) >= target) return true;
+// One warp waits until every CTA's completed-stage flag (flags[0 .. n)) is >= target, each
+// lane reading every 32nd flag with acquire loads, so a poll is one round trip to L2 and no two
+// CTAs ever write the same word.  Returns the same answer in every lane: false when the status
+// word already holds an error, or after about a second (then LAQ_ERR_TIMEOUT is recorded).
+__device__ bool wait_flags(const uint32_t* flags, int n, uint32_t target, uint32_t* status,
+                           int lane) {
     const unsigned long long t0 = gtimer();
     for (int spin = 0; spin < kWaitSpins; ++spin) {
-        if (ld_acq(cnt) >= target) return true;
-        if ((spin & 31) == 31) {
-            if (ld_rlx(status) != 0u) return false;
-            if (gtimer() - t0 > kWaitNs) break;
+        if ((spin & 31) == 0) {
+            const uint32_t st = lane == 0 ? ld_rlx(status) : 0u;
+            if (__shfl_sync(0xffffffffu, st, 0) != 0u) return false;
+            const bool late = lane == 0 && spin > 0 && gtimer() - t0 > kWaitNs;
+            if (__shfl_sync(0xffffffffu, (int)late, 0)) break;
         }
+        bool ok = true;
+        for (int j = lane; j < n; j += 32) ok = ok && ld_acq(flags + j) >= target;
+        if (__all_sync(0xffffffffu, ok)) return true;
     }
-    record_timeout(status);
+    if (lane == 0) record_timeout(status);
     return false;
 }
 
@@ -540,7 +546,7 @@ struct PassParams {
     const Seg* seg;
     const LTile* tile;
     const XItem* xi;
-    uint32_t* ws;  // [0] status, [1] finished CTAs, [2 + s] CTAs done with stage s
+    uint32_t* ws;  // [0] status, [1] finished CTAs, [2 + j] stages CTA j has completed
     int nstages, ns, xs_bytes, max_segs, max_nx;
     Exps exps;
 };
@@ -655,14 +661,14 @@ __device__ void pass_consumer(const PassParams& p, uint8_t* smem, const PassSmem
 
     for (int s = 0; s < p.nstages; ++s) {
         const StageDesc* dp = p.stage + (size_t)blockIdx.x * p.nstages + s;
-        // Stage s reads what earlier stages wrote: thread 0 waits until every CTA has finished
-        // stage s - 1 (and, by induction, all before it), at once, so that the wait is not
-        // queued behind a table load; a CTA without work in the stage waits too, long before
-        // the stage as a whole can finish.  Meanwhile warps 1-15 copy the stage's tables
-        // (constants) into shared memory: every consumer has passed the previous stage's last
-        // barrier, so nothing reads the old ones any more.
+        // Stage s reads what earlier stages wrote: warp 0 waits until every CTA has completed
+        // stage s - 1 (hence all before it), at once, so that the wait is not queued behind a
+        // table load; a CTA without work in the stage waits too, long before the stage as a
+        // whole can finish.  Meanwhile warps 1-15 copy the stage's tables (constants) into
+        // shared memory: every consumer has passed the previous stage's last barrier, so
+        // nothing reads the old ones any more.
         bool bad = false;
-        if (tid == 0 && s > 0) bad = !wait_ge(p.ws + 2 + (s - 1), gridDim.x, p.ws);
+        if (warp == 0 && s > 0) bad = !wait_flags(p.ws + 2, gridDim.x, (uint32_t)s, p.ws, lane);
         if (tid == 0 && bad) *abort_flag = 1;
         if (warp > 0) {
             const int nseg = dp->nseg, nt = dp->nt, nx = dp->nx;
@@ -798,7 +804,7 @@ __device__ void pass_consumer(const PassParams& p, uint8_t* smem, const PassSmem
             }
             cbar();
         }
-        if (tid == 0) red_rel_add(p.ws + 2 + s, 1u);
+        if (tid == 0) st_rel(p.ws + 2 + blockIdx.x, (uint32_t)(s + 1));  // after its Y stores
     }
 }
 
@@ -832,11 +838,12 @@ __global__ void __launch_bounds__(kPThreads, 1) pass_kernel(const PassParams p) 
         pass_consumer<BITS>(p, smem, L, full_s, empty_s, abort_flag, warp, lane);
     __syncthreads();
 
-    // The last CTA to finish zeroes the stage counters for the next call on the stream.
+    // The last CTA to finish (every other one has made its last flag read) zeroes the flags
+    // for the next call on the stream.
     if (threadIdx.x == 0 && *abort_flag == 0) {
         const uint32_t done = atom_acq_rel_add(p.ws + 1, 1u);
         if (done == gridDim.x - 1) {
-            for (int s = 0; s < p.nstages; ++s) p.ws[2 + s] = 0u;
+            for (unsigned j = 0; j < gridDim.x; ++j) p.ws[2 + j] = 0u;
             p.ws[1] = 0u;
         }
     }
