@@ -688,11 +688,11 @@ __device__ void pass_consumer(const PassParams& p, uint8_t* smem, const PassSmem
             const int len = (n >> 4) + (warp < (n & 15) ? 1 : 0);
             int k = k0, i = 0, gi = 0;
             Seg sg = k < k1 ? segs[k] : Seg{0, 0, 0, 0, 0, 0};
-            float D[2][4], y[4];
+            float D[4][4], y[4];  // four accumulator chains: k16 steps j, j + 4 share one
             // scale and zero row pairs of the lane's block columns 2c, 2c + 1
             uint32_t sw[2] = {0u, 0u}, zw[2] = {0u, 0u};
 #pragma unroll
-            for (int v = 0; v < 4; ++v) D[0][v] = D[1][v] = y[v] = 0.f;
+            for (int v = 0; v < 4; ++v) D[0][v] = D[1][v] = D[2][v] = D[3][v] = y[v] = 0.f;
             bool aborted = false;
             for (int r = 0; r < nr; ++r) {
                 // (every lane polls; the answer is made warp-wide before the aligned MMAs)
@@ -730,7 +730,7 @@ __device__ void pass_consumer(const PassParams& p, uint8_t* smem, const PassSmem
                     extract<BITS>(wd, p.exps, a);
 #pragma unroll
                     for (int j = 0; j < 8; ++j)
-                        mma16816(D[j & 1], a[j][0], a[j][1], a[j][2], a[j][3], B[j][0], B[j][1]);
+                        mma16816(D[j & 3], a[j][0], a[j][1], a[j][2], a[j][3], B[j][0], B[j][1]);
                     // The lanes whose accumulator columns include gi keep the record's scale
                     // and zero pairs of their output rows R, R + 8 (converted in the epilogue).
                     if (c == (gi >> 1)) {
@@ -754,13 +754,13 @@ __device__ void pass_consumer(const PassParams& p, uint8_t* smem, const PassSmem
                             const int col = 2 * c + (v & 1);
                             if (col <= gi) {
                                 const float2 spv = sp[gb + col];  // (S, P)
-                                const float dv = D[0][v] + D[1][v];
+                                const float dv = (D[0][v] + D[1][v]) + (D[2][v] + D[3][v]);
                                 const float sc = __half2float(__ushort_as_half(
                                     (uint16_t)(sw[v & 1] >> (16 * (v >> 1)))));
                                 const float zc = (float)((zw[v & 1] >> (8 * (v >> 1))) & 0xffu);
                                 y[v] = fmaf(sc, dv - spv.y - zc * spv.x, y[v]);
                             }
-                            D[0][v] = D[1][v] = 0.f;
+                            D[0][v] = D[1][v] = D[2][v] = D[3][v] = 0.f;
                         }
                         gi = 0;
                     } else {
