@@ -393,3 +393,13 @@ def test_plan_buffer_and_run_arguments(L):
     empty, dev0 = _lib.pass_plan(fake_entries([]), 0, 8)
     assert parse(empty)["h"]["nstages"] == 0 and parse(empty)["h"]["records"] == 0
     assert L.laq_pass_run(empty, D, WS, 256, None) == 0
+
+
+def test_segment_limit_per_sm_stage(L):
+    """An SM's share of a stage holds at most 255 warp segments (one-group tiles here: a segment
+    per tile); one more is rejected with LAQ_ERR_SHAPE."""
+    assert sizes(L, fake_entries([(128, 16 * 255, 0)]), 1, 1) == 0
+    assert sizes(L, fake_entries([(128, 16 * 256, 0)]), 1, 1) == 4
+    plan, dev = _lib.pass_plan(fake_entries([(128, 16 * 255, 0)]), 1, 1)
+    tb = check_plan([(128, 16 * 255, 0)], 1, 3, plan, dev)
+    assert tb["h"]["max_segs"] == 255
