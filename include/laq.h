@@ -255,7 +255,7 @@ laq_status laq_gemm_chain_static(const laq_gemv *gemvs, int32_t count, void *str
  * activations), while the stages wait for their inputs.  It serves the decode-step weight pass
  * (Sec. 5.2, "Inference": a decode step streams every projection's weights once), and each
  * entry's Y is that of laq_gemm_wxg128 (fp32 sums of Eq. (1) products, one fp16 rounding; the
- * summation orders differ).  M = 1 only.
+ * summation orders differ).  M = 1..4, the same for every entry.
  *
  * Usage: laq_pass_plan_sizes -> allocate the host plan (plan_bytes) and the device buffer
  * (device_bytes, 256-byte aligned) -> laq_pass_plan_build -> laq_pass_prepare -> a zeroed
@@ -264,12 +264,12 @@ laq_status laq_gemm_chain_static(const laq_gemv *gemvs, int32_t count, void *str
 
 /* Host bytes of the plan and device bytes of the streams and tables for `count` entries
  * (HOST array, read during the call) on a device with `num_sms` SMs.  Host work only (no CUDA
- * call).  Entries as laq_gemm_chain's, with M = 1, one `bits` for all, K <= 24576 (an entry's X
- * must fit the kernel's staging area), N % 16 == 0, K, N > 0.  The device buffer holds every
+ * call).  Entries as laq_gemm_chain's, with one M (1..4) and one `bits` for all, M * K * 2 <=
+ * 106496 bytes (an entry's X must fit the kernel's staging area), N % 16 == 0, K, N > 0.  The device buffer holds every
  * packed record once more (K * N * bits / 8 + 3 * N * K / 128 bytes per entry) plus tables.
- * Errors: LAQ_ERR_NULL, LAQ_ERR_BITS (invalid or mixed bits), LAQ_ERR_M_RANGE (M != 1),
- * LAQ_ERR_SHAPE (count outside 0..LAQ_CHAIN_MAX, num_sms outside 1..1024, a bad K or N, or an
- * SM's share of one stage above 255 warp segments), LAQ_ERR_ALIGN (a pointer not 16-byte
+ * Errors: LAQ_ERR_NULL, LAQ_ERR_BITS (invalid or mixed bits), LAQ_ERR_M_RANGE (M outside 1..4
+ * or mixed), LAQ_ERR_SHAPE (count outside 0..LAQ_CHAIN_MAX, num_sms outside 1..1024, a bad K or
+ * N, an SM's share of one stage above 255 warp segments, or the X it stages above 106496 bytes), LAQ_ERR_ALIGN (a pointer not 16-byte
  * aligned). */
 laq_status laq_pass_plan_sizes(const laq_gemv *gemvs, int32_t count, int32_t num_sms,
                                size_t *plan_bytes, size_t *device_bytes);

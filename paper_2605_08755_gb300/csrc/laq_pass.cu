@@ -59,7 +59,8 @@ constexpr int kPThreads = (kPW + 1) * 32;      // and the producer warp
 constexpr int kPRec = 16;                      // records per round (one per consumer warp)
 constexpr int kSZ = 48;                        // a record's 16 fp16 scales and 16 uint8 zeros
 constexpr int kMaxSegs = 255;                  // warp segments per (SM, stage)
-constexpr int kMaxXsBytes = 48 * 1024;         // staged X per (SM, stage)
+constexpr int kMaxXsBytes = 104 * 1024;        // staged X per (SM, stage), all M rows
+constexpr int kMaxM = 4;                       // batch rows
 constexpr int kMaxRing = 16;                   // ring slots
 constexpr int kMaxSms = 1024;
 constexpr unsigned long long kWaitNs = 1000000000ull;  // wait limit (1 s)
@@ -89,8 +90,10 @@ struct Seg {           // groups [g0, g0 + ng) of tile t of entry e, as one warp
     int16_t lt;        // local tile (index into the stage's local tiles)
 };
 struct LTile {         // a tile of the SM's stage share: its 16 outputs, its segments' slots
-    uint16_t* y;       // Y + 16 t of its entry
+    uint16_t* y;       // Y + 16 t of its entry (row 0)
     int32_t slot0, nslot;
+    int32_t ldy;       // the entry's N: the distance between Y rows
+    int32_t pad;
 };
 struct XItem {         // one entry's X staged for the SM's stage share
     const uint16_t* x;
@@ -107,7 +110,7 @@ struct GatherRec {     // stream record i is record rid = t * G + g of entry e
     int32_t e, rid;
 };
 static_assert(sizeof(SmDesc) == 16 && sizeof(StageDesc) == 48 && sizeof(Seg) == 16 &&
-                  sizeof(LTile) == 16 && sizeof(XItem) == 16 && sizeof(PrepEntry) == 32 &&
+                  sizeof(LTile) == 24 && sizeof(XItem) == 16 && sizeof(PrepEntry) == 32 &&
                   sizeof(GatherRec) == 8,
               "plan table layout");
 
@@ -116,7 +119,9 @@ struct PlanHeader {
     int32_t version;
     int32_t count, nstages, sms, bits;
     int32_t rb;        // stream bytes of a record (packed codes + scales + zeros)
-    int32_t xs_bytes;  // largest staged X of an (SM, stage)
+    int32_t M;         // batch rows of every entry
+    int32_t xg_row;    // groups of one staged X row: the most any (SM, stage) stages
+    int32_t xs_bytes;  // the X area: M rows of xg_row groups (256 bytes each)
     int32_t max_segs;  // most segments of an (SM, stage)
     int32_t max_nx;    // most staged X items of an (SM, stage)
     int64_t records, rounds, segs, ltiles, xitems;
@@ -136,8 +141,8 @@ int record_bytes(int bits) { return (bits == 4 ? 1024 : 768) + kSZ; }
 // ---- host planner ------------------------------------------------------------------------------
 
 struct HostPlan {
-    int count = 0, nstages = 0, sms = 0, bits = 3;
-    int xs_bytes = 0, max_segs = 0, max_nx = 0;
+    int count = 0, nstages = 0, sms = 0, bits = 3, M = 1;
+    int xg_row = 0, max_segs = 0, max_nx = 0;
     std::vector<SmDesc> sm;
     std::vector<uint8_t> rounds;
     std::vector<StageDesc> stage;
@@ -163,9 +168,11 @@ laq_status plan_pass(const laq_gemv* g, int32_t count, int32_t P, HostPlan& H) {
         if (e.bits != 3 && e.bits != 4) return LAQ_ERR_BITS;
         if (i == 0) H.bits = e.bits;
         if (e.bits != H.bits) return LAQ_ERR_BITS;
-        if (e.M != 1) return LAQ_ERR_M_RANGE;
+        if (e.M < 1 || e.M > kMaxM) return LAQ_ERR_M_RANGE;
+        if (i == 0) H.M = (int)e.M;
+        if (e.M != H.M) return LAQ_ERR_M_RANGE;
         if (e.K <= 0 || e.N <= 0 || e.K % 128 != 0 || e.N % 16 != 0) return LAQ_ERR_SHAPE;
-        if (e.K * 2 > kMaxXsBytes || e.N / 16 > ((int64_t)1 << 24)) return LAQ_ERR_SHAPE;
+        if (e.K * 2 * e.M > kMaxXsBytes || e.N / 16 > ((int64_t)1 << 24)) return LAQ_ERR_SHAPE;
         if (!e.X || !e.packed || !e.s || !e.z || !e.Y) return LAQ_ERR_NULL;
         if (!aligned16(e.X) || !aligned16(e.packed) || !aligned16(e.s) || !aligned16(e.z) ||
             !aligned16(e.Y))
@@ -253,8 +260,8 @@ laq_status plan_pass(const laq_gemv* g, int32_t count, int32_t P, HostPlan& H) {
                 }
                 xg_of[k] = H.xi.back().xg;
             }
-            if (xg * 256 > kMaxXsBytes) return LAQ_ERR_SHAPE;
-            if (xg * 256 > H.xs_bytes) H.xs_bytes = xg * 256;
+            if ((int64_t)xg * 256 * H.M > kMaxXsBytes) return LAQ_ERR_SHAPE;
+            if (xg > H.xg_row) H.xg_row = xg;
             if (d.nx > H.max_nx) H.max_nx = d.nx;
             // record offset of each local tile
             std::vector<int64_t> toff(tl.size() + 1, 0);
@@ -288,6 +295,8 @@ laq_status plan_pass(const laq_gemv* g, int32_t count, int32_t P, HostPlan& H) {
                 t.y = static_cast<uint16_t*>(g[tl[k].e].Y) + tl[k].t * 16;
                 t.slot0 = -1;
                 t.nslot = 0;
+                t.ldy = (int32_t)g[tl[k].e].N;
+                t.pad = 0;
                 H.tile.push_back(t);
             }
             for (int k = 0; k < nseg; ++k) {
@@ -334,7 +343,9 @@ void layout(const HostPlan& H, PlanHeader& h) {
     h.sms = H.sms;
     h.bits = H.bits;
     h.rb = record_bytes(H.bits);
-    h.xs_bytes = H.xs_bytes;
+    h.M = H.M;
+    h.xg_row = H.xg_row;
+    h.xs_bytes = H.xg_row * 256 * H.M;
     h.max_segs = H.max_segs;
     h.max_nx = H.max_nx;
     h.records = (int64_t)H.gather.size();
@@ -370,7 +381,8 @@ const PlanHeader* as_plan(const void* plan) {
     if (h->magic != kPassMagic || h->version != kPassVersion) return nullptr;
     if (h->sms < 1 || h->sms > kMaxSms || h->nstages < 0 || h->nstages > LAQ_CHAIN_MAX ||
         (h->bits != 3 && h->bits != 4) || h->rb != record_bytes(h->bits) ||
-        h->xs_bytes < 0 || h->xs_bytes > kMaxXsBytes || h->max_segs < 0 ||
+        h->M < 1 || h->M > kMaxM || h->xg_row < 0 || h->xs_bytes != h->xg_row * 256 * h->M ||
+        h->xs_bytes > kMaxXsBytes || h->max_segs < 0 ||
         h->max_segs > kMaxSegs || h->max_nx < 0 || h->max_nx > kMaxSegs)
         return nullptr;
     return h;
@@ -386,16 +398,20 @@ size_t pass_workspace(const PlanHeader& h) {
 struct PassSmem {
     int xs, sp, seg, tile, xi, slot, zero, bar, flag, total;
 };
+// Regions: the ring (ns slots of 16 records), the X area (xs_bytes) and its (S, P) pair per
+// group, the stage's segments, local tiles and staged X items, the segment partials (mp rows of
+// 16 outputs per segment), a zero block, the ring's mbarriers and the abort flag.
 __host__ __device__ inline PassSmem pass_smem(int rb, int ns, int xs_bytes, int max_segs,
-                                              int max_nx) {
+                                              int max_nx, int mp) {
+    auto a16 = [](int v) { return (v + 15) / 16 * 16; };
     PassSmem m;
     m.xs = (ns * kPRec * rb + 127) / 128 * 128;
     m.sp = m.xs + xs_bytes;
-    m.seg = (m.sp + xs_bytes / 256 * 8 + 15) / 16 * 16;
-    m.tile = m.seg + max_segs * (int)sizeof(Seg);
-    m.xi = m.tile + max_segs * (int)sizeof(LTile);
-    m.slot = m.xi + max_nx * (int)sizeof(XItem);
-    m.zero = m.slot + max_segs * 16 * 4;
+    m.seg = a16(m.sp + xs_bytes / 256 * 8);
+    m.tile = a16(m.seg + max_segs * (int)sizeof(Seg));
+    m.xi = a16(m.tile + max_segs * (int)sizeof(LTile));
+    m.slot = a16(m.xi + max_nx * (int)sizeof(XItem));
+    m.zero = a16(m.slot + max_segs * mp * 16 * 4);
     m.bar = m.zero + 64;
     m.flag = m.bar + 2 * kMaxRing * 8;
     m.total = m.flag + 16;
@@ -548,6 +564,8 @@ struct PassParams {
     const XItem* xi;
     uint32_t* ws;  // [0] status, [1] finished CTAs, [2 + j] stages CTA j has completed
     int nstages, ns, xs_bytes, max_segs, max_nx;
+    int M;       // batch rows (1..4)
+    int xg_row;  // groups of one staged X row
     Exps exps;
 };
 
@@ -596,25 +614,31 @@ __device__ void pass_producer(const PassParams& p, const SmDesc& sd, uint32_t ri
 
 // ---- the consumer warps ------------------------------------------------------------------------
 
-// Stage one entry's X (K fp16) at group xg of the X area: 16-byte chunk ci of the entry lands
-// at xs[16 xg + ci]; the 16 lanes holding a group's chunks sum S_g = sum_k x_k and
-// P_g = sum_k c_k x_k (chunk q of a group holds pairs 4 (q % 4) + w, w < 4, of the record
-// layout) into sp[xg + group].
+// Stage one entry's X (M rows of K fp16) in the X area, whose rows are xg_row groups apart:
+// 16-byte chunk cr of row b lands at xs[16 (b xg_row + xg) + cr]; the 16 lanes holding a
+// group's chunks sum S = sum_k x_k and P = sum_k c_k x_k (chunk q of a group holds pairs
+// 4 (q % 4) + w, w < 4, of the record layout) into sp[b xg_row + xg + group].  K / 8 is a
+// multiple of 16, so the 16 lanes of a group are a half-warp of one row.
 template <int BITS>
-__device__ void pass_stage_x(const XItem& X, uint4* xs, float2* sp, int tid) {
-    const int nch = X.K >> 3;  // a multiple of 16
-    for (int c0 = 0; c0 < nch; c0 += 4 * 512) {
+__device__ void pass_stage_x(const XItem& X, int M, int xg_row, uint4* xs, float2* sp,
+                             int tid) {
+    const int nch = X.K >> 3;  // chunks per row
+    const int total = M * nch;
+    for (int c0 = 0; c0 < total; c0 += 4 * 512) {
         uint4 v[4];
 #pragma unroll
         for (int u = 0; u < 4; ++u) {
             const int ci = c0 + u * 512 + tid;
-            v[u] = ci < nch ? ld_cg16(X.x + 8 * (size_t)ci) : make_uint4(0u, 0u, 0u, 0u);
+            const int b = ci / nch;
+            v[u] = ci < total ? ld_cg16(X.x + (size_t)b * X.K + 8 * (size_t)(ci - b * nch))
+                              : make_uint4(0u, 0u, 0u, 0u);
         }
 #pragma unroll
         for (int u = 0; u < 4; ++u) {
             const int wfirst = c0 + u * 512 + (tid & ~31);  // the warp's first chunk
-            if (wfirst >= nch) break;                       // warp-uniform
+            if (wfirst >= total) break;                     // warp-uniform
             const int ci = wfirst + (tid & 31);
+            const int b = ci / nch, cr = ci - b * nch;
             const uint32_t w4[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
             float sx = 0.f, px = 0.f;
 #pragma unroll
@@ -622,22 +646,26 @@ __device__ void pass_stage_x(const XItem& X, uint4* xs, float2* sp, int tid) {
                 const float2 f = __half22float2(*reinterpret_cast<const __half2*>(&w4[w]));
                 const float pair = f.x + f.y;
                 sx += pair;
-                px = fmaf(row_offset<BITS>((ci & 3) * 4 + w), pair, px);
+                px = fmaf(row_offset<BITS>((cr & 3) * 4 + w), pair, px);
             }
 #pragma unroll
             for (int o = 1; o < 16; o <<= 1) {
                 sx += __shfl_xor_sync(0xffffffffu, sx, o);
                 px += __shfl_xor_sync(0xffffffffu, px, o);
             }
-            if (ci < nch) {
-                xs[16 * X.xg + ci] = v[u];
-                if ((ci & 15) == 0) sp[X.xg + (ci >> 4)] = make_float2(sx, px);
+            if (ci < total) {
+                xs[16 * (b * xg_row + X.xg) + cr] = v[u];
+                if ((cr & 15) == 0)
+                    sp[b * xg_row + X.xg + (cr >> 4)] = make_float2(sx, px);
             }
         }
     }
 }
 
-template <int BITS>
+// MP: the batch rows M rounded up to 1, 2 or 4.  The MMA's 8 columns hold GPA = 8 / MP groups
+// of each of MP batch rows: column col is batch row col / GPA and record col % GPA of a block of
+// GPA records (at M = 1 the 8 columns are 8 groups of the one row).
+template <int BITS, int MP>
 __device__ void pass_consumer(const PassParams& p, uint8_t* smem, const PassSmem& L,
                               uint32_t full_s, uint32_t empty_s, volatile int* abort_flag,
                               int warp, int lane) {
@@ -646,8 +674,11 @@ __device__ void pass_consumer(const PassParams& p, uint8_t* smem, const PassSmem
     constexpr int SLOT = kPRec * RB;
     constexpr int WPL = BITS == 4 ? 8 : 6;
     const int tid = warp * 32 + lane;
+    constexpr int GPA = 8 / MP;  // records per block: groups sharing one accumulator
+    constexpr int LPB = 4 / MP;  // lanes of one output row that hold one batch row's columns
     const int c = lane & 3, R = lane >> 2;
-    const int NS = p.ns;
+    const int bl = R / GPA, gil = R % GPA;  // batch row and block record of MMA column R
+    const int NS = p.ns, M = p.M, XR = p.xg_row;
     uint4* xs = reinterpret_cast<uint4*>(smem + L.xs);
     float2* sp = reinterpret_cast<float2*>(smem + L.sp);
     Seg* segs = reinterpret_cast<Seg*>(smem + L.seg);
@@ -680,7 +711,7 @@ __device__ void pass_consumer(const PassParams& p, uint8_t* smem, const PassSmem
         const int n = dp->n, nr = dp->nr, nt = dp->nt, nx = dp->nx;
         const int k0 = dp->wseg[warp], k1 = dp->wseg[warp + 1];
         if (n > 0) {
-            for (int i = 0; i < nx; ++i) pass_stage_x<BITS>(xitems[i], xs, sp, tid);
+            for (int i = 0; i < nx; ++i) pass_stage_x<BITS>(xitems[i], M, XR, xs, sp, tid);
             cbar();
 
             // This warp's records: the first q + (warp < rem) of the stage's rounds, at
@@ -704,9 +735,11 @@ __device__ void pass_consumer(const PassParams& p, uint8_t* smem, const PassSmem
                 if (r < len) {
                     const uint8_t* rec = ring + (size_t)slot * SLOT + (size_t)warp * RB;
                     const int g = sg.g0 + i;
-                    // B fragments: x of the record's group for the lanes of MMA column gi
-                    // (rows 32c .. 32c + 31 of the group), zeros for the other columns.
-                    const uint4* xsrc = R == gi ? xs + 16 * (sg.xg + g) + 4 * c : zblk;
+                    // B fragments: x of batch row bl of the record's group (rows 32c .. 32c +
+                    // 31 of the group) for the lanes of the MMA columns of block record gi,
+                    // zeros for the other columns.
+                    const uint4* xsrc =
+                        gil == gi && bl < M ? xs + 16 * (bl * XR + sg.xg + g) + 4 * c : zblk;
                     uint32_t B[8][2];
 #pragma unroll
                     for (int qq = 0; qq < 4; ++qq) {
@@ -731,12 +764,14 @@ __device__ void pass_consumer(const PassParams& p, uint8_t* smem, const PassSmem
 #pragma unroll
                     for (int j = 0; j < 8; ++j)
                         mma16816(D[j & 3], a[j][0], a[j][1], a[j][2], a[j][3], B[j][0], B[j][1]);
-                    // The lanes whose accumulator columns include gi keep the record's scale
-                    // and zero pairs of their output rows R, R + 8 (converted in the epilogue).
-                    if (c == (gi >> 1)) {
+                    // The lanes whose accumulator columns 2c, 2c + 1 include block record gi
+                    // keep its scale and zero pairs of their output rows R, R + 8 (converted in
+                    // the epilogue).
+                    const bool u0 = (2 * c) % GPA == gi, u1 = (2 * c + 1) % GPA == gi;
+                    if (u0 || u1) {
                         const uint32_t sr = reinterpret_cast<const uint32_t*>(rec + RBC)[R];
                         const uint32_t zr = reinterpret_cast<const uint16_t*>(rec + RBC + 32)[R];
-                        if (gi & 1) {
+                        if (u1) {
                             sw[1] = sr;
                             zw[1] = zr;
                         } else {
@@ -745,15 +780,17 @@ __device__ void pass_consumer(const PassParams& p, uint8_t* smem, const PassSmem
                         }
                     }
                     ++i;
-                    if (gi == 7 || i == sg.ng) {
+                    if (gi == GPA - 1 || i == sg.ng) {
                         // Block epilogue (Eq. (1)): value v is output row R + 8 (v >> 1) and
-                        // MMA column 2c + (v & 1), the block's record of that index.
+                        // MMA column col = 2c + (v & 1): batch row col / GPA, block record
+                        // col % GPA.
                         const int gb = sg.xg + sg.g0 + i - 1 - gi;  // the block's first group
 #pragma unroll
                         for (int v = 0; v < 4; ++v) {
                             const int col = 2 * c + (v & 1);
-                            if (col <= gi) {
-                                const float2 spv = sp[gb + col];  // (S, P)
+                            const int b = col / GPA, giv = col % GPA;
+                            if (giv <= gi && b < M) {
+                                const float2 spv = sp[b * XR + gb + giv];  // (S, P)
                                 const float dv = (D[0][v] + D[1][v]) + (D[2][v] + D[3][v]);
                                 const float sc = __half2float(__ushort_as_half(
                                     (uint16_t)(sw[v & 1] >> (16 * (v >> 1)))));
@@ -767,16 +804,19 @@ __device__ void pass_consumer(const PassParams& p, uint8_t* smem, const PassSmem
                         ++gi;
                     }
                     if (i == sg.ng) {
-                        // Segment end: the four lanes of an output row hold its two columns'
-                        // partial sums; the slot of segment k gets the 16 outputs.
+                        // Segment end: a lane's two columns belong to one batch row (c / LPB);
+                        // its LPB lanes of the output row add up, and slot (k, b) gets the 16
+                        // outputs of batch row b.
                         float lo = y[0] + y[1], hi = y[2] + y[3];
-                        lo += __shfl_xor_sync(0xffffffffu, lo, 1);
-                        hi += __shfl_xor_sync(0xffffffffu, hi, 1);
-                        lo += __shfl_xor_sync(0xffffffffu, lo, 2);
-                        hi += __shfl_xor_sync(0xffffffffu, hi, 2);
-                        if (c == 0) {
-                            slots[16 * k + R] = lo;
-                            slots[16 * k + R + 8] = hi;
+#pragma unroll
+                        for (int o = 1; o < LPB; o <<= 1) {
+                            lo += __shfl_xor_sync(0xffffffffu, lo, o);
+                            hi += __shfl_xor_sync(0xffffffffu, hi, o);
+                        }
+                        const int b = c / LPB;
+                        if (c % LPB == 0 && b < M) {
+                            slots[16 * (k * MP + b) + R] = lo;
+                            slots[16 * (k * MP + b) + R + 8] = hi;
                         }
 #pragma unroll
                         for (int v = 0; v < 4; ++v) y[v] = 0.f;
@@ -795,12 +835,12 @@ __device__ void pass_consumer(const PassParams& p, uint8_t* smem, const PassSmem
             if (cbar_any(aborted || *abort_flag)) return;
 
             // The SM's tiles of the stage: each output is its segments' slots summed in order.
-            for (int idx = tid; idx < nt * 16; idx += 512) {
-                const LTile t = tiles[idx >> 4];
-                const int col = idx & 15;
+            for (int idx = tid; idx < nt * M * 16; idx += 512) {
+                const int lt = idx / (M * 16), b = (idx >> 4) - lt * M, col = idx & 15;
+                const LTile t = tiles[lt];
                 float acc = 0.f;
-                for (int q = 0; q < t.nslot; ++q) acc += slots[16 * (t.slot0 + q) + col];
-                t.y[col] = __half_as_ushort(__float2half_rn(acc));
+                for (int q = 0; q < t.nslot; ++q) acc += slots[16 * ((t.slot0 + q) * MP + b) + col];
+                t.y[(size_t)b * t.ldy + col] = __half_as_ushort(__float2half_rn(acc));
             }
             cbar();
         }
@@ -808,11 +848,11 @@ __device__ void pass_consumer(const PassParams& p, uint8_t* smem, const PassSmem
     }
 }
 
-template <int BITS>
+template <int BITS, int MP>
 __global__ void __launch_bounds__(kPThreads, 1) pass_kernel(const PassParams p) {
     extern __shared__ __align__(128) uint8_t smem[];
     constexpr int RB = RecordFmt<BITS>::kBytes + kSZ;
-    const PassSmem L = pass_smem(RB, p.ns, p.xs_bytes, p.max_segs, p.max_nx);
+    const PassSmem L = pass_smem(RB, p.ns, p.xs_bytes, p.max_segs, p.max_nx, MP);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const uint32_t base = (uint32_t)__cvta_generic_to_shared(smem);
     const uint32_t full_s = base + (uint32_t)L.bar;
@@ -835,7 +875,7 @@ __global__ void __launch_bounds__(kPThreads, 1) pass_kernel(const PassParams p) 
     if (warp == kPW)
         pass_producer<BITS>(p, sd, base, full_s, empty_s, abort_flag, lane);
     else
-        pass_consumer<BITS>(p, smem, L, full_s, empty_s, abort_flag, warp, lane);
+        pass_consumer<BITS, MP>(p, smem, L, full_s, empty_s, abort_flag, warp, lane);
     __syncthreads();
 
     // The last CTA to finish (every other one has made its last flag read) zeroes the flags
@@ -879,7 +919,13 @@ __global__ void pass_gather_kernel(const GatherRec* __restrict__ gt,
     }
 }
 
-std::atomic<int> g_pass_attr[2];  // dynamic shared memory granted to pass_kernel<3>, <4>
+std::atomic<int> g_pass_attr[2][3];  // shared memory granted to pass_kernel<bits, 1 | 2 | 4>
+
+template <int BITS>
+const void* pick_pass(int mp) {
+    return mp == 1 ? (const void*)pass_kernel<BITS, 1>
+                   : mp == 2 ? (const void*)pass_kernel<BITS, 2> : (const void*)pass_kernel<BITS, 4>;
+}
 
 int device_sms(int* sms, int* smem_optin) {
     int dev = 0;
@@ -979,11 +1025,13 @@ laq_status laq_pass_run(const void* plan, const void* device, void* workspace,
     if (device_sms(&sms, &optin) != 0) return LAQ_ERR_CUDA;
     if (sms != h->sms) return LAQ_ERR_CONFIG;  // planned for another SM count
     // ring depth: as many 16-record slots as the shared memory left over holds
+    const int mp = h->M == 1 ? 1 : h->M == 2 ? 2 : 4;
     int ns = kMaxRing;
-    while (ns >= 2 && pass_smem(h->rb, ns, h->xs_bytes, h->max_segs, h->max_nx).total > optin)
+    while (ns >= 2 &&
+           pass_smem(h->rb, ns, h->xs_bytes, h->max_segs, h->max_nx, mp).total > optin)
         --ns;
     if (ns < 2) return LAQ_ERR_SHAPE;
-    const PassSmem L = pass_smem(h->rb, ns, h->xs_bytes, h->max_segs, h->max_nx);
+    const PassSmem L = pass_smem(h->rb, ns, h->xs_bytes, h->max_segs, h->max_nx, mp);
 
     const uint8_t* dev = static_cast<const uint8_t*>(device);
     const uint8_t* t = dev + h->stream_bytes;
@@ -1001,12 +1049,14 @@ laq_status laq_pass_run(const void* plan, const void* device, void* workspace,
     P.xs_bytes = h->xs_bytes;
     P.max_segs = h->max_segs;
     P.max_nx = h->max_nx;
+    P.M = h->M;
+    P.xg_row = h->xg_row;
     P.exps = exps_for(h->bits);
 
-    const void* fn = h->bits == 4 ? (const void*)pass_kernel<4> : (const void*)pass_kernel<3>;
+    const void* fn = h->bits == 4 ? pick_pass<4>(mp) : pick_pass<3>(mp);
     // First call with this much shared memory (before any stream capture): raise the kernel's
     // limit and check that a CTA fits an SM, as the cooperative launch requires.
-    std::atomic<int>& granted = g_pass_attr[h->bits == 4];
+    std::atomic<int>& granted = g_pass_attr[h->bits == 4][mp == 1 ? 0 : mp == 2 ? 1 : 2];
     if (granted.load() < L.total) {
         if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, L.total) !=
             cudaSuccess)

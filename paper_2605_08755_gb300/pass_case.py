@@ -4,7 +4,7 @@
 
 Builds the Qwen3-4B-shaped pass (36 layers, synthetic weights) in one of its forms
 (``graph_252``, ``graph_fused``, ``chain_252``, ``chain_fused``, and the planned pass over
-per-SM weight streams, ``planned_252`` and ``planned_fused``, M = 1), captures it into a CUDA
+per-SM weight streams, ``planned_252`` and ``planned_fused``, M <= 4), captures it into a CUDA
 graph (the capture is preceded by one eager run of the pass), replays the graph ``replays``
 times and prints the mean device time per replay.  Under a profiler, the first replay's kernels
 follow the eager run's: for a graph form, ``-k regex:gemm_kernel -s L -c L`` with L = the

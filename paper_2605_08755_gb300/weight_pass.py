@@ -70,14 +70,14 @@ class WeightPass:
     the projection before it (k and v after q, up after gate), so each layer has the four
     dependency points q|k|v -> o -> gate|up -> down -> next layer.
 
-    With ``planned`` (M = 1), the same entries run through ``laq_pass_run`` after
+    With ``planned`` (M <= 4), the same entries run through ``laq_pass_run`` after
     ``laq_pass_prepare`` has laid their weights out as per-SM streams (``_lib.PassPlan``)."""
 
     def __init__(self, model="qwen3-4b", bits=3, M=1, layers=inputs.LAYERS, seed=0,
                  outliers=False, device="cuda", pdl=True, fuse=False, chain=False,
                  planned=False):
-        if planned and M != 1:
-            raise ValueError("the planned pass runs M = 1 only")
+        if planned and not 1 <= M <= 4:
+            raise ValueError("the planned pass runs M = 1..4")
         self.model, self.bits, self.M, self.layers = model, bits, M, layers
         self.seed, self.outliers, self.fuse, self.chain = seed, outliers, fuse, chain
         self.planned = planned

@@ -34,24 +34,25 @@ def run(entries):
 
 
 @pytest.mark.parametrize("bits", [3, 4])
+@pytest.mark.parametrize("M", [1, 2, 3, 4])
 @pytest.mark.parametrize("K,N", [(128, 16), (384, 48), (1024, 1024), (2560, 1040),
-                                 (9728, 2560), (24576, 32)])
-def test_single_entry(bits, K, N):
+                                 (9728, 2560), (13312, 32)])
+def test_single_entry(bits, M, K, N):
     lin = Lin(K, N, bits, seed=K + N + bits)
-    X = inputs.activations(1, K, seed=K)
-    Y = nan_like(1, N)
+    X = inputs.activations(M, K, seed=K + M)
+    Y = nan_like(M, N)
     run([(torch.from_numpy(X).cuda(), lin.packed, lin.s, lin.z, bits, Y, 1)])
     check_y(Y, X, lin)
 
 
-@pytest.mark.parametrize("bits", [3, 4])
-def test_dependencies_and_stages(bits):
+@pytest.mark.parametrize("bits,M", [(3, 1), (4, 1), (3, 2), (4, 4)])
+def test_dependencies_and_stages(bits, M):
     """e0 | e1 e2 (both read Y0) | e3 (reads Y1) | e4 (reads Y3) e5 (reads X0)."""
     dims = [(512, 1024), (1024, 3200), (1024, 16), (3200, 768), (768, 128), (512, 2560)]
     lins = [Lin(K, N, bits, seed=100 + i) for i, (K, N) in enumerate(dims)]
-    X0 = inputs.activations(1, 512, seed=7)
+    X0 = inputs.activations(M, 512, seed=7)
     X0d = torch.from_numpy(X0).cuda()
-    Ys = [nan_like(1, N) for _, N in dims]
+    Ys = [nan_like(M, N) for _, N in dims]
     src = [X0d, Ys[0], Ys[0], Ys[1], Ys[3], X0d]
     wait = [1, 1, 0, 1, 1, 0]
     run([(src[i], lins[i].packed, lins[i].s, lins[i].z, bits, Ys[i], wait[i])
@@ -168,9 +169,10 @@ def test_longest_chain():
         check_y(Ys[i], Xs[i], lins[i % 3])
 
 
-@pytest.mark.parametrize("bits,fuse", [(3, True), (4, True), (3, False)])
-def test_qwen3_4b_pass_planned(bits, fuse):
-    wp = WeightPass(model="qwen3-4b", bits=bits, M=1, fuse=fuse, planned=True)
+@pytest.mark.parametrize("bits,fuse,M", [(3, True, 1), (4, True, 1), (3, False, 1),
+                                         (3, True, 2), (4, True, 4)])
+def test_qwen3_4b_pass_planned(bits, fuse, M):
+    wp = WeightPass(model="qwen3-4b", bits=bits, M=M, fuse=fuse, planned=True)
     assert wp.launches == 1
     g = wp.capture()
     wp.Ybuf.fill_(float("nan"))

@@ -12,7 +12,8 @@ from oracle import c_oracle as co
 from paper_2605_08755_gb300 import _lib, inputs
 
 HDR = np.dtype([("magic", "<u4"), ("version", "<i4"), ("count", "<i4"), ("nstages", "<i4"),
-                ("sms", "<i4"), ("bits", "<i4"), ("rb", "<i4"), ("xs_bytes", "<i4"),
+                ("sms", "<i4"), ("bits", "<i4"), ("rb", "<i4"), ("M", "<i4"),
+                ("xg_row", "<i4"), ("xs_bytes", "<i4"),
                 ("max_segs", "<i4"), ("max_nx", "<i4"), ("records", "<i8"), ("rounds", "<i8"),
                 ("segs", "<i8"), ("ltiles", "<i8"), ("xitems", "<i8"), ("tables_h", "<i8"),
                 ("tables_bytes", "<i8"), ("stream_bytes", "<i8"), ("o_sm", "<i8"),
@@ -25,7 +26,8 @@ STAGE = np.dtype([("n", "<i4"), ("nr", "<i4"), ("seg0", "<i4"), ("tile0", "<i4")
                   ("wseg", "u1", (17,)), ("pad2", "u1", (3,))])
 SEG = np.dtype([("e", "<i4"), ("t", "<i4"), ("g0", "<i2"), ("ng", "<i2"), ("xg", "<i2"),
                 ("lt", "<i2")])
-TILE = np.dtype([("y", "<u8"), ("slot0", "<i4"), ("nslot", "<i4")])
+TILE = np.dtype([("y", "<u8"), ("slot0", "<i4"), ("nslot", "<i4"), ("ldy", "<i4"),
+                 ("pad", "<i4")])
 XIT = np.dtype([("x", "<u8"), ("K", "<i4"), ("xg", "<i4")])
 PREP = np.dtype([("packed", "<u8"), ("s", "<u8"), ("z", "<u8"), ("N", "<i4"), ("G", "<i4")])
 GATHER = np.dtype([("e", "<i4"), ("rid", "<i4")])
@@ -89,10 +91,11 @@ def warp_records(tb, seg0, wseg, w):
     return out
 
 
-def check_plan(shapes, P, bits, plan, dev_bytes):
+def check_plan(shapes, P, bits, plan, dev_bytes, M=1):
     """Every promise of the plan, checked from its tables."""
     tb = parse(plan)
     h = tb["h"]
+    assert h["M"] == M
     S = len(stage_starts(shapes))
     starts = stage_starts(shapes) + [len(shapes)]
     rb = (1024 if bits == 4 else 768) + 48
@@ -150,7 +153,7 @@ def check_plan(shapes, P, bits, plan, dev_bytes):
             assert int(d["nt"]) == len(tiles)
             for lt, (e, t) in enumerate(tiles):
                 ti = tb["tile"][int(d["tile0"]) + lt]
-                assert ti["y"] == addr(e, "Y") + 32 * t
+                assert ti["y"] == addr(e, "Y") + 32 * t and ti["ldy"] == shapes[e][1]
                 ks = sorted({r[3] for r in recs if r[:2] == (e, t)})
                 assert ks == list(range(int(ti["slot0"]), int(ti["slot0"] + ti["nslot"])))
                 assert all(int(tb["seg"][seg0 + k]["lt"]) == lt for k in ks)
@@ -162,7 +165,7 @@ def check_plan(shapes, P, bits, plan, dev_bytes):
             assert list(xi["xg"]) == list(np.cumsum([0] + [G[e] for e in ents])[:-1])
             for (e, t, g, k, xg) in recs:
                 assert xg == int(xi["xg"][ents.index(e)])
-            xs_max = max(xs_max, 256 * sum(G[e] for e in ents))
+            xs_max = max(xs_max, sum(G[e] for e in ents))
             nx_max = max(nx_max, len(ents))
             # the stream: round r, position w holds warp w's r-th record
             for r in range(nr):
@@ -174,7 +177,8 @@ def check_plan(shapes, P, bits, plan, dev_bytes):
         assert r_at == len(rnds)
     assert rec == len(gat)
     assert len(owner) == sum(T)
-    assert (h["xs_bytes"], h["max_segs"], h["max_nx"]) == (xs_max, segs_max, nx_max)
+    assert (h["xg_row"], h["max_segs"], h["max_nx"]) == (xs_max, segs_max, nx_max)
+    assert h["xs_bytes"] == 256 * M * xs_max
     # balance: an SM's share of a stage exceeds the even share by less than one tile
     for s in range(S):
         n = [int(tb["stage"][j * S + s]["n"]) for j in range(P)]
@@ -196,17 +200,21 @@ def row_offsets(bits):
 
 def emulate(tb, shapes, bits, data):
     """Y of every entry, computed by walking the plan as the kernel does, in float64.
-    ``data[e]`` = (x [K] float64, codes [K, N], s [G, N] float64, z [G, N]).  Each record's codes,
-    scales and zeros come from the stream record the gather table puts at the warp's position of
-    its round; its x from the warp's own segment; the block epilogue uses the kernel's indices
-    (the block's first group gb, one MMA column per record) and Eq. (1) in the kernel's form
-    y += s (D - P - z S) with D = sum_k (c_k + q_k) x_k."""
+    ``data[e]`` = (x [M, K] float64, codes [K, N], s [G, N] float64, z [G, N]).  Each record's
+    codes, scales and zeros come from the stream record the gather table puts at the warp's
+    position of its round; its x from the warp's own segment, in the X area whose rows are
+    xg_row groups apart; blocks hold 8 / MP records (MP = M rounded up to 1, 2, 4) and the block
+    epilogue uses the kernel's indices (the block's first group gb, MMA column = batch row b and
+    block record giv) and Eq. (1) in the kernel's form y += s (D - P - z S) with
+    D = sum_k (c_k + q_k) x_k; slots hold one row of 16 outputs per (segment, batch row)."""
     h = tb["h"]
-    P, S = int(h["sms"]), int(h["nstages"])
+    P, S, M, XR = int(h["sms"]), int(h["nstages"]), int(h["M"]), int(h["xg_row"])
+    MP = 1 if M == 1 else 2 if M == 2 else 4
+    GPA = 8 // MP
     G = [K // 128 for K, _, _ in shapes]
     c = row_offsets(bits)
     x_of = {addr(e, "X"): e for e in range(len(shapes))}
-    Y = [np.full(N, np.nan) for _, N, _ in shapes]
+    Y = [np.full((M, N), np.nan) for _, N, _ in shapes]
     for j in range(P):
         base = int(tb["sm"][j]["rec0"])
         for s in range(S):
@@ -214,20 +222,20 @@ def emulate(tb, shapes, bits, data):
             n = int(d["n"])
             if n == 0:
                 continue
-            xs = np.full(int(h["xs_bytes"]) // 2, np.nan)
+            xs = np.full((M, XR * 128), np.nan)
             for it in tb["x"][int(d["x0"]):int(d["x0"] + d["nx"])]:
                 e = x_of[int(it["x"])]
-                xs[128 * int(it["xg"]):128 * int(it["xg"]) + int(it["K"])] = data[e][0]
-            xg_all = xs.reshape(-1, 128)
-            sp = np.stack([xg_all.sum(1), xg_all @ c], 1)  # (S_g, P_g) per staged group
-            slots = np.full((int(d["nseg"]), 16), np.nan)
+                xs[:, 128 * int(it["xg"]):128 * int(it["xg"]) + int(it["K"])] = data[e][0]
+            xg3 = xs.reshape(M, XR, 128)
+            sp = np.stack([xg3.sum(2), xg3 @ c], 2)  # (S, P) per (row, staged group)
+            slots = np.full((int(d["nseg"]), MP, 16), np.nan)
             seg0, wseg = int(d["seg0"]), d["wseg"]
             for w in range(16):
                 r = 0
                 for k in range(int(wseg[w]), int(wseg[w + 1])):
                     sg = tb["seg"][seg0 + k]
                     ng, g0, xg = int(sg["ng"]), int(sg["g0"]), int(sg["xg"])
-                    y = np.zeros(16)
+                    y = np.zeros((M, 16))
                     i = gi = 0
                     Dcol, scol, zcol = {}, {}, {}
                     while i < ng:
@@ -236,27 +244,30 @@ def emulate(tb, shapes, bits, data):
                         t, g = divmod(rid, G[e])
                         codes, sc, zc = data[e][1], data[e][2], data[e][3]
                         q = codes[128 * g:128 * g + 128, 16 * t:16 * t + 16].astype(np.float64)
-                        x = xs[128 * (xg + g0 + i):128 * (xg + g0 + i) + 128]
-                        Dcol[gi] = (c[:, None] + q).T @ x
+                        for b in range(M):  # MMA column b * GPA + gi
+                            x = xs[b, 128 * (xg + g0 + i):128 * (xg + g0 + i) + 128]
+                            Dcol[b, gi] = (c[:, None] + q).T @ x
                         scol[gi] = sc[g, 16 * t:16 * t + 16]
                         zcol[gi] = zc[g, 16 * t:16 * t + 16].astype(np.float64)
                         i += 1
                         r += 1
-                        if gi == 7 or i == ng:
+                        if gi == GPA - 1 or i == ng:
                             gb = xg + g0 + i - 1 - gi
-                            for col in range(gi + 1):
-                                S_, P_ = sp[gb + col]
-                                y += scol[col] * (Dcol[col] - P_ - zcol[col] * S_)
+                            for b in range(M):
+                                for giv in range(gi + 1):
+                                    S_, P_ = sp[b, gb + giv]
+                                    y[b] += scol[giv] * (Dcol[b, giv] - P_ - zcol[giv] * S_)
                             gi = 0
                         else:
                             gi += 1
-                    slots[k] = y
+                    slots[k, :M] = y
             for ti in tb["tile"][int(d["tile0"]):int(d["tile0"] + d["nt"])]:
                 e = next(e for e in range(len(shapes))
                          if addr(e, "Y") <= int(ti["y"]) < addr(e, "Y") + 2 * shapes[e][1])
+                assert int(ti["ldy"]) == shapes[e][1]
                 t = (int(ti["y"]) - addr(e, "Y")) // 32
                 k0, nk = int(ti["slot0"]), int(ti["nslot"])
-                Y[e][16 * t:16 * t + 16] = slots[k0:k0 + nk].sum(0)
+                Y[e][:, 16 * t:16 * t + 16] = slots[k0:k0 + nk, :M].sum(0)
             base += n
     return Y
 
@@ -265,18 +276,19 @@ SMALL = [(256, 48, 0), (384, 32, 0), (128, 16, 1), (1024, 160, 1), (256, 64, 0),
          (128, 512, 1), (1024, 32, 1), (2048, 16, 0)]
 
 
-@pytest.mark.parametrize("bits,P", [(3, 5), (4, 7), (3, 1), (4, 3)])
-def test_plan_emulation_reproduces_the_oracle(L, bits, P):
-    arr = fake_entries(SMALL, bits)
+@pytest.mark.parametrize("bits,P,M", [(3, 5, 1), (4, 7, 1), (3, 1, 1), (4, 3, 1), (3, 5, 2),
+                                      (4, 3, 3), (3, 7, 4)])
+def test_plan_emulation_reproduces_the_oracle(L, bits, P, M):
+    arr = fake_entries(SMALL, bits, M)
     plan, dev = _lib.pass_plan(arr, len(SMALL), P)
-    tb = check_plan(SMALL, P, bits, plan, dev)
+    tb = check_plan(SMALL, P, bits, plan, dev, M)
     data, refs = [], []
     for e, (K, N, _) in enumerate(SMALL):
         W = inputs.weights(K, N, seed=300 + e)
         codes, s, z = co.quantize_rtn(W, bits)
-        x = inputs.activations(1, K, seed=400 + e)
-        data.append((x[0].astype(np.float64), codes, s.astype(np.float64), z))
-        refs.append(co.gemm(x, codes, s, z)[0])
+        x = inputs.activations(M, K, seed=400 + e)
+        data.append((x.astype(np.float64), codes, s.astype(np.float64), z))
+        refs.append(co.gemm(x, codes, s, z))
     Y = emulate(tb, SMALL, bits, data)
     for e in range(len(SMALL)):
         assert np.all(np.isfinite(Y[e])), e
@@ -341,12 +353,19 @@ def test_plan_rejects_invalid_entries(L):
     arr = fake_entries(ok)
     arr[0].bits = 5
     assert sizes(L, arr, 2, 4) == 2
-    assert sizes(L, fake_entries(ok, M=2), 2, 4) == 6            # M != 1
+    assert sizes(L, fake_entries(ok, M=4), 2, 4) == 0
+    assert sizes(L, fake_entries(ok, M=5), 2, 4) == 6            # M outside 1..4
+    assert sizes(L, fake_entries(ok, M=0), 2, 4) == 6
+    arr = fake_entries(ok)
+    arr[1].M = 2
+    assert sizes(L, arr, 2, 4) == 6                              # mixed M
+    assert sizes(L, fake_entries([(13312, 16, 0)], M=4), 1, 4) == 0   # 4 x 13312 x 2 = 104 KB
+    assert sizes(L, fake_entries([(13440, 16, 0)], M=4), 1, 4) == 4
     assert sizes(L, fake_entries([(100, 16, 0)]), 1, 4) == 4     # K % 128
     assert sizes(L, fake_entries([(128, 24, 0)]), 1, 4) == 4     # N % 16
     assert sizes(L, fake_entries([(0, 16, 0)]), 1, 4) == 4
-    assert sizes(L, fake_entries([(24576, 16, 0)]), 1, 4) == 0   # largest K
-    assert sizes(L, fake_entries([(24576 + 128, 16, 0)]), 1, 4) == 4
+    assert sizes(L, fake_entries([(53248, 16, 0)]), 1, 4) == 0   # largest K at M = 1
+    assert sizes(L, fake_entries([(53248 + 128, 16, 0)]), 1, 4) == 4
     assert sizes(L, fake_entries(ok), 2, 0) == 4                 # no SMs
     assert sizes(L, fake_entries(ok), 2, 1025) == 4
     assert sizes(L, fake_entries([(128, 16, 0)] * 385), 385, 4) == 4
@@ -358,7 +377,7 @@ def test_plan_rejects_invalid_entries(L):
     arr[0].s = arr[0].s + 2
     assert sizes(L, arr, 2, 4) == 5                              # misaligned
     # two entries of one stage whose X together exceed the staging area on one SM
-    assert sizes(L, fake_entries([(16384, 16, 0), (16384, 16, 0)]), 2, 1) == 4
+    assert sizes(L, fake_entries([(32768, 16, 0), (32768, 16, 0)]), 2, 1) == 4
     pb = ctypes.c_size_t(0)
     assert int(L.laq_pass_plan_sizes(fake_entries(ok), 2, 4, None, ctypes.byref(pb))) == 1
 
