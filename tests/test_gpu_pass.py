@@ -201,3 +201,40 @@ def test_qwen3_8b_fused_pass_planned():
     torch.cuda.synchronize()
     assert wp.plan.status() == 0
     _sampled(wp, layers={0, 35})
+
+
+@pytest.mark.parametrize("bits,M", [(3, 1), (4, 2)])
+def test_prepared_buffer_bit_exact(bits, M):
+    """laq_pass_prepare's output byte for byte: every stream record is its entry's packed record
+    followed by the scale/zero row pairs of its (group, tile), in the plan's order, and the
+    tables are the plan's."""
+    from tests.test_pass_lanes import stream_sz
+    from tests.test_pass_plan import parse
+    dims = [(384, 48), (1024, 160), (256, 16)]
+    lins = [Lin(K, N, bits, seed=40 + i) for i, (K, N) in enumerate(dims)]
+    Xs = [torch.from_numpy(inputs.activations(M, K, seed=i)).cuda() for i, (K, _) in enumerate(dims)]
+    Ys = [nan_like(M, N) for _, N in dims]
+    plan = _lib.PassPlan([(Xs[i], lins[i].packed, lins[i].s, lins[i].z, bits, Ys[i], i % 2)
+                          for i in range(3)], "cuda")
+    torch.cuda.synchronize()
+    tb = parse(plan.plan)
+    h = tb["h"]
+    buf = plan.buffer.cpu().numpy()
+    rb, rbc = int(h["rb"]), int(h["rb"]) - 48
+    host = np.frombuffer(plan.plan, dtype=np.uint8)
+    tables = host[int(h["tables_h"]):int(h["tables_h"] + h["tables_bytes"])]
+    s0 = int(h["stream_bytes"])
+    assert np.array_equal(buf[s0:s0 + tables.size], tables)
+    packed = [l.packed.cpu().numpy() for l in lins]
+    s16 = [l.s.cpu().numpy().view(np.uint16) for l in lins]
+    z8 = [l.z.cpu().numpy() for l in lins]
+    for i, gr in enumerate(tb["gather"]):
+        e, rid = int(gr["e"]), int(gr["rid"])
+        G = dims[e][0] // 128
+        t, g = divmod(rid, G)
+        rec = buf[i * rb:(i + 1) * rb]
+        assert np.array_equal(rec[:rbc], packed[e][rid * rbc:(rid + 1) * rbc]), i
+        sw, zw = stream_sz(s16[e][g, 16 * t:16 * t + 16].view(np.float16),
+                           z8[e][g, 16 * t:16 * t + 16])
+        assert list(rec[rbc:rbc + 32].view("<u4")) == sw, i
+        assert list(rec[rbc + 32:rbc + 48].view("<u2")) == zw, i
