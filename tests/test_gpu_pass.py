@@ -212,7 +212,8 @@ def test_prepared_buffer_bit_exact(bits, M):
     from tests.test_pass_plan import parse
     dims = [(384, 48), (1024, 160), (256, 16)]
     lins = [Lin(K, N, bits, seed=40 + i) for i, (K, N) in enumerate(dims)]
-    Xs = [torch.from_numpy(inputs.activations(M, K, seed=i)).cuda() for i, (K, _) in enumerate(dims)]
+    Xs = [torch.from_numpy(inputs.activations(M, K, seed=i)).cuda()
+          for i, (K, _) in enumerate(dims)]
     Ys = [nan_like(M, N) for _, N in dims]
     plan = _lib.PassPlan([(Xs[i], lins[i].packed, lins[i].s, lins[i].z, bits, Ys[i], i % 2)
                           for i in range(3)], "cuda")
