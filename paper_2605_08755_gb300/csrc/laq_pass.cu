@@ -186,9 +186,12 @@ laq_status plan_pass(const laq_gemv* g, int32_t count, int32_t P, HostPlan& H) {
     H.nstages = S;
     start.push_back(count);
 
-    // Whole tiles to SMs, in order: a tile goes to the SM whose equal share of the stage's
-    // records holds the tile's middle record, so SM shares are contiguous tile ranges and
-    // differ from the mean by less than one tile.  first[s][j] = SM j's first stage tile.
+    // Whole tiles to shares, in order: a tile goes to the share whose equal part of the stage's
+    // records holds the tile's middle record, so shares are contiguous tile ranges and differ
+    // from the mean by less than one tile.  first[s][v] = share v's first stage tile.  SM j
+    // takes share (j + 41 s) mod P of stage s: the shares that hold one tile more than the
+    // others fall on other SMs from stage to stage, so no SM streams more than its part of the
+    // whole pass.
     std::vector<std::vector<int64_t>> first(S);
     for (int s = 0; s < S; ++s) {
         int64_t tiles = 0, W = 0;
@@ -224,7 +227,8 @@ laq_status plan_pass(const laq_gemv* g, int32_t count, int32_t P, HostPlan& H) {
             // the SM's tiles of the stage
             std::vector<TileRef> tl;
             {
-                int64_t ta = first[s][(size_t)j], tb = first[s][(size_t)j + 1], base = 0;
+                const size_t v = (size_t)(((int64_t)j + 41 * (int64_t)s) % P);
+                int64_t ta = first[s][v], tb = first[s][v + 1], base = 0;
                 for (int e = start[s]; e < start[s + 1] && ta < tb; ++e) {
                     const int64_t T = g[e].N / 16;
                     for (; ta < tb && ta < base + T; ++ta)
