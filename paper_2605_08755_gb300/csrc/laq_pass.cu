@@ -7,9 +7,10 @@
 // on the host, when the chain is planned:
 //
 //  * Plan (host only).  The chain is cut into stages at the entries that wait for their
-//    predecessors.  Each stage's 16-column tiles are dealt to the SMs in order as whole tiles,
-//    balanced by records (tile x group of 128 rows), so no output tile is split between SMs and
-//    no cross-SM reduction sits on the critical path.  An SM's records of a stage are cut into
+//    predecessors.  Each stage's 16-column tiles are dealt in order, as whole tiles, to shares
+//    balanced by records (tile x group of 128 rows), and the shares rotated over the SMs from
+//    stage to stage, so no output tile is split between SMs, no cross-SM reduction sits on the
+//    critical path, and every SM streams an equal part of the pass.  An SM's records of a stage are cut into
 //    16 contiguous warp shares that differ by at most one record.  The SM's records, all
 //    stages in order, form its stream, laid out in rounds: round r holds the r-th record of
 //    every warp that has one, warp w's at position w.
