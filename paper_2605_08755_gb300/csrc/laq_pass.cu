@@ -430,15 +430,13 @@ __device__ __forceinline__ unsigned long long gtimer() {
     asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
     return t;
 }
-__device__ __forceinline__ uint32_t ld_acq(const uint32_t* p) {
-    uint32_t v;
-    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
-    return v;
-}
 __device__ __forceinline__ uint32_t ld_rlx(const uint32_t* p) {
     uint32_t v;
     asm volatile("ld.relaxed.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
     return v;
+}
+__device__ __forceinline__ void fence_acq_rel_gpu() {
+    asm volatile("fence.acq_rel.gpu;" ::: "memory");
 }
 __device__ __forceinline__ void st_rel(uint32_t* p, uint32_t v) {
     asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
@@ -537,23 +535,37 @@ __device__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort_fla
     return false;
 }
 
-// One warp waits until every CTA's completed-stage flag (flags[0 .. n)) is >= target, each
-// lane reading every 32nd flag with acquire loads, so a poll is one round trip to L2 and no two
-// CTAs ever write the same word.  Returns the same answer in every lane: false when the status
-// word already holds an error, or after about a second (then LAQ_ERR_TIMEOUT is recorded).
+// One warp waits until every CTA's completed-stage flag (flags[0 .. n)) is >= target.  Each
+// lane reads every 32nd flag with relaxed loads that are all in flight at once (no load waits
+// for another), so a poll costs one round trip to L2 and no two CTAs ever write the same word;
+// once every flag is seen, one acquire fence orders what the warp's CTA reads next after the
+// releases it observed.  Returns the same answer in every lane: false when the status word holds
+// an error (checked every 16th poll), or after about a second (then LAQ_ERR_TIMEOUT is
+// recorded).
 __device__ bool wait_flags(const uint32_t* flags, int n, uint32_t target, uint32_t* status,
                            int lane) {
     const unsigned long long t0 = gtimer();
     for (int spin = 0; spin < kWaitSpins; ++spin) {
-        if ((spin & 31) == 0) {
-            const uint32_t st = lane == 0 ? ld_rlx(status) : 0u;
-            if (__shfl_sync(0xffffffffu, st, 0) != 0u) return false;
-            const bool late = lane == 0 && spin > 0 && gtimer() - t0 > kWaitNs;
-            if (__shfl_sync(0xffffffffu, (int)late, 0)) break;
+        uint32_t v[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+            const int j = lane + 32 * u;
+            v[u] = j < n ? ld_rlx(flags + j) : target;
         }
         bool ok = true;
-        for (int j = lane; j < n; j += 32) ok = ok && ld_acq(flags + j) >= target;
-        if (__all_sync(0xffffffffu, ok)) return true;
+#pragma unroll
+        for (int u = 0; u < 8; ++u) ok &= v[u] >= target;
+        for (int j = lane + 256; j < n; j += 32) ok &= ld_rlx(flags + j) >= target;
+        if (__all_sync(0xffffffffu, ok)) {
+            fence_acq_rel_gpu();
+            return true;
+        }
+        if ((spin & 15) == 15) {
+            const uint32_t st = lane == 0 ? ld_rlx(status) : 0u;
+            if (__shfl_sync(0xffffffffu, st, 0) != 0u) return false;
+            const bool late = lane == 0 && gtimer() - t0 > kWaitNs;
+            if (__shfl_sync(0xffffffffu, (int)late, 0)) break;
+        }
     }
     if (lane == 0) record_timeout(status);
     return false;
@@ -869,7 +881,8 @@ __global__ void __launch_bounds__(kPThreads, 1) pass_kernel(const PassParams p) 
             mbar_init(full_s + 8u * i, 1u);
             mbar_init(empty_s + 8u * i, (uint32_t)kPW);
         }
-        *abort_flag = 0;
+        // an error recorded by an earlier call: the call does nothing
+        *abort_flag = ld_rlx(p.ws) != 0u ? 1 : 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     if (threadIdx.x < 4)
@@ -877,7 +890,9 @@ __global__ void __launch_bounds__(kPThreads, 1) pass_kernel(const PassParams p) 
     __syncthreads();
 
     const SmDesc sd = p.sm[blockIdx.x];
-    if (warp == kPW)
+    if (*abort_flag) {
+        // no copy is issued, no stage runs, and the workspace stays as it is
+    } else if (warp == kPW)
         pass_producer<BITS>(p, sd, base, full_s, empty_s, abort_flag, lane);
     else
         pass_consumer<BITS, MP>(p, smem, L, full_s, empty_s, abort_flag, warp, lane);
