@@ -231,12 +231,16 @@ laq_status laq_gemm_chain(const laq_gemv *gemvs, int32_t count, void *workspace,
  * Same entries, results and restrictions as laq_gemm_chain.  The workspace lives in a scratch
  * array inside the library (a static device array of 68,352 bytes, enough for LAQ_CHAIN_MAX
  * entries), held by every GPU that loads the library until the process exits.  Nothing is
- * allocated: each call clears the counters and flags it uses (cudaMemsetAsync on `stream`)
- * and launches.
+ * allocated: once every argument has passed its checks, each call clears the counters and
+ * flags it uses (cudaMemsetAsync on `stream`) and launches; a call rejected by a check
+ * enqueues nothing.
+ *   count < 0              -> LAQ_ERR_SHAPE (as laq_gemm_chain)
  *   count > LAQ_CHAIN_MAX  -> LAQ_ERR_WORKSPACE (the scratch holds no more).
  * The first call on each device looks up the scratch array's device address (and, like every
  * first call of a kernel variant, sets its shared-memory limit): make it before any stream
- * capture.  All calls share the one array, so calls whose executions overlap on the GPU (other
+ * capture.  The address belongs to the CUDA context it was looked up in; after
+ * cudaDeviceReset the next call looks it up again in the new context (that call, too, should
+ * come before any capture).  All calls share the one array, so calls whose executions overlap on the GPU (other
  * streams, or other host threads) race and give undefined results; serialize them.  A
  * device-side timeout is not reported here (laq_gemm_chain's workspace status word is the way
  * to observe one).

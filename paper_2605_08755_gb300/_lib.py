@@ -287,23 +287,32 @@ class PassPlan:
     """The entries of a ``Chain`` planned for laq_pass_run on ``device``: the host plan, the
     prepared device buffer (per-SM weight streams and tables) and a zeroed workspace.  The
     entries' X and Y tensors are kept alive; their packed weights are no longer read once
-    ``prepare`` has run on the stream."""
+    ``prepare`` has run on the stream.  laq_pass_prepare and laq_pass_run work on the current
+    device, so both calls are made with ``device`` current (and, without ``stream``, on that
+    device's current stream)."""
 
     def __init__(self, entries, device, stream=None):
         import torch
         self.chain = Chain(entries)
         self.device = torch.device(device)
+        if self.device.index is None:
+            self.device = torch.device("cuda", torch.cuda.current_device())
         sms = torch.cuda.get_device_properties(self.device).multi_processor_count
         self.plan, dev_bytes = pass_plan(self.chain.array, self.chain.count, sms)
         self.buffer = torch.empty((max(dev_bytes, 256),), dtype=torch.uint8, device=self.device)
         self.ws = torch.zeros((max(256, int(lib().laq_pass_workspace_bytes(self.plan))),),
                               dtype=torch.uint8, device=self.device)
-        _check(lib().laq_pass_prepare(self.plan, _ptr(self.buffer), self.buffer.numel(),
-                                      _stream(stream)), "laq_pass_prepare")
+        with torch.cuda.device(self.device):
+            st = stream if stream is not None else torch.cuda.current_stream(self.device)
+            _check(lib().laq_pass_prepare(self.plan, _ptr(self.buffer), self.buffer.numel(),
+                                          _stream(st)), "laq_pass_prepare")
 
     def run(self, stream=None):
-        _check(lib().laq_pass_run(self.plan, _ptr(self.buffer), _ptr(self.ws), self.ws.numel(),
-                                  _stream(stream)), "laq_pass_run")
+        import torch
+        with torch.cuda.device(self.device):
+            st = stream if stream is not None else torch.cuda.current_stream(self.device)
+            _check(lib().laq_pass_run(self.plan, _ptr(self.buffer), _ptr(self.ws),
+                                      self.ws.numel(), _stream(st)), "laq_pass_run")
 
     def status(self):
         """The device-side status word (synchronizes the device)."""

@@ -1,10 +1,12 @@
 // laq_api.cu -- the C ABI of include/laq.h: argument validation, launch planning and dispatch.
 // Validation happens before any CUDA call, so invalid arguments are reported without a device.
+#include <cuda.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
 #include <atomic>
 #include <climits>
+#include <mutex>
 #include <vector>
 
 #include "laq.h"
@@ -256,12 +258,18 @@ size_t chain_ws_bytes(int32_t count) {
     return (laq::chain_workspace_bytes(count) + 255) / 256 * 256;
 }
 
+laq_status static_scratch(void** out, size_t* bytes);
+
+// With use_static, the workspace is the library's static scratch (laq_gemm_chain_static): its
+// address is looked up, and the counters and flags it must start with at zero are cleared on
+// the stream, only once every argument has passed its checks, just before the launch.
 laq_status run_chain(const laq_gemv* g, int32_t count, void* workspace, size_t workspace_bytes,
-                     void* stream) {
+                     void* stream, bool use_static = false) {
     if (count < 0 || count > LAQ_CHAIN_MAX) return LAQ_ERR_SHAPE;
     if (count == 0) return LAQ_OK;
     if (!g) return LAQ_ERR_NULL;
-    if (!workspace || !aligned(workspace, 16) || workspace_bytes < chain_ws_bytes(count))
+    if (!use_static &&
+        (!workspace || !aligned(workspace, 16) || workspace_bytes < chain_ws_bytes(count)))
         return LAQ_ERR_WORKSPACE;
     const int bits = g[0].bits;
     laq_status st = check_bits(bits);
@@ -310,6 +318,11 @@ laq_status run_chain(const laq_gemv* g, int32_t count, void* workspace, size_t w
     }
     stages[nst - 1].records = (int)stage_records;
 
+    if (use_static) {
+        st = static_scratch(&workspace, &workspace_bytes);
+        if (st != LAQ_OK) return st;
+        if (workspace_bytes < chain_ws_bytes(count)) return LAQ_ERR_WORKSPACE;
+    }
     DeviceFacts f;
     st = device_facts(&f);
     if (st != LAQ_OK) return st;
@@ -349,6 +362,9 @@ laq_status run_chain(const laq_gemv* g, int32_t count, void* workspace, size_t w
     L.bits = bits;
     L.xs_bytes = (int)xs_need;
     L.ws = static_cast<uint32_t*>(workspace);
+    if (use_static && cudaMemsetAsync(workspace, 0, laq::chain_workspace_zeroed_bytes(count),
+                                      static_cast<cudaStream_t>(stream)) != cudaSuccess)
+        return LAQ_ERR_CUDA;
     return from_cuda(laq::launch_chain(L, f.sms, static_cast<cudaStream_t>(stream)));
 }
 
@@ -362,21 +378,63 @@ laq_status run_chain(const laq_gemv* g, int32_t count, void* workspace, size_t w
 constexpr size_t kStaticScratchBytes = 68352;
 static __device__ __align__(256) uint32_t g_chain_scratch[kStaticScratchBytes / 4];
 
-// Device address of g_chain_scratch per device, looked up on the first call with that device
-// current (the array's name is only a host-side stand-in for it).
-std::atomic<void*> g_scratch_addr[kMaxDevices];
+// Device address of g_chain_scratch per device (the array's name is only a host-side stand-in
+// for it), looked up with the device current on the first call in each CUDA context: after
+// cudaDeviceReset the device's next context holds the array at another address, so the cached
+// address is tied to the unique id of the context it was looked up in.
+struct ScratchAddr {
+    unsigned long long ctx_id;
+    void* ptr;
+};
+ScratchAddr g_scratch_addr[kMaxDevices];
+std::mutex g_scratch_mu;
 
-laq_status static_scratch(void** out) {
+// The unique id of the calling thread's current context.  The two driver calls are reached
+// through the runtime's entry-point query, so the library does not link the driver library
+// itself (it still loads where no driver is installed, for its host-only entry points).
+using CtxGetCurrentFn = CUresult (*)(CUcontext*);
+using CtxGetIdFn = CUresult (*)(CUcontext, unsigned long long*);
+
+laq_status current_ctx_id(unsigned long long* id) {
+    static CtxGetCurrentFn get_current = nullptr;
+    static CtxGetIdFn get_id = nullptr;
+    if (!get_current || !get_id) {
+        void* f0 = nullptr;
+        void* f1 = nullptr;
+        cudaDriverEntryPointQueryResult q0, q1;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &f0, 12000, cudaEnableDefault,
+                                             &q0) != cudaSuccess ||
+            q0 != cudaDriverEntryPointSuccess ||
+            cudaGetDriverEntryPointByVersion("cuCtxGetId", &f1, 12000, cudaEnableDefault,
+                                             &q1) != cudaSuccess ||
+            q1 != cudaDriverEntryPointSuccess || !f0 || !f1)
+            return LAQ_ERR_CUDA;
+        get_current = reinterpret_cast<CtxGetCurrentFn>(f0);
+        get_id = reinterpret_cast<CtxGetIdFn>(f1);
+    }
+    CUcontext ctx = nullptr;
+    if (get_current(&ctx) != CUDA_SUCCESS || !ctx) return LAQ_ERR_CUDA;
+    return get_id(ctx, id) == CUDA_SUCCESS ? LAQ_OK : LAQ_ERR_CUDA;
+}
+
+laq_status static_scratch(void** out, size_t* bytes) {
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return LAQ_ERR_CUDA;
     if (dev < 0 || dev >= kMaxDevices) return LAQ_ERR_CUDA;
-    void* ptr = g_scratch_addr[dev].load();
-    if (!ptr) {
+    std::lock_guard<std::mutex> lock(g_scratch_mu);
+    unsigned long long id = 0;
+    const bool have_ctx = current_ctx_id(&id) == LAQ_OK;  // none yet: the lookup makes one
+    ScratchAddr& a = g_scratch_addr[dev];
+    if (!have_ctx || !a.ptr || a.ctx_id != id) {
+        void* ptr = nullptr;
         if (cudaGetSymbolAddress(&ptr, g_chain_scratch) != cudaSuccess || !ptr)
             return LAQ_ERR_CUDA;
-        g_scratch_addr[dev].store(ptr);
+        if (current_ctx_id(&id) != LAQ_OK) return LAQ_ERR_CUDA;
+        a.ptr = ptr;
+        a.ctx_id = id;
     }
-    *out = ptr;
+    *out = a.ptr;
+    *bytes = kStaticScratchBytes;
     return LAQ_OK;
 }
 
@@ -492,20 +550,11 @@ laq_status laq_gemm_chain(const laq_gemv* gemvs, int32_t count, void* workspace,
 }
 
 laq_status laq_gemm_chain_static(const laq_gemv* gemvs, int32_t count, void* stream) {
-    if (count < 0 || count > LAQ_CHAIN_MAX) return LAQ_ERR_WORKSPACE;  // beyond the scratch
-    if (count == 0) return LAQ_OK;
-    if (!gemvs) return LAQ_ERR_NULL;
-    void* scratch = nullptr;
-    laq_status st = static_scratch(&scratch);
-    if (st != LAQ_OK) return st;
-    // Counters and flags must start at zero; a previous call that gave up may have left them
-    // set.  (The published parts need no clearing.)
-    const size_t used = chain_ws_bytes(count);
-    if (used > kStaticScratchBytes) return LAQ_ERR_WORKSPACE;
-    if (cudaMemsetAsync(scratch, 0, laq::chain_workspace_zeroed_bytes(count),
-                        static_cast<cudaStream_t>(stream)) != cudaSuccess)
-        return LAQ_ERR_CUDA;
-    return run_chain(gemvs, count, scratch, used, stream);
+    if (count > LAQ_CHAIN_MAX) return LAQ_ERR_WORKSPACE;  // beyond the scratch
+    // Counters and flags must start at zero (a previous call that gave up may have left them
+    // set; the published parts need no clearing): run_chain clears them only once every
+    // argument has passed its checks, right before the launch.
+    return run_chain(gemvs, count, nullptr, 0, stream, true);
 }
 
 }  // extern "C"

@@ -174,6 +174,8 @@ laq_status plan_pass(const laq_gemv* g, int32_t count, int32_t P, HostPlan& H) {
         if (e.M != H.M) return LAQ_ERR_M_RANGE;
         if (e.K <= 0 || e.N <= 0 || e.K % 128 != 0 || e.N % 16 != 0) return LAQ_ERR_SHAPE;
         if (e.K * 2 * e.M > kMaxXsBytes || e.N / 16 > ((int64_t)1 << 24)) return LAQ_ERR_SHAPE;
+        // a record's id t * G + g (GatherRec::rid) is a 32-bit int
+        if ((e.N / 16) * (e.K / 128) > (int64_t)INT_MAX) return LAQ_ERR_SHAPE;
         if (!e.X || !e.packed || !e.s || !e.z || !e.Y) return LAQ_ERR_NULL;
         if (!aligned16(e.X) || !aligned16(e.packed) || !aligned16(e.s) || !aligned16(e.z) ||
             !aligned16(e.Y))

@@ -213,26 +213,3 @@ class DecodeStep:
         M, D, Hkv = self.M, self.D, self.Hkv
         kv = self.layers * M * Hkv * D * 2 * 2 * (self.context + 1)
         return (self.wp.bytes_per_pass() + self.lm.bytes_per_call(M) + kv + M * self.H * 2)
-
-    # ---- host copies for the oracle (tests) ----
-
-    def oracle_model(self):
-        """The model as numpy arrays for oracle.decoder.decode_step: quantized projections as
-        (codes, s, z) re-derived on the host by the C oracle from the same fp16 weights."""
-        from oracle import c_oracle
-        layers = []
-        for l in range(self.layers):
-            ws = []
-            for i, (_, members, _, _) in enumerate(self.wp.linears[4 * l:4 * l + 4]):
-                W = self.wp.weight(l, members).cpu().numpy()
-                ws.append(c_oracle.quantize_rtn(W, self.bits))
-            nw = {k: v.cpu().numpy() for k, v in self.norms[l].items()}
-            layers.append(dict(qkv=ws[0], o=ws[1], gate_up=ws[2], down=ws[3], **nw))
-            if self.rot:
-                layers[-1]["rot"] = {name: (t["alpha"].cpu().numpy(), t["pairs"].cpu().numpy(),
-                                            t["theta"].cpu().numpy())
-                                     for name, t in self.rot[l].items()}
-        E = self.E.cpu().numpy()
-        return {"E": E, "layers": layers, "final_w": self.final_w.cpu().numpy(),
-                "lm": c_oracle.quantize_rtn(E.T.copy(), self.bits), "Hq": self.Hq,
-                "Hkv": self.Hkv, "D": self.D, "I": self.I, "theta": self.theta, "eps": self.eps}

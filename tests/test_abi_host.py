@@ -203,8 +203,16 @@ def test_chain_static_argument_validation(L):
     arr = (_lib.Gemv * 1)(chain_entry())
     assert L.laq_gemm_chain_static(arr, 0, None) == 0
     assert L.laq_gemm_chain_static(arr, _lib.CHAIN_MAX + 1, None) == code["LAQ_ERR_WORKSPACE"]
-    assert L.laq_gemm_chain_static(arr, -1, None) == code["LAQ_ERR_WORKSPACE"]
+    assert L.laq_gemm_chain_static(arr, -1, None) == code["LAQ_ERR_SHAPE"]
     assert L.laq_gemm_chain_static(None, 1, None) == code["LAQ_ERR_NULL"]
+    # every entry is checked before the static scratch is looked up or cleared: these return
+    # without a device
+    bad = (_lib.Gemv * 1)(chain_entry(bits=5))
+    assert L.laq_gemm_chain_static(bad, 1, None) == code["LAQ_ERR_BITS"]
+    bad = (_lib.Gemv * 1)(chain_entry(X=ODD))
+    assert L.laq_gemm_chain_static(bad, 1, None) == code["LAQ_ERR_ALIGN"]
+    bad = (_lib.Gemv * 1)(chain_entry(N=0))
+    assert L.laq_gemm_chain_static(bad, 1, None) == code["LAQ_ERR_SHAPE"]
 
 
 def test_plan_shares_x_across_tiles_at_m_above_one(L):

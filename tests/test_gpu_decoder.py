@@ -258,6 +258,29 @@ def test_gemm_prologue_rejects_aliasing():
 
 # ---- one whole decode step (2 layers, real Qwen3-4B widths, small vocabulary) ----
 
+def oracle_model(st):
+    """The decode step ``st`` (a DecodeStep) as numpy arrays for oracle.decoder.decode_step: the
+    quantized projections as (codes, s, z) re-derived on the host by the C oracle from the same
+    fp16 weights, the norm weights, the rotation tables and the embedding."""
+    from oracle import c_oracle
+    layers = []
+    for l in range(st.layers):
+        ws = []
+        for _, members, _, _ in st.wp.linears[4 * l:4 * l + 4]:
+            W = st.wp.weight(l, members).cpu().numpy()
+            ws.append(c_oracle.quantize_rtn(W, st.bits))
+        nw = {k: v.cpu().numpy() for k, v in st.norms[l].items()}
+        layers.append(dict(qkv=ws[0], o=ws[1], gate_up=ws[2], down=ws[3], **nw))
+        if st.rot:
+            layers[-1]["rot"] = {name: (t["alpha"].cpu().numpy(), t["pairs"].cpu().numpy(),
+                                        t["theta"].cpu().numpy())
+                                 for name, t in st.rot[l].items()}
+    E = st.E.cpu().numpy()
+    return {"E": E, "layers": layers, "final_w": st.final_w.cpu().numpy(),
+            "lm": c_oracle.quantize_rtn(E.T.copy(), st.bits), "Hq": st.Hq, "Hkv": st.Hkv,
+            "D": st.D, "I": st.I, "theta": st.theta, "eps": st.eps}
+
+
 @pytest.mark.parametrize("bits,M,fused,norms,rot", [
     (3, 1, True, True, 0), (4, 2, True, True, 0), (3, 2, False, False, 0), (4, 1, True, False, 0),
     # the rotation-based variant: a pairwise rotation before every projection of a layer
@@ -272,7 +295,7 @@ def test_decode_step(bits, M, fused, norms, rot):
     pos = [st.context - 1] * M
     st.run()
     logits, nxt = host(st.logits), host(st.next)
-    model = st.oracle_model()
+    model = oracle_model(st)
     rl, rn, rk, rv = dec.decode_step(model, tokens, pos, kc0, vc0)
     close(logits, rl, "logits")
     # the greedy token: equal unless the oracle's top two logits are within the tolerance

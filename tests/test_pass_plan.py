@@ -366,6 +366,8 @@ def test_plan_rejects_invalid_entries(L):
     assert sizes(L, fake_entries([(0, 16, 0)]), 1, 4) == 4
     assert sizes(L, fake_entries([(53248, 16, 0)]), 1, 4) == 0   # largest K at M = 1
     assert sizes(L, fake_entries([(53248 + 128, 16, 0)]), 1, 4) == 4
+    # 2^23 tiles of 416 groups: record ids t * G + g would pass 2^31
+    assert sizes(L, fake_entries([(53248, 16 << 23, 0)]), 1, 4) == 4
     assert sizes(L, fake_entries(ok), 2, 0) == 4                 # no SMs
     assert sizes(L, fake_entries(ok), 2, 1025) == 4
     assert sizes(L, fake_entries([(128, 16, 0)] * 385), 385, 4) == 4
