@@ -63,6 +63,18 @@ constexpr int kMaxSegs = 255;                  // warp segments per (SM, stage)
 constexpr int kMaxXsBytes = 104 * 1024;        // staged X per (SM, stage), all M rows
 constexpr int kMaxM = 4;                       // batch rows
 constexpr int kMaxRing = 16;                   // ring slots
+// Rounds a producer keeps in flight.  About four rounds per SM (50-70 KB, 8-10 MB over the GPU)
+// already sustain the full HBM rate; many more queue so deep in the memory system that the
+// latency-critical loads of a stage change (the completed-stage flags, the stage's X) wait
+// behind them: with the whole ring refilled at once after a large stage, a single flag poll
+// took 5 us.
+constexpr int kInflight = 4;
+// Stages the producer may run ahead of the consumers: it copies the rounds of stage s only once
+// the consumers have seen stage s - kLead's dependency met.  Copies issued while the stages hand
+// over (every SM's release store, the flag polls and the next stage's X loads) queue those
+// latency-critical accesses behind HBM reads: after a large stage, with every SM refilling its
+// ring at once, the 152 release stores took up to 5 us to become visible.
+constexpr int kLead = 1;
 constexpr int kMaxSms = 1024;
 constexpr unsigned long long kWaitNs = 1000000000ull;  // wait limit (1 s)
 constexpr int kWaitSpins = 1 << 24;                    // and an iteration limit besides
@@ -395,9 +407,16 @@ const PlanHeader* as_plan(const void* plan) {
     return h;
 }
 
-// Workspace: [0] status, [1] finished CTAs, [2 + j] the stages CTA j has completed.
-size_t pass_workspace(const PlanHeader& h) {
-    return (size_t)align_up(4 * (2 + (int64_t)h.sms), 256);
+// Workspace: uint32 [0] status, [1] finished CTAs; then kCounters stage counters, each in a
+// 128-byte line of its own: every CTA adds 1 to counter s % kCounters when it has completed
+// stage s, so stage s is complete once that counter reaches P (s / kCounters + 1).  (Measured on
+// GB300 with all 152 CTAs arriving at once: the last arrival is seen 0.96 us later, against
+// 2.1 us for per-CTA 16-bit flags packed into three lines and 1.5 us for per-CTA flags in lines
+// of their own: many writers into the lines every CTA polls are what costs.)
+constexpr int kCounters = 8;
+constexpr int kCounterStride = 32;  // uint32 words: one 128-byte line
+size_t pass_workspace(const PlanHeader&) {
+    return (size_t)align_up(4 * kCounterStride * (1 + kCounters), 256);
 }
 
 // ---- shared memory layout of the pass kernel (host and device) -------------------------------
@@ -432,16 +451,18 @@ __device__ __forceinline__ unsigned long long gtimer() {
     asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
     return t;
 }
+__device__ __forceinline__ uint32_t ld_acq(const uint32_t* p) {
+    uint32_t v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
 __device__ __forceinline__ uint32_t ld_rlx(const uint32_t* p) {
     uint32_t v;
     asm volatile("ld.relaxed.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
     return v;
 }
-__device__ __forceinline__ void fence_acq_rel_gpu() {
-    asm volatile("fence.acq_rel.gpu;" ::: "memory");
-}
-__device__ __forceinline__ void st_rel(uint32_t* p, uint32_t v) {
-    asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+__device__ __forceinline__ void red_rel_add(uint32_t* p, uint32_t v) {
+    asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
 }
 __device__ __forceinline__ uint32_t atom_acq_rel_add(uint32_t* p, uint32_t v) {
     uint32_t old;
@@ -537,31 +558,18 @@ __device__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort_fla
     return false;
 }
 
-// One warp waits until every CTA's completed-stage flag (flags[0 .. n)) is >= target.  Each
-// lane reads every 32nd flag with relaxed loads that are all in flight at once (no load waits
-// for another), so a poll costs one round trip to L2 and no two CTAs ever write the same word;
-// once every flag is seen, one acquire fence orders what the warp's CTA reads next after the
-// releases it observed.  Returns the same answer in every lane: false when the status word holds
-// an error (checked every 16th poll), or after about a second (then LAQ_ERR_TIMEOUT is
-// recorded).
-__device__ bool wait_flags(const uint32_t* flags, int n, uint32_t target, uint32_t* status,
-                           int lane) {
+// One warp waits until stage `stage` is complete: its counter has reached the number of CTAs
+// times the count of stages so far that share the counter.  Lane 0 polls with acquire loads;
+// the answer is warp-wide: false when the status word holds an error (checked every 16th poll),
+// or after about a second (then LAQ_ERR_TIMEOUT is recorded).
+__device__ bool wait_stage_done(const uint32_t* ws, int stage, uint32_t ctas, uint32_t* status,
+                                int lane) {
+    const uint32_t* cnt = ws + kCounterStride * (1 + stage % kCounters);
+    const uint32_t target = ctas * (uint32_t)(stage / kCounters + 1);
     const unsigned long long t0 = gtimer();
     for (int spin = 0; spin < kWaitSpins; ++spin) {
-        uint32_t v[8];
-#pragma unroll
-        for (int u = 0; u < 8; ++u) {
-            const int j = lane + 32 * u;
-            v[u] = j < n ? ld_rlx(flags + j) : target;
-        }
-        bool ok = true;
-#pragma unroll
-        for (int u = 0; u < 8; ++u) ok &= v[u] >= target;
-        for (int j = lane + 256; j < n; j += 32) ok &= ld_rlx(flags + j) >= target;
-        if (__all_sync(0xffffffffu, ok)) {
-            fence_acq_rel_gpu();
-            return true;
-        }
+        const int ok = lane == 0 ? (int)(ld_acq(cnt) >= target) : 0;
+        if (__shfl_sync(0xffffffffu, ok, 0)) return true;
         if ((spin & 15) == 15) {
             const uint32_t st = lane == 0 ? ld_rlx(status) : 0u;
             if (__shfl_sync(0xffffffffu, st, 0) != 0u) return false;
@@ -581,7 +589,7 @@ struct PassParams {
     const Seg* seg;
     const LTile* tile;
     const XItem* xi;
-    uint32_t* ws;  // [0] status, [1] finished CTAs, [2 + j] stages CTA j has completed
+    uint32_t* ws;  // [0] status, [1] finished CTAs, then the stage counters
     int nstages, ns, xs_bytes, max_segs, max_nx;
     int M;       // batch rows (1..4)
     int xg_row;  // groups of one staged X row
@@ -590,10 +598,36 @@ struct PassParams {
 
 // ---- the producer warp -------------------------------------------------------------------------
 
+// Lane 0 waits until the consumers have met the dependency of stage `target` (*cur_stage, set by
+// the consumers, is at least target); the answer is warp-wide.  False when the CTA aborts or
+// after about a second (then the abort flag and LAQ_ERR_TIMEOUT are set).
+__device__ bool wait_stage(volatile int* cur_stage, int target, volatile int* abort_flag,
+                           uint32_t* status, int lane) {
+    int ok = 1;
+    if (lane == 0 && *cur_stage < target) {
+        ok = 0;
+        const unsigned long long t0 = gtimer();
+        for (int spin = 0; spin < kWaitSpins; ++spin) {
+            if (*cur_stage >= target) {
+                ok = 1;
+                break;
+            }
+            if (*abort_flag) break;
+            __nanosleep(64);
+            if ((spin & 63) == 63 && gtimer() - t0 > kWaitNs) {
+                *abort_flag = 1;
+                record_timeout(status);
+                break;
+            }
+        }
+    }
+    return __shfl_sync(0xffffffffu, ok, 0) != 0;
+}
+
 template <int BITS>
 __device__ void pass_producer(const PassParams& p, const SmDesc& sd, uint32_t ring_s,
                               uint32_t full_s, uint32_t empty_s, volatile int* abort_flag,
-                              int lane) {
+                              volatile int* cur_stage, int lane) {
     constexpr int RB = RecordFmt<BITS>::kBytes + kSZ;
     constexpr uint32_t SLOT = (uint32_t)(kPRec * RB);
     const int NS = p.ns, NR = sd.nrounds;
@@ -602,18 +636,42 @@ __device__ void pass_producer(const PassParams& p, const SmDesc& sd, uint32_t ri
     const uint64_t pol = evict_first_policy();
     int issued = 0;
     bool ok = true;
+    // the stage of round r: rounds [stage_end - nr(stage), stage_end)
+    const StageDesc* sdp = p.stage + (size_t)blockIdx.x * p.nstages;
+    int stage = -1, stage_end = 0;
     for (int r0 = 0; r0 < NR && ok; r0 += 32) {
         const int mine = r0 + lane < NR ? (int)rt[r0 + lane] : 0;
         const int lim = NR - r0 < 32 ? NR - r0 : 32;
         for (int i = 0; i < lim; ++i) {
             const int cnt = __shfl_sync(0xffffffffu, mine, i);
             const int r = r0 + i, slot = r % NS, k = r / NS;
+            if (r == stage_end) {
+                do {
+                    ++stage;
+                    stage_end += sdp[stage].nr;
+                } while (r == stage_end);
+                // the consumers have met stage (stage - kLead)'s dependency
+                if (stage - kLead > 0 && !wait_stage(cur_stage, stage - kLead, abort_flag, p.ws, lane)) {
+                    ok = false;
+                    break;
+                }
+            }
             // slot reuse: every consumer warp has released the round that used it last
             if (k > 0 && !__all_sync(0xffffffffu,
                                      mbar_wait(empty_s + 8u * slot, (uint32_t)((k - 1) & 1),
                                                abort_flag, p.ws))) {
                 ok = false;
                 break;
+            }
+            // at most kInflight rounds in flight: round r - kInflight has landed
+            if (r >= kInflight) {
+                const int ro = r - kInflight;
+                if (!__all_sync(0xffffffffu, mbar_wait(full_s + 8u * (ro % NS),
+                                                       (uint32_t)((ro / NS) & 1), abort_flag,
+                                                       p.ws))) {
+                    ok = false;
+                    break;
+                }
             }
             if (lane == 0) {
                 const uint32_t bytes = (uint32_t)(cnt * RB);
@@ -635,29 +693,30 @@ __device__ void pass_producer(const PassParams& p, const SmDesc& sd, uint32_t ri
 
 // Stage one entry's X (M rows of K fp16) in the X area, whose rows are xg_row groups apart:
 // 16-byte chunk cr of row b lands at xs[16 (b xg_row + xg) + cr]; the 16 lanes holding a
-// group's chunks sum S = sum_k x_k and P = sum_k c_k x_k (chunk q of a group holds pairs
-// 4 (q % 4) + w, w < 4, of the record layout) into sp[b xg_row + xg + group].  K / 8 is a
-// multiple of 16, so the 16 lanes of a group are a half-warp of one row.
-template <int BITS>
-__device__ void pass_stage_x(const XItem& X, int M, int xg_row, uint4* xs, float2* sp,
-                             int tid) {
+// group's chunks sum S = sum_k x_k and P = sum_k c_k x_k into sp[b xg_row + xg + group].  K / 8
+// is a multiple of 16, so the 16 lanes of a group are a half-warp of one row, and a thread's
+// chunks all sit at the same position q % 4 of their group (q = tid % 4): chunk q holds pairs
+// 4 q + w, w < 4, of the record layout, whose offsets c_k the thread keeps in off[w].
+__device__ void pass_stage_x(const XItem& X, int M, int xg_row, uint4* xs, float2* sp, int tid,
+                             const float (&off)[4]) {
     const int nch = X.K >> 3;  // chunks per row
     const int total = M * nch;
     for (int c0 = 0; c0 < total; c0 += 4 * 512) {
         uint4 v[4];
+        int bb[4], cc[4];
 #pragma unroll
         for (int u = 0; u < 4; ++u) {
             const int ci = c0 + u * 512 + tid;
-            const int b = ci / nch;
-            v[u] = ci < total ? ld_cg16(X.x + (size_t)b * X.K + 8 * (size_t)(ci - b * nch))
+            const int b = (ci >= nch) + (ci >= 2 * nch) + (ci >= 3 * nch);  // M <= 4 rows
+            bb[u] = b;
+            cc[u] = ci - b * nch;
+            v[u] = ci < total ? ld_cg16(X.x + (size_t)b * X.K + 8 * (size_t)cc[u])
                               : make_uint4(0u, 0u, 0u, 0u);
         }
 #pragma unroll
         for (int u = 0; u < 4; ++u) {
-            const int wfirst = c0 + u * 512 + (tid & ~31);  // the warp's first chunk
-            if (wfirst >= total) break;                     // warp-uniform
-            const int ci = wfirst + (tid & 31);
-            const int b = ci / nch, cr = ci - b * nch;
+            if (c0 + u * 512 + (tid & ~31) >= total) break;  // warp-uniform
+            const int ci = c0 + u * 512 + tid;
             const uint32_t w4[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
             float sx = 0.f, px = 0.f;
 #pragma unroll
@@ -665,7 +724,7 @@ __device__ void pass_stage_x(const XItem& X, int M, int xg_row, uint4* xs, float
                 const float2 f = __half22float2(*reinterpret_cast<const __half2*>(&w4[w]));
                 const float pair = f.x + f.y;
                 sx += pair;
-                px = fmaf(row_offset<BITS>((cr & 3) * 4 + w), pair, px);
+                px = fmaf(off[w], pair, px);
             }
 #pragma unroll
             for (int o = 1; o < 16; o <<= 1) {
@@ -673,9 +732,9 @@ __device__ void pass_stage_x(const XItem& X, int M, int xg_row, uint4* xs, float
                 px += __shfl_xor_sync(0xffffffffu, px, o);
             }
             if (ci < total) {
+                const int b = bb[u], cr = cc[u];
                 xs[16 * (b * xg_row + X.xg) + cr] = v[u];
-                if ((cr & 15) == 0)
-                    sp[b * xg_row + X.xg + (cr >> 4)] = make_float2(sx, px);
+                if ((cr & 15) == 0) sp[b * xg_row + X.xg + (cr >> 4)] = make_float2(sx, px);
             }
         }
     }
@@ -684,17 +743,130 @@ __device__ void pass_stage_x(const XItem& X, int M, int xg_row, uint4* xs, float
 // MP: the batch rows M rounded up to 1, 2 or 4.  The MMA's 8 columns hold GPA = 8 / MP groups
 // of each of MP batch rows: column col is batch row col / GPA and record col % GPA of a block of
 // GPA records (at M = 1 the 8 columns are 8 groups of the one row).
+
+// A position in the ring: the slot of a round and the phase parity of that slot's use.
+struct RingPos {
+    int slot;
+    uint32_t par;
+};
+__device__ __forceinline__ void ring_next(RingPos& q, int NS) {
+    if (++q.slot == NS) {
+        q.slot = 0;
+        q.par ^= 1u;
+    }
+}
+
+// Wait for the n rounds from ring position q on (every lane polls; the answer is warp-wide).
+// False when the CTA is aborting or a wait gave up.
+__device__ __forceinline__ bool wait_rounds(uint32_t full_s, RingPos q, int n, int NS,
+                                            volatile int* abort_flag, uint32_t* status) {
+    bool ok = true;
+    for (int i = 0; i < n && ok; ++i) {
+        ok = mbar_wait(full_s + 8u * q.slot, q.par, abort_flag, status);
+        ring_next(q, NS);
+    }
+    return __all_sync(0xffffffffu, ok);
+}
+
+// This warp is done with the n rounds from ring position q on: one arrival each on their slots'
+// empty barriers (after every lane's reads), and q moves past them.
+__device__ __forceinline__ void release_rounds(uint32_t empty_s, RingPos& q, int n, int NS,
+                                               int lane) {
+    __syncwarp();
+    for (int i = 0; i < n; ++i) {
+        if (lane == 0) mbar_arrive(empty_s + 8u * q.slot);
+        ring_next(q, NS);
+    }
+}
+
+// One record: its packed codes (this lane's words at rec), the B fragments at xsrc (this lane's
+// x values, or the zero block), the mask-and-or extraction and the 8 MMAs of the 8 k16 steps of
+// the group, accumulated on four chains (steps j and j + 4 share chain j % 4).
+template <int BITS>
+__device__ __forceinline__ void pass_record(const uint8_t* rec, const uint4* xsrc,
+                                            const Exps& ex, float (&D)[4][4], int lane) {
+    constexpr int WPL = BITS == 4 ? 8 : 6;
+    uint32_t B[8][2];
+#pragma unroll
+    for (int qq = 0; qq < 4; ++qq) {
+        const uint4 v = xsrc[qq];
+        B[2 * qq][0] = v.x;
+        B[2 * qq][1] = v.y;
+        B[2 * qq + 1][0] = v.z;
+        B[2 * qq + 1][1] = v.w;
+    }
+    uint32_t wd[WPL];
+    const uint4 c0 = *reinterpret_cast<const uint4*>(rec + lane * 16);
+    wd[0] = c0.x;
+    wd[1] = c0.y;
+    wd[2] = c0.z;
+    wd[3] = c0.w;
+    if constexpr (BITS == 4) {
+        const uint4 c1 = *reinterpret_cast<const uint4*>(rec + 512 + lane * 16);
+        wd[4] = c1.x;
+        wd[5] = c1.y;
+        wd[6] = c1.z;
+        wd[7] = c1.w;
+    } else {
+        const uint2 c1 = *reinterpret_cast<const uint2*>(rec + 512 + lane * 8);
+        wd[4] = c1.x;
+        wd[5] = c1.y;
+    }
+    uint32_t a[8][4];
+    extract<BITS>(wd, ex, a);
+#pragma unroll
+    for (int j = 0; j < 8; ++j)
+        mma16816(D[j & 3], a[j][0], a[j][1], a[j][2], a[j][3], B[j][0], B[j][1]);
+}
+
+// The block epilogue (Eq. (1)) of a block of len records whose first record is at ring slot
+// slot0: accumulator value v of this lane is output row R + 8 (v >> 1) and MMA column
+// col = 2c + (v & 1), i.e. batch row col / GPA and block record col % GPA; it adds
+// s (D - P - z S) with the record's scale and zero (read from the record's ring slot, which the
+// warp still holds) and the group's (S, P) sums (spb: the block's first group, row 0).
 template <int BITS, int MP>
-__device__ void pass_consumer(const PassParams& p, uint8_t* smem, const PassSmem& L,
-                              uint32_t full_s, uint32_t empty_s, volatile int* abort_flag,
-                              int warp, int lane) {
+__device__ __forceinline__ void pass_epilogue(const uint8_t* ring, int slot0, int NS, int warp,
+                                              int lane, int len, int M, int XR,
+                                              const float2* spb, const float (&D)[4][4],
+                                              float (&y)[4]) {
     constexpr int RBC = RecordFmt<BITS>::kBytes;
     constexpr int RB = RBC + kSZ;
     constexpr int SLOT = kPRec * RB;
-    constexpr int WPL = BITS == 4 ? 8 : 6;
-    const int tid = warp * 32 + lane;
+    constexpr int GPA = 8 / MP;
+    const int c = lane & 3, R = lane >> 2;
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {  // the lane's two MMA columns
+        const int col = 2 * c + h;
+        const int b = col / GPA, giv = col % GPA;
+        if (giv < len && b < M) {
+            int sl = slot0 + giv;
+            if (sl >= NS) sl -= NS;
+            const uint8_t* sz = ring + (size_t)sl * SLOT + (size_t)warp * RB + RBC;
+            const uint32_t sw = reinterpret_cast<const uint32_t*>(sz)[R];   // s of rows R, R + 8
+            const uint32_t zw = reinterpret_cast<const uint16_t*>(sz + 32)[R];  // z of R, R + 8
+            const float2 spv = spb[b * XR + giv];                             // (S, P)
+#pragma unroll
+            for (int hi = 0; hi < 2; ++hi) {
+                const int v = 2 * hi + h;
+                const float dv = (D[0][v] + D[1][v]) + (D[2][v] + D[3][v]);
+                const float sc = __half2float(__ushort_as_half((uint16_t)(sw >> (16 * hi))));
+                const float zc = (float)((zw >> (8 * hi)) & 0xffu);
+                y[v] = fmaf(sc, dv - spv.y - zc * spv.x, y[v]);
+            }
+        }
+    }
+}
+
+template <int BITS, int MP>
+__device__ void pass_consumer(const PassParams& p, uint8_t* smem, const PassSmem& L,
+                              uint32_t full_s, uint32_t empty_s, volatile int* abort_flag,
+                              volatile int* cur_stage, int warp, int lane) {
+    constexpr int RBC = RecordFmt<BITS>::kBytes;
+    constexpr int RB = RBC + kSZ;
+    constexpr int SLOT = kPRec * RB;
     constexpr int GPA = 8 / MP;  // records per block: groups sharing one accumulator
     constexpr int LPB = 4 / MP;  // lanes of one output row that hold one batch row's columns
+    const int tid = warp * 32 + lane;
     const int c = lane & 3, R = lane >> 2;
     const int bl = R / GPA, gil = R % GPA;  // batch row and block record of MMA column R
     const int NS = p.ns, M = p.M, XR = p.xg_row;
@@ -706,8 +878,10 @@ __device__ void pass_consumer(const PassParams& p, uint8_t* smem, const PassSmem
     float* slots = reinterpret_cast<float*>(smem + L.slot);
     const uint4* zblk = reinterpret_cast<const uint4*>(smem + L.zero);
     const uint8_t* ring = smem;
-    int slot = 0;        // ring position of the SM's next round
-    uint32_t par = 0u;   // and the phase parity of its slot
+    float off[4];        // offsets c_k of this thread's pairs of X (see pass_stage_x)
+#pragma unroll
+    for (int w = 0; w < 4; ++w) off[w] = row_offset<BITS>((tid & 3) * 4 + w);
+    RingPos pos{0, 0u};  // ring position of the SM's next round
 
     for (int s = 0; s < p.nstages; ++s) {
         const StageDesc* dp = p.stage + (size_t)blockIdx.x * p.nstages + s;
@@ -718,7 +892,7 @@ __device__ void pass_consumer(const PassParams& p, uint8_t* smem, const PassSmem
         // shared memory: every consumer has passed the previous stage's last barrier, so
         // nothing reads the old ones any more.
         bool bad = false;
-        if (warp == 0 && s > 0) bad = !wait_flags(p.ws + 2, gridDim.x, (uint32_t)s, p.ws, lane);
+        if (warp == 0 && s > 0) bad = !wait_stage_done(p.ws, s - 1, gridDim.x, p.ws, lane);
         if (tid == 0 && bad) *abort_flag = 1;
         if (warp > 0) {
             const int nseg = dp->nseg, nt = dp->nt, nx = dp->nx;
@@ -727,143 +901,96 @@ __device__ void pass_consumer(const PassParams& p, uint8_t* smem, const PassSmem
             for (int i = tid - 32; i < nx; i += 480) xitems[i] = p.xi[dp->x0 + i];
         }
         if (cbar_any(bad || *abort_flag)) return;
+        if (tid == 0) *cur_stage = s;  // the producer may copy the stage's rounds
         const int n = dp->n, nr = dp->nr, nt = dp->nt, nx = dp->nx;
         const int k0 = dp->wseg[warp], k1 = dp->wseg[warp + 1];
         if (n > 0) {
-            for (int i = 0; i < nx; ++i) pass_stage_x<BITS>(xitems[i], M, XR, xs, sp, tid);
+            for (int i = 0; i < nx; ++i) pass_stage_x(xitems[i], M, XR, xs, sp, tid, off);
             cbar();
 
-            // This warp's records: the first q + (warp < rem) of the stage's rounds, at
-            // position `warp` of each round's slot.
+            // This warp's records are the first len rounds of the stage (position `warp` of
+            // each round's slot); walked segment by segment, in blocks of up to GPA records.
             const int len = (n >> 4) + (warp < (n & 15) ? 1 : 0);
-            int k = k0, i = 0, gi = 0;
-            Seg sg = k < k1 ? segs[k] : Seg{0, 0, 0, 0, 0, 0};
-            float D[4][4], y[4];  // four accumulator chains: k16 steps j, j + 4 share one
-            // scale and zero row pairs of the lane's block columns 2c, 2c + 1
-            uint32_t sw[2] = {0u, 0u}, zw[2] = {0u, 0u};
-#pragma unroll
-            for (int v = 0; v < 4; ++v) D[0][v] = D[1][v] = D[2][v] = D[3][v] = y[v] = 0.f;
+            RingPos q = pos;
             bool aborted = false;
-            for (int r = 0; r < nr; ++r) {
-                // (every lane polls; the answer is made warp-wide before the aligned MMAs)
-                if (!__all_sync(0xffffffffu,
-                                mbar_wait(full_s + 8u * slot, par, abort_flag, p.ws))) {
-                    aborted = true;
-                    break;
-                }
-                if (r < len) {
-                    const uint8_t* rec = ring + (size_t)slot * SLOT + (size_t)warp * RB;
-                    const int g = sg.g0 + i;
-                    // B fragments: x of batch row bl of the record's group (rows 32c .. 32c +
-                    // 31 of the group) for the lanes of the MMA columns of block record gi,
-                    // zeros for the other columns.
-                    const uint4* xsrc =
-                        gil == gi && bl < M ? xs + 16 * (bl * XR + sg.xg + g) + 4 * c : zblk;
-                    uint32_t B[8][2];
-#pragma unroll
-                    for (int qq = 0; qq < 4; ++qq) {
-                        const uint4 v = xsrc[qq];
-                        B[2 * qq][0] = v.x;
-                        B[2 * qq][1] = v.y;
-                        B[2 * qq + 1][0] = v.z;
-                        B[2 * qq + 1][1] = v.w;
+            for (int k = k0; k < k1 && !aborted; ++k) {
+                const Seg sg = segs[k];
+                float y[4] = {0.f, 0.f, 0.f, 0.f};
+                for (int i = 0; i < sg.ng; i += GPA) {
+                    const int bn = sg.ng - i < GPA ? sg.ng - i : GPA;
+                    if (!wait_rounds(full_s, q, bn, NS, abort_flag, p.ws)) {
+                        aborted = true;
+                        break;
                     }
-                    uint32_t wd[WPL];
-                    const uint4 c0 = *reinterpret_cast<const uint4*>(rec + lane * 16);
-                    wd[0] = c0.x; wd[1] = c0.y; wd[2] = c0.z; wd[3] = c0.w;
-                    if constexpr (BITS == 4) {
-                        const uint4 c1 = *reinterpret_cast<const uint4*>(rec + 512 + lane * 16);
-                        wd[4] = c1.x; wd[5] = c1.y; wd[6] = c1.z; wd[7] = c1.w;
+                    const int gb = sg.xg + sg.g0 + i;  // the block's first group in the X area
+                    // B fragments of this lane: x of batch row bl of block record gil (rows
+                    // 32c .. 32c + 31 of its group) when that record exists, else zeros
+                    const uint4* xrow =
+                        gil < bn && bl < M ? xs + 16 * (bl * XR + gb + gil) + 4 * c : zblk;
+                    float D[4][4];
+#pragma unroll
+                    for (int v = 0; v < 4; ++v) D[0][v] = D[1][v] = D[2][v] = D[3][v] = 0.f;
+                    if (bn == GPA) {
+                        int sl = q.slot;
+#pragma unroll
+                        for (int gi = 0; gi < GPA; ++gi) {
+                            pass_record<BITS>(ring + (size_t)sl * SLOT + (size_t)warp * RB,
+                                              gil == gi ? xrow : zblk, p.exps, D, lane);
+                            if (++sl == NS) sl = 0;
+                        }
                     } else {
-                        const uint2 c1 = *reinterpret_cast<const uint2*>(rec + 512 + lane * 8);
-                        wd[4] = c1.x; wd[5] = c1.y;
-                    }
-                    uint32_t a[8][4];
-                    extract<BITS>(wd, p.exps, a);
-#pragma unroll
-                    for (int j = 0; j < 8; ++j)
-                        mma16816(D[j & 3], a[j][0], a[j][1], a[j][2], a[j][3], B[j][0], B[j][1]);
-                    // The lanes whose accumulator columns 2c, 2c + 1 include block record gi
-                    // keep its scale and zero pairs of their output rows R, R + 8 (converted in
-                    // the epilogue).
-                    const bool u0 = (2 * c) % GPA == gi, u1 = (2 * c + 1) % GPA == gi;
-                    if (u0 || u1) {
-                        const uint32_t sr = reinterpret_cast<const uint32_t*>(rec + RBC)[R];
-                        const uint32_t zr = reinterpret_cast<const uint16_t*>(rec + RBC + 32)[R];
-                        if (u1) {
-                            sw[1] = sr;
-                            zw[1] = zr;
-                        } else {
-                            sw[0] = sr;
-                            zw[0] = zr;
+                        int sl = q.slot;
+                        for (int gi = 0; gi < bn; ++gi) {
+                            pass_record<BITS>(ring + (size_t)sl * SLOT + (size_t)warp * RB,
+                                              gil == gi ? xrow : zblk, p.exps, D, lane);
+                            if (++sl == NS) sl = 0;
                         }
                     }
-                    ++i;
-                    if (gi == GPA - 1 || i == sg.ng) {
-                        // Block epilogue (Eq. (1)): value v is output row R + 8 (v >> 1) and
-                        // MMA column col = 2c + (v & 1): batch row col / GPA, block record
-                        // col % GPA.
-                        const int gb = sg.xg + sg.g0 + i - 1 - gi;  // the block's first group
-#pragma unroll
-                        for (int v = 0; v < 4; ++v) {
-                            const int col = 2 * c + (v & 1);
-                            const int b = col / GPA, giv = col % GPA;
-                            if (giv <= gi && b < M) {
-                                const float2 spv = sp[b * XR + gb + giv];  // (S, P)
-                                const float dv = (D[0][v] + D[1][v]) + (D[2][v] + D[3][v]);
-                                const float sc = __half2float(__ushort_as_half(
-                                    (uint16_t)(sw[v & 1] >> (16 * (v >> 1)))));
-                                const float zc = (float)((zw[v & 1] >> (8 * (v >> 1))) & 0xffu);
-                                y[v] = fmaf(sc, dv - spv.y - zc * spv.x, y[v]);
-                            }
-                            D[0][v] = D[1][v] = D[2][v] = D[3][v] = 0.f;
-                        }
-                        gi = 0;
-                    } else {
-                        ++gi;
-                    }
-                    if (i == sg.ng) {
-                        // Segment end: a lane's two columns belong to one batch row (c / LPB);
-                        // its LPB lanes of the output row add up, and slot (k, b) gets the 16
-                        // outputs of batch row b.
-                        float lo = y[0] + y[1], hi = y[2] + y[3];
-#pragma unroll
-                        for (int o = 1; o < LPB; o <<= 1) {
-                            lo += __shfl_xor_sync(0xffffffffu, lo, o);
-                            hi += __shfl_xor_sync(0xffffffffu, hi, o);
-                        }
-                        const int b = c / LPB;
-                        if (c % LPB == 0 && b < M) {
-                            slots[16 * (k * MP + b) + R] = lo;
-                            slots[16 * (k * MP + b) + R + 8] = hi;
-                        }
-#pragma unroll
-                        for (int v = 0; v < 4; ++v) y[v] = 0.f;
-                        ++k;
-                        i = 0;
-                        if (k < k1) sg = segs[k];
-                    }
+                    pass_epilogue<BITS, MP>(ring, q.slot, NS, warp, lane, bn, M, XR, sp + gb, D,
+                                            y);
+                    release_rounds(empty_s, q, bn, NS, lane);
                 }
-                __syncwarp();
-                if (lane == 0) mbar_arrive(empty_s + 8u * slot);
-                if (++slot == NS) {
-                    slot = 0;
-                    par ^= 1u;
+                if (aborted) break;
+                // Segment end: a lane's two columns belong to one batch row (c / LPB); its LPB
+                // lanes of the output row add up, and slot (k, b) gets the 16 outputs of batch
+                // row b.
+                float lo = y[0] + y[1], hi = y[2] + y[3];
+#pragma unroll
+                for (int o = 1; o < LPB; o <<= 1) {
+                    lo += __shfl_xor_sync(0xffffffffu, lo, o);
+                    hi += __shfl_xor_sync(0xffffffffu, hi, o);
+                }
+                const int b = c / LPB;
+                if (c % LPB == 0 && b < M) {
+                    slots[16 * (k * MP + b) + R] = lo;
+                    slots[16 * (k * MP + b) + R + 8] = hi;
                 }
             }
+            // the stage's last round, when it holds no record of this warp
+            if (!aborted && len < nr) {
+                if (wait_rounds(full_s, q, 1, NS, abort_flag, p.ws))
+                    release_rounds(empty_s, q, 1, NS, lane);
+                else
+                    aborted = true;
+            }
+            pos = q;
             if (cbar_any(aborted || *abort_flag)) return;
 
             // The SM's tiles of the stage: each output is its segments' slots summed in order.
-            for (int idx = tid; idx < nt * M * 16; idx += 512) {
-                const int lt = idx / (M * 16), b = (idx >> 4) - lt * M, col = idx & 15;
-                const LTile t = tiles[lt];
-                float acc = 0.f;
-                for (int q = 0; q < t.nslot; ++q) acc += slots[16 * ((t.slot0 + q) * MP + b) + col];
-                t.y[(size_t)b * t.ldy + col] = __half_as_ushort(__float2half_rn(acc));
+            for (int b = 0; b < M; ++b) {
+                for (int idx = tid; idx < nt * 16; idx += 512) {
+                    const int lt = idx >> 4, col = idx & 15;
+                    const LTile t = tiles[lt];
+                    float acc = 0.f;
+                    for (int qq = 0; qq < t.nslot; ++qq)
+                        acc += slots[16 * ((t.slot0 + qq) * MP + b) + col];
+                    t.y[(size_t)b * t.ldy + col] = __half_as_ushort(__float2half_rn(acc));
+                }
             }
             cbar();
         }
-        if (tid == 0) st_rel(p.ws + 2 + blockIdx.x, (uint32_t)(s + 1));  // after its Y stores
+        // the stage is complete here once its Y stores are (release: ordered after them)
+        if (tid == 0) red_rel_add(p.ws + kCounterStride * (1 + s % kCounters), 1u);
     }
 }
 
@@ -877,6 +1004,7 @@ __global__ void __launch_bounds__(kPThreads, 1) pass_kernel(const PassParams p) 
     const uint32_t full_s = base + (uint32_t)L.bar;
     const uint32_t empty_s = full_s + 8u * kMaxRing;
     volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L.flag);
+    volatile int* cur_stage = abort_flag + 1;  // the last stage whose dependency is met
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < p.ns; ++i) {
@@ -885,6 +1013,7 @@ __global__ void __launch_bounds__(kPThreads, 1) pass_kernel(const PassParams p) 
         }
         // an error recorded by an earlier call: the call does nothing
         *abort_flag = ld_rlx(p.ws) != 0u ? 1 : 0;
+        *cur_stage = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     if (threadIdx.x < 4)
@@ -895,17 +1024,17 @@ __global__ void __launch_bounds__(kPThreads, 1) pass_kernel(const PassParams p) 
     if (*abort_flag) {
         // no copy is issued, no stage runs, and the workspace stays as it is
     } else if (warp == kPW)
-        pass_producer<BITS>(p, sd, base, full_s, empty_s, abort_flag, lane);
+        pass_producer<BITS>(p, sd, base, full_s, empty_s, abort_flag, cur_stage, lane);
     else
-        pass_consumer<BITS, MP>(p, smem, L, full_s, empty_s, abort_flag, warp, lane);
+        pass_consumer<BITS, MP>(p, smem, L, full_s, empty_s, abort_flag, cur_stage, warp, lane);
     __syncthreads();
 
-    // The last CTA to finish (every other one has made its last flag read) zeroes the flags
-    // for the next call on the stream.
+    // The last CTA to finish (every other one has made its last counter read) zeroes the
+    // counters for the next call on the stream.
     if (threadIdx.x == 0 && *abort_flag == 0) {
         const uint32_t done = atom_acq_rel_add(p.ws + 1, 1u);
         if (done == gridDim.x - 1) {
-            for (unsigned j = 0; j < gridDim.x; ++j) p.ws[2 + j] = 0u;
+            for (int j = 0; j < kCounters; ++j) p.ws[kCounterStride * (1 + j)] = 0u;
             p.ws[1] = 0u;
         }
     }
@@ -1052,7 +1181,8 @@ laq_status laq_pass_run(const void* plan, const void* device, void* workspace,
     while (ns >= 2 &&
            pass_smem(h->rb, ns, h->xs_bytes, h->max_segs, h->max_nx, mp).total > optin)
         --ns;
-    if (ns < 2) return LAQ_ERR_SHAPE;
+    // a warp holds the rounds of one block (8 / MP records) at once, in distinct slots
+    if (ns < 8 / mp) return LAQ_ERR_SHAPE;
     const PassSmem L = pass_smem(h->rb, ns, h->xs_bytes, h->max_segs, h->max_nx, mp);
 
     const uint8_t* dev = static_cast<const uint8_t*>(device);

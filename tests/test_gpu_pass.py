@@ -131,8 +131,9 @@ def test_plan_for_another_sm_count_is_rejected():
     sms = torch.cuda.get_device_properties(0).multi_processor_count
     plan, dev_bytes = _lib.pass_plan(chain.array, 1, sms - 1)
     buf = torch.empty((dev_bytes,), dtype=torch.uint8, device="cuda")
-    ws = torch.zeros((256,), dtype=torch.uint8, device="cuda")
-    st = _lib.lib().laq_pass_run(plan, _lib._ptr(buf), _lib._ptr(ws), 256, _lib._stream(None))
+    nws = int(_lib.lib().laq_pass_workspace_bytes(plan))
+    ws = torch.zeros((nws,), dtype=torch.uint8, device="cuda")
+    st = _lib.lib().laq_pass_run(plan, _lib._ptr(buf), _lib._ptr(ws), nws, _lib._stream(None))
     assert st == 9                                  # LAQ_ERR_CONFIG, nothing launched
 
 

@@ -394,7 +394,7 @@ def test_plan_buffer_and_run_arguments(L):
     plan, dev = _lib.pass_plan(arr, 2, 8)
     assert dev == db.value
     ws = int(L.laq_pass_workspace_bytes(plan))
-    assert ws == 256                       # status, finished count, 2 stage counters
+    assert ws == 1280                      # status and finished count, 8 stage counters (lines)
     junk = (ctypes.c_uint8 * 512)()
     assert L.laq_pass_workspace_bytes(junk) == 0
     assert L.laq_pass_workspace_bytes(None) == 0
@@ -413,7 +413,7 @@ def test_plan_buffer_and_run_arguments(L):
     # an empty chain plans to nothing and runs as a no-op
     empty, dev0 = _lib.pass_plan(fake_entries([]), 0, 8)
     assert parse(empty)["h"]["nstages"] == 0 and parse(empty)["h"]["records"] == 0
-    assert L.laq_pass_run(empty, D, WS, 256, None) == 0
+    assert L.laq_pass_run(empty, D, WS, L.laq_pass_workspace_bytes(empty), None) == 0
 
 
 def test_segment_limit_per_sm_stage(L):
