@@ -2,15 +2,19 @@
 
 One step = one replay of a CUDA graph holding every quantized projection of the model once
 (36 layers x q, k, v, o, gate, up, down, M = 1), i.e. the weight streaming of one batch-1
-decode step.  The pass has four equivalent forms (252 ``laq_gemm_wxg128`` launches; 144 with
-q|k|v and gate|up fused over concatenated columns; one persistent ``laq_gemm_chain`` launch of
-either list); each is timed briefly and the fastest gets the full timed run.  Quantization and packing (``laq_quantize_rtn``,
-``laq_pack``) are the offline model-preparation steps and run once before timing; their time is
-reported as ``prep_ms``.  Synthetic weights ~ N(0, 0.02^2) and activations ~ N(0, 1) stand in
-for the paper's Qwen3 checkpoints.
+decode step.  The pass has equivalent forms (252 ``laq_gemm_wxg128`` launches; 144 with q|k|v
+and gate|up fused over concatenated columns; one persistent ``laq_pass_run`` launch over per-SM
+weight streams); each is timed briefly and the fastest gets the full timed run.  Quantization
+and packing (``laq_quantize_rtn``, ``laq_pack``) are the offline model-preparation steps and run
+once before timing; their time is reported as ``prep_ms``.  Synthetic weights ~ N(0, 0.02^2)
+and activations ~ N(0, 1) stand in for the paper's Qwen3 checkpoints.
 
 Prints one JSON line.  ``value`` is the achieved HBM bandwidth of the pass (algorithmic bytes =
 packed codes + s + z + X + Y, per step, all ranks) over the device time of the timed replays.
+Unless ``--no-sweep``, the line also carries ``sweep``: the other measured workloads (one
+1024 x 1024 GEMV, each projection of a Qwen3-4B layer, the Qwen3-4B pass at W3 and W4 for
+M = 1, 2, 4, 8, 16, the Qwen3-8B pass with outliers at M = 1 and 16, and a whole decode step
+with and without an online rotation), each timed on its own after the headline.
 
     python bench.py [--steps K] [--warmup W] [--model qwen3-4b|qwen3-8b] [--bits 3|4] [--M 1]
     python bench.py --impl reference      # the CPU oracle, timed on the host cores
@@ -43,6 +47,7 @@ def parse():
     ap.add_argument("--M", type=int, default=1)
     ap.add_argument("--layers", type=int, default=36)
     ap.add_argument("--no-fp16", action="store_true", help="skip the fp16 torch.matmul context")
+    ap.add_argument("--no-sweep", action="store_true", help="skip the other workloads")
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
                     help="CPU work budget of the oracle baseline sample")
     return ap.parse_args()
@@ -50,7 +55,39 @@ def parse():
 
 def workload_name(a):
     return (f"{a.model} decode-step weight pass, {a.layers} layers x 7 projections, "
-            f"W{a.bits}G128, M={a.M}, one CUDA graph")
+            f"W{a.bits}G128, M={a.M}")
+
+
+def workload_config(a):
+    """The ``config`` of both arms: the same workload."""
+    return {"workload": workload_name(a), "bits": a.bits, "M": a.M, "layers": a.layers,
+            "shapes": a.model,
+            "l2": "inputs larger than L2 (packed weights per step >> 129 MB)"}
+
+
+def host_cpu():
+    """(CPU model name, cores available to this process)."""
+    name = None
+    try:
+        with open("/proc/cpuinfo") as f:
+            for line in f:
+                k, _, v = line.partition(":")
+                if k.strip() in ("model name", "Model Name", "CPU part") and v.strip():
+                    name = v.strip()
+                    if k.strip() != "CPU part":
+                        break
+    except OSError:
+        pass
+    if name is None or name.startswith("0x"):
+        try:
+            out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+            for line in out.splitlines():
+                if line.split(":")[0].strip() == "Model name":
+                    name = line.split(":", 1)[1].strip()
+                    break
+        except (OSError, subprocess.SubprocessError):
+            pass
+    return name or "unknown", len(os.sched_getaffinity(0))
 
 
 def load_peaks():
@@ -218,8 +255,9 @@ class OracleSample:
     def nbytes(self, K, N):
         return K * N * self.bits // 8 + (K // 128) * N * 3 + 2 * self.M * K + 2 * self.M * N
 
-    def run(self, seconds, max_cols=None):
-        """Oracle work for about ``seconds``; returns (bytes, seconds spent, items done)."""
+    def run(self, seconds, max_cols=None, threaded=False):
+        """Oracle work for about ``seconds`` (``threaded``: the all-cores GEMM, its output
+        columns split over the host's threads); returns (bytes, seconds spent, items done)."""
         done = 0
         spent = 0.0
         names = []
@@ -233,7 +271,7 @@ class OracleSample:
                 N = max_cols
                 name += f"[:, :{N}]"
             t0 = time.perf_counter()
-            self.co.gemm(X, codes, s, z)
+            (self.co.gemm_threads if threaded else self.co.gemm)(X, codes, s, z)
             spent += time.perf_counter() - t0
             done += self.nbytes(K, N)
             names.append(name)
@@ -246,39 +284,44 @@ class OracleSample:
 
 
 def run_reference(a, world, rank):
-    """The oracle, as it stands, on the host cores: each step is a bounded sample of the pass
-    (a column slice of one projection, sized so the whole run stays within a few minutes)."""
+    """The oracle, as it stands, on the host cores (its all-cores GEMM): each step is a bounded
+    sample of the pass (a column slice of one layer-0 projection, sized so the whole run stays
+    within a few minutes)."""
     if rank != 0:
         return
     smp = OracleSample(a.model, a.bits, a.M)
+    cpu_name, avail = host_cpu()
     per_step_s = min(0.25, max(0.002, 90.0 / max(1, a.steps + a.warmup)))
     # calibrate columns per step on the first projection
     name, codes, *_ = smp.items[0]
     K, N = codes.shape
-    b, sp, _ = smp.run(0.0, max_cols=64)
-    cols = int(max(16, min(N, 64 * per_step_s / max(sp, 1e-6))) // 16 * 16)
+    b, sp, _ = smp.run(0.0, max_cols=256, threaded=True)
+    cols = int(max(64, min(N, 256 * per_step_s / max(sp, 1e-6))) // 64 * 64)
     smp.next = 0
     for _ in range(a.warmup):
-        smp.run(0.0, max_cols=cols)
+        smp.run(0.0, max_cols=cols, threaded=True)
     tot_b, tot_s, names = 0, 0.0, []
     step_s = []
     for _ in range(a.steps):
-        b, sp, nm = smp.run(0.0, max_cols=cols)
+        b, sp, nm = smp.run(0.0, max_cols=cols, threaded=True)
         tot_b += b
         tot_s += sp
         step_s.append(sp)
         names += nm
     value = tot_b / tot_s / 1e9
-    sample = (f"C oracle (fp64, one thread) dequantize-and-multiply; each step = the first "
-              f"{cols} columns of one layer-0 projection, round-robin over q,k,v,o,gate,up,down; "
-              f"{tot_s:.1f} s of CPU work over {a.steps} steps; quantization not timed")
+    threads = smp.co.threads()
+    sample = (f"C oracle (fp64) dequantize-and-multiply, output columns split over {threads} "
+              f"threads; each step = the first {cols} columns of one layer-0 projection, "
+              f"round-robin over q,k,v,o,gate,up,down; {tot_s:.1f} s of CPU work over "
+              f"{a.steps} steps; quantization not timed; host CPU {cpu_name}, {avail} cores "
+              f"available")
     line = {"metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": a.gpus,
             "steps": a.steps, "warmup": a.warmup,
             "ms_per_step": 1e3 * statistics.median(step_s), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "impl": "reference", "config": {"workload": workload_name(a), "model": a.model},
-            "cpu_baseline": {"value": value, "unit": "GB/s", "cores": 1, "kind": "oracle",
-                             "sample": sample},
+            "impl": "reference", "config": workload_config(a),
+            "cpu_baseline": {"value": value, "unit": "GB/s", "cores": threads, "kind": "oracle",
+                             "cpu": cpu_name, "sample": sample},
             "e2e": {"value": value, "unit": "GB/s", "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
@@ -375,31 +418,186 @@ def kernel_breakdown(wp, stream, dev, reps=200):
 
 
 VARIANTS = {
-    # name: (fused q|k|v and gate|up, one persistent laq_gemm_chain launch)
-    "graph_252": (False, False),
-    "graph_fused": (True, False),
-    "chain_252": (False, True),
-    "chain_fused": (True, True),
+    # name: (fused q|k|v and gate|up, form): "graph" = one laq_gemm_wxg128 launch per GEMV in a
+    # CUDA graph (PDL), "planned" = one persistent laq_pass_run launch (M <= 4)
+    "graph_252": (False, "graph"),
+    "graph_fused": (True, "graph"),
+    "planned_fused": (True, "planned"),
 }
 
 
 def describe(name, wp):
-    fused, chain = VARIANTS[name]
+    fused, form = VARIANTS[name]
     what = ("252 projections as 144 GEMVs (q|k|v and gate|up over concatenated columns, "
             "identical per-column codes and results)" if fused else "252 GEMVs")
-    how = ("one persistent laq_gemm_chain launch (stages q|k|v -> o -> gate|up -> down)"
-           if chain else f"{wp.launches} laq_gemm_wxg128 launches in one CUDA graph (PDL)")
+    how = ("one persistent laq_pass_run launch over per-SM weight streams (stages q|k|v -> o -> "
+           "gate|up -> down)" if form == "planned"
+           else f"{wp.launches} laq_gemm_wxg128 launches in one CUDA graph (PDL)")
     return f"{what}, {how}"
 
 
-def build_pass(a, dev, name):
+def build_pass(a, dev, name, model=None, bits=None, M=None):
     from paper_2605_08755_gb300.weight_pass import WeightPass
-    fused, chain = VARIANTS[name]
-    chain = chain and a.M <= 4
-    if VARIANTS[name][1] and not chain:
+    model = model or a.model
+    bits = bits or a.bits
+    M = M or a.M
+    fused, form = VARIANTS[name]
+    if form == "planned" and M > 4:
         return None
-    return WeightPass(model=a.model, bits=a.bits, M=a.M, layers=a.layers,
-                      outliers=(a.model == "qwen3-8b"), device=dev, fuse=fused, chain=chain)
+    return WeightPass(model=model, bits=bits, M=M, layers=a.layers,
+                      outliers=(model == "qwen3-8b"), device=dev, fuse=fused,
+                      planned=(form == "planned"))
+
+
+def pass_status_ok(wp):
+    return wp.plan.status() == 0 if wp.planned else True
+
+
+# ------------------------------------------------------------------ the other workloads
+
+
+def sweep_gemv_1024(a, dev, stream):
+    """One 1024 x 1024 W3G128 GEMV at M = 1 (421,888 algorithmic bytes, L2-resident on its
+    own): timed over 640 distinct copies (270 MB, more than twice L2) launched back to back in
+    one CUDA graph, so each launch reads its weights from HBM."""
+    import torch
+
+    from paper_2605_08755_gb300 import _lib, inputs
+    K = N = 1024
+    copies = 640
+    W = inputs.weights_torch(K, N, 1, dev)
+    codes, s_, z_ = _lib.laq_quantize_rtn(W, 3)
+    packed = _lib.laq_pack(codes, 3)
+    P = packed.repeat(copies).view(copies, -1)
+    S = s_.repeat(copies, 1).view(copies, *s_.shape)
+    Z = z_.repeat(copies, 1).view(copies, *z_.shape)
+    X = inputs.activations_torch(1, K, 1, dev)
+    Y = torch.empty((copies, 1, N), dtype=torch.float16, device=dev)
+    cfg = _lib.laq_gemm_plan(1, K, N, 3, torch.cuda.get_device_properties(dev).multi_processor_count)
+    cfg.pdl = 1
+
+    def run(st=None):
+        for i in range(copies):
+            _lib.laq_gemm_wxg128(X, P[i], S[i], Z[i], 3, Y=Y[i], config=cfg, stream=st)
+    run()
+    torch.cuda.synchronize(dev)
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        run(stream)
+    ms = min(time_graph(g, stream, 20, dev) for _ in range(2))
+    us = ms * 1e3 / copies
+    nbytes = K * N * 3 // 8 + (K // 128) * N * 3 + 2 * K + 2 * N
+    del g, P, S, Z, Y
+    return {"us_per_gemv": us, "gbs": nbytes / (us * 1e-6) / 1e9, "bytes_per_gemv": nbytes,
+            "l2": f"{copies} distinct copies per replay ({copies * nbytes / 1e6:.0f} MB)",
+            "launch": "back to back in one CUDA graph, PDL"}
+
+
+def sweep_layer_projections(a, dev, stream):
+    """Each projection of a Qwen3-4B layer (W3G128, M = 1): a CUDA graph of that projection's
+    36 launches of the 36-layer pass (36 distinct weights, HBM-cold), µs per GEMV."""
+    import torch
+
+    from paper_2605_08755_gb300 import _lib
+    wp = build_pass(a, dev, "graph_252", model="qwen3-4b", bits=3, M=1)
+    out = {}
+    for name in ("q", "k", "v", "o", "gate", "up", "down"):
+        idx = [i for i, (_, _, nm, _) in enumerate(wp.linears) if nm == name]
+
+        def run(st=None, idx=idx):
+            for i in idx:
+                q = wp.linears[i][3]
+                _lib.laq_gemm_wxg128(wp.X[i], q.packed, q.s, q.z, q.bits, Y=wp.Y[i],
+                                     config=wp.configs[i], stream=st)
+        run()
+        torch.cuda.synchronize(dev)
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            run(stream)
+        ms = min(time_graph(g, stream, 50, dev) for _ in range(2))
+        us = ms * 1e3 / len(idx)
+        q = wp.linears[idx[0]][3]
+        nb = q.bytes_per_call(1)
+        out[name] = {"K": q.K, "N": q.N, "us_per_gemv": us, "gbs": nb / (us * 1e-6) / 1e9}
+        del g
+    del wp
+    torch.cuda.empty_cache()
+    return out
+
+
+def sweep_pass(a, dev, stream, model, bits, M, variants):
+    """A whole decode-step weight pass in each form of ``variants``: µs per pass and GB/s."""
+    import torch
+    res = {}
+    for name in variants:
+        wp = build_pass(a, dev, name, model=model, bits=bits, M=M)
+        if wp is None:
+            continue
+        g = wp.capture(stream=stream)
+        ms = min(time_graph(g, stream, 30, dev) for _ in range(2))
+        if not pass_status_ok(wp):
+            raise RuntimeError(f"{name}: device-side error")
+        res[name] = {"us_per_pass": ms * 1e3,
+                     "gbs": wp.bytes_per_pass() / (ms * 1e-3) / 1e9}
+        del g, wp
+        torch.cuda.empty_cache()
+    best = min(res, key=lambda n: res[n]["us_per_pass"])
+    return {"best": best, "us_per_pass": res[best]["us_per_pass"], "gbs": res[best]["gbs"],
+            "variants": res}
+
+
+def sweep_decode_step(a, dev, stream, rounds):
+    """A whole Qwen3-4B decode step (W3G128, M = 1, context 2048) on the library's kernels, and
+    the same step with an online pairwise rotation of ``rounds`` rounds before every projection
+    (the rotation-based comparison): µs and tokens per second."""
+    import torch
+
+    from paper_2605_08755_gb300.decode_case import time_graph as tg
+    from paper_2605_08755_gb300.decode_step import DecodeStep
+    out = {}
+    for label, rot in (("laquant", 0), (f"rotated_{rounds}_rounds", rounds)):
+        st = DecodeStep(model="qwen3-4b", bits=3, M=1, context=2048, rotation_rounds=rot)
+        g = st.capture(stream=stream)
+        us = tg(g, stream, 30)
+        out[label] = {"us_per_token": us, "tokens_per_s": 1e6 / us, "launches": st.launches}
+        del g, st
+        torch.cuda.empty_cache()
+    out["faster_without_rotation"] = (out[f"rotated_{rounds}_rounds"]["us_per_token"]
+                                      / out["laquant"]["us_per_token"] - 1.0)
+    return out
+
+
+def run_sweep(a, dev, stream):
+    """The workloads besides the headline, each on its own; a failing item records its error."""
+    sweep = {}
+    items = [
+        ("gemv_1024x1024_w3_m1", lambda: sweep_gemv_1024(a, dev, stream)),
+        ("qwen3_4b_layer_w3_m1_per_projection", lambda: sweep_layer_projections(a, dev, stream)),
+    ]
+    for bits in (3, 4):
+        for M in (1, 2, 4, 8, 16):
+            items.append((f"qwen3_4b_pass_w{bits}_m{M}",
+                          lambda bits=bits, M=M: sweep_pass(
+                              a, dev, stream, "qwen3-4b", bits, M,
+                              ["graph_fused", "planned_fused"])))
+    for M in (1, 16):
+        items.append((f"qwen3_8b_outliers_pass_w3_m{M}",
+                      lambda M=M: sweep_pass(a, dev, stream, "qwen3-8b", 3, M,
+                                             ["graph_fused", "planned_fused"])))
+    items.append(("qwen3_4b_decode_step_w3_m1", lambda: sweep_decode_step(a, dev, stream, 8)))
+    t_all = time.perf_counter()
+    for name, fn in items:
+        t0 = time.perf_counter()
+        try:
+            sweep[name] = fn()
+        except Exception as e:  # noqa: BLE001 - recorded, the headline stands
+            sweep[name] = {"error": f"{type(e).__name__}: {e}"[:300]}
+        sweep[name]["wall_s"] = round(time.perf_counter() - t0, 2)
+    sweep["wall_s"] = round(time.perf_counter() - t_all, 2)
+    return sweep
+
+
+# ------------------------------------------------------------------ the headline
 
 
 def run_laq(a, world, rank, local):
@@ -427,6 +625,8 @@ def run_laq(a, world, rank, local):
             prep_ms = (time.perf_counter() - t0) * 1e3
         g = wp.capture(stream=stream)
         ms = min(time_graph(g, stream, max(20, min(a.steps, 300)), dev) for _ in range(2))
+        if not pass_status_ok(wp):
+            raise RuntimeError(f"{name}: laq_pass_run reported a device-side error")
         variants[name] = {"launches_per_step": wp.launches, "us_per_step": ms * 1e3,
                           "gbs": wp.bytes_per_pass() / (ms * 1e-3) / 1e9,
                           "what": describe(name, wp)}
@@ -459,16 +659,15 @@ def run_laq(a, world, rank, local):
     total_ms = max_over_ranks(world, starts[0].elapsed_time(ends[-1]), dev)
     ms_per_step = total_ms / a.steps
     value = sum_over_ranks(world, bytes_step * a.steps, dev) / (total_ms * 1e-3) / 1e9
-    if wp.chain:
-        from paper_2605_08755_gb300 import chain_status
-        if chain_status(wp.ws) != 0:
-            raise RuntimeError("laq_gemm_chain reported a device-side error")
+    if not pass_status_ok(wp):
+        raise RuntimeError("laq_pass_run reported a device-side error")
 
-    # The dominant kernel: the chain kernel itself, or the GEMV instance of the graph with the
-    # most device time (per-instance graphs of the step's launches, timed on their stream).
-    if wp.chain:
-        rows = [("chain_kernel<%d, %d>" % (a.bits, 1 if a.M <= 1 else 2 if a.M <= 2 else 4),
-                 1, bytes_step, ms_per_step * 1e3, None)]
+    # The dominant kernel: the persistent pass kernel itself, or the GEMV instance of the graph
+    # with the most device time (per-instance graphs of the step's launches, timed on their
+    # stream).
+    if wp.planned:
+        mp = 1 if a.M <= 1 else 2 if a.M <= 2 else 4
+        rows = [(f"pass_kernel<{a.bits}, {mp}>", 1, bytes_step, ms_per_step * 1e3, None)]
     else:
         rows = kernel_breakdown(wp, stream, dev)
     dom = max(rows, key=lambda r: r[3])
@@ -520,6 +719,8 @@ def run_laq(a, world, rank, local):
     stream.wait_stream(copy)
     e_b.record(stream)
     torch.cuda.synchronize(dev)
+    if not pass_status_ok(wp):
+        raise RuntimeError("laq_pass_run reported a device-side error")
     e2e_ms = max_over_ranks(world, e_a.elapsed_time(e_b), dev) / e2e_steps
     e2e_gbs = sum_over_ranks(world, bytes_step, dev) / (e2e_ms * 1e-3) / 1e9
     h2d, d2h = wp.Xbuf.numel() * 2, wp.Ybuf.numel() * 2
@@ -531,15 +732,26 @@ def run_laq(a, world, rank, local):
     if not a.no_fp16 and rank == 0:
         fp16_us, _ = fp16_context(a, dev)
 
+    sweep = None
+    if not a.no_sweep and rank == 0:
+        sweep = run_sweep(a, dev, stream)
+
     cpu = None
     if rank == 0:
         smp = OracleSample(a.model, a.bits, a.M)
-        b, spent, names = smp.run(a.cpu_seconds)
-        cpu = {"value": b / spent / 1e9, "unit": "GB/s", "cores": 1, "kind": "oracle",
-               "sample": f"C oracle (fp64, one thread) dequantize-and-multiply of "
-                         f"{len(names)} whole projections of layer 0, round-robin over "
-                         f"q,k,v,o,gate,up,down, {spent:.1f} s of CPU work; quantization not "
-                         f"timed"}
+        cpu_name, avail = host_cpu()
+        b1, s1, n1 = smp.run(min(4.0, a.cpu_seconds / 3))
+        smp.next = 0
+        b, spent, names = smp.run(a.cpu_seconds, threaded=True)
+        threads = smp.co.threads()
+        cpu = {"value": b / spent / 1e9, "unit": "GB/s", "cores": threads, "kind": "oracle",
+               "cpu": cpu_name, "cores_available": avail,
+               "single_thread_value": b1 / s1 / 1e9,
+               "sample": f"C oracle (fp64) dequantize-and-multiply, output columns split over "
+                         f"{threads} threads, of {len(names)} whole projections of layer 0, "
+                         f"round-robin over q,k,v,o,gate,up,down, {spent:.1f} s of wall time "
+                         f"(single-threaded: {len(n1)} projections in {s1:.1f} s); "
+                         f"quantization not timed"}
 
     if rank != 0:
         return
@@ -549,21 +761,20 @@ def run_laq(a, world, rank, local):
         "warmup": a.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None,
         "dtype": f"u{a.bits} codes + fp16 (fp32 accumulate)", "data": "synthetic",
-        "config": {"workload": workload_name(a) + ": " + variants[head]["what"],
-                   "model": a.model, "bits": a.bits, "M": a.M, "pass_variant": head,
-                   "launches_per_step": launches, "bytes_per_step": bytes_step,
-                   "us_per_step": ms_per_step * 1e3,
-                   "pct_of_peak": 100.0 * value / world / peak,
-                   "peak_gbs": peak, "peak_kind": peak_kind,
-                   "l2": "inputs larger than L2 (packed weights per step >> 129 MB)",
-                   "step_ms_p10_p50_p90": [pct(0.1), pct(0.5), pct(0.9)],
-                   "prep_ms": prep_ms,
-                   "variants_us_per_step": {k: round(v["us_per_step"], 1)
-                                            for k, v in variants.items()},
-                   "variants_gbs": {k: round(v["gbs"], 1) for k, v in variants.items()},
-                   "fp16_torch_matmul_us_per_step": fp16_us,
-                   "speedup_vs_fp16_torch": (fp16_us / (ms_per_step * 1e3)) if fp16_us else None,
-                   "parallelism": f"replicas x{world}"},
+        "config": workload_config(a),
+        "details": {"pass_variant": head, "what": variants[head]["what"],
+                    "launches_per_step": launches, "bytes_per_step": bytes_step,
+                    "us_per_step": ms_per_step * 1e3,
+                    "pct_of_peak": 100.0 * value / world / peak,
+                    "peak_gbs": peak, "peak_kind": peak_kind,
+                    "step_ms_p10_p50_p90": [pct(0.1), pct(0.5), pct(0.9)],
+                    "prep_ms": prep_ms,
+                    "variants_us_per_step": {k: round(v["us_per_step"], 1)
+                                             for k, v in variants.items()},
+                    "variants_gbs": {k: round(v["gbs"], 1) for k, v in variants.items()},
+                    "fp16_torch_matmul_us_per_step": fp16_us,
+                    "speedup_vs_fp16_torch": (fp16_us / (ms_per_step * 1e3)) if fp16_us else None,
+                    "parallelism": f"replicas x{world}"},
         "roofline": {"bound": "hbm", "achieved": kernel_gbs, "peak": peak, "unit": "GB/s",
                      "frac": kernel_gbs / peak, "traffic": traffic_for(dom[0], a, head, dom[4]),
                      "kernel": dom[0], "launches_per_step": dom[1],
@@ -577,6 +788,7 @@ def run_laq(a, world, rank, local):
                 "d2h_bytes_per_step": d2h, "us_per_step": e2e_ms * 1e3},
         "gpu_launches": launches * a.steps,
         "clocks": clocks,
+        "sweep": sweep,
     }
     print(json.dumps(line), flush=True)
 

@@ -25,6 +25,7 @@ def _lib():
         "laqo_dequant": [P, P, P, I64, I64, P],
         "laqo_gemm": [P, I64, I64, I64, P, P, P, P],
         "laqo_gemm_columns": [P, I64, I64, I64, P, P, P, P, I64, P],
+        "laqo_gemm_threads": [P, I64, I64, I64, P, P, P, P],
         "laqo_pack": [P, I64, I64, I, P],
         "laqo_unpack": [P, I64, I64, I, P],
         "laqo_layout_bit": [I, I, I, I, P, P, P],
@@ -33,6 +34,8 @@ def _lib():
         f = getattr(lib, name)
         f.argtypes = args
         f.restype = I
+    lib.laqo_threads.argtypes = []
+    lib.laqo_threads.restype = I
     lib.laqo_half_to_double.argtypes = [ctypes.c_uint16]
     lib.laqo_half_to_double.restype = ctypes.c_double
     lib.laqo_packed_words.argtypes = [I64, I64, I]
@@ -97,6 +100,23 @@ def gemm(X, codes, s, z):
     _check(_lib().laqo_gemm(_ptr(Xb), M, K, N, _ptr(codes), _ptr(_bits16(s)),
                             _ptr(np.ascontiguousarray(z)), _ptr(Y)), "laqo_gemm")
     return Y
+
+
+def gemm_threads(X, codes, s, z):
+    """``gemm`` with the output columns split over the host's threads (bit-identical)."""
+    Xb = _bits16(X)
+    M, K = Xb.shape
+    codes = np.ascontiguousarray(codes, np.uint8)
+    N = codes.shape[1]
+    Y = np.zeros((M, N), np.float64)
+    _check(_lib().laqo_gemm_threads(_ptr(Xb), M, K, N, _ptr(codes), _ptr(_bits16(s)),
+                                    _ptr(np.ascontiguousarray(z)), _ptr(Y)), "laqo_gemm_threads")
+    return Y
+
+
+def threads():
+    """Threads ``gemm_threads`` runs with (OMP_NUM_THREADS, else every available core)."""
+    return int(_lib().laqo_threads())
 
 
 def gemm_columns(X, codes, s, z, cols):

@@ -34,6 +34,9 @@
 #include <stdint.h>
 #include <stdlib.h>
 #include <string.h>
+#ifdef _OPENMP
+#include <omp.h>
+#endif
 
 #define LAQO_GROUP 128
 
@@ -152,6 +155,45 @@ int laqo_gemm(const uint16_t *X, int64_t M, int64_t K, int64_t N, const uint8_t 
         }
     }
     return 0;
+}
+
+/* laqo_gemm with the output columns split over the host's threads (OpenMP, when the oracle is
+ * built with it): every column is still its own k-ascending fp64 sum, so the result is
+ * laqo_gemm's bit for bit.  Used to time the oracle on all host cores. */
+int laqo_gemm_threads(const uint16_t *X, int64_t M, int64_t K, int64_t N, const uint8_t *codes,
+                      const uint16_t *s, const uint8_t *z, double *Y)
+{
+    if (M < 0 || K < 0 || N < 0 || K % LAQO_GROUP) return 4;
+    const int64_t cb = 64; /* columns per task */
+    const int64_t ntask = (N + cb - 1) / cb;
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int64_t t = 0; t < ntask; ++t) {
+        const int64_t n0 = t * cb, n1 = n0 + cb < N ? n0 + cb : N;
+        for (int64_t m = 0; m < M; ++m) {
+            double *y = Y + m * N;
+            for (int64_t n = n0; n < n1; ++n) y[n] = 0.0;
+            for (int64_t k = 0; k < K; ++k) {
+                double x = laqo_half_to_double(X[m * K + k]);
+                int64_t g = k / LAQO_GROUP;
+                for (int64_t n = n0; n < n1; ++n) {
+                    double w = laqo_half_to_double(s[g * N + n]) *
+                               (double)((int)codes[k * N + n] - (int)z[g * N + n]);
+                    y[n] += x * w;
+                }
+            }
+        }
+    }
+    return 0;
+}
+
+/* Threads the oracle runs laqo_gemm_threads with (1 without OpenMP). */
+int laqo_threads(void)
+{
+#ifdef _OPENMP
+    return omp_get_max_threads();
+#else
+    return 1;
+#endif
 }
 
 /* Same sum restricted to the listed output columns (for sampled checks of large layers). */

@@ -12,8 +12,6 @@ GOLDEN = os.path.join(ROOT, "tests", "golden")
 
 def pytest_configure(config):
     config.addinivalue_line("markers", "gpu: needs a CUDA GPU (sm_103a) and the built library")
-    config.addinivalue_line("markers", "pass_first_run: GPU tests of the planned pass (laq_pass_*) "
-                            "awaiting its first run on a GPU; selected only by name")
 
 
 def pytest_collection_modifyitems(config, items):
@@ -26,7 +24,7 @@ def pytest_collection_modifyitems(config, items):
         return
     skip = pytest.mark.skip(reason="no CUDA device")
     for item in items:
-        if "gpu" in item.keywords or "pass_first_run" in item.keywords:
+        if "gpu" in item.keywords:
             item.add_marker(skip)
 
 

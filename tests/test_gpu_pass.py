@@ -1,9 +1,8 @@
 """The planned pass (laq_pass_plan_build, laq_pass_prepare, laq_pass_run) against the oracle.
 
-Marked ``pass_first_run`` rather than ``gpu`` until the kernel's first runs on a GPU have
-passed: ``pytest -m pass_first_run`` selects them.  Every entry's Y must satisfy the GEMV
-tolerance against the oracle's fp64 product of the oracle's own codes, scales and zeros; chains
-with dependencies feed one entry's Y to the next entry as X, every Y pre-filled with NaN.
+Every entry's Y must satisfy the GEMV tolerance against the oracle's fp64 product of the oracle's
+own codes, scales and zeros; chains with dependencies feed one entry's Y to the next entry as X,
+every Y pre-filled with NaN.
 """
 import numpy as np
 import pytest
@@ -15,7 +14,7 @@ from paper_2605_08755_gb300.weight_pass import WeightPass
 from tests.test_gpu_chain import Lin, check_y, nan_like
 from tests.test_gpu_workloads import _sampled, check_projection
 
-pytestmark = pytest.mark.pass_first_run
+pytestmark = pytest.mark.gpu
 
 
 @pytest.fixture(scope="module", autouse=True)

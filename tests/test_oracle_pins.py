@@ -288,3 +288,13 @@ def test_bad_arguments_are_rejected():
         co.quantize_rtn(np.zeros((100, 16), np.float16), 3)
     with pytest.raises(ValueError):
         co.pack(np.zeros((128, 10), np.uint8), 3)
+
+
+@pytest.mark.parametrize("bits", [3, 4])
+def test_threaded_gemm_is_the_plain_gemm(bits):
+    """The oracle's all-cores GEMM (output columns split over threads, each column its own
+    k-ascending sum) equals the single-threaded definition bit for bit, on a ragged N."""
+    W = inputs.weights(384, 16 * 37 + 8, seed=bits)
+    X = inputs.activations(3, 384, seed=bits)
+    codes, s, z = co.quantize_rtn(W, bits)
+    assert np.array_equal(co.gemm_threads(X, codes, s, z), co.gemm(X, codes, s, z))
