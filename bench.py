@@ -48,6 +48,9 @@ def parse():
     ap.add_argument("--layers", type=int, default=36)
     ap.add_argument("--no-fp16", action="store_true", help="skip the fp16 torch.matmul context")
     ap.add_argument("--no-sweep", action="store_true", help="skip the other workloads")
+    ap.add_argument("--variant", default=None, choices=["graph_252", "graph_fused", "planned_fused"],
+                    help="time only this form of the pass (for profiling runs, where the "
+                         "profiler's serialised launches would change which form is fastest)")
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
                     help="CPU work budget of the oracle baseline sample")
     return ap.parse_args()
@@ -615,7 +618,7 @@ def run_laq(a, world, rank, local):
     # the headline and gets the full timed run below.
     variants = {}
     prep_ms = None
-    for name in VARIANTS:
+    for name in ([a.variant] if a.variant else VARIANTS):
         t0 = time.perf_counter()
         wp = build_pass(a, dev, name)
         if wp is None:

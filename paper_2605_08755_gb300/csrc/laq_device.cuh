@@ -106,9 +106,11 @@ inline Exps exps_for(int bits) {
 
 // Extract the A fragments of one record (one lane's words) into a[j][0..3] for the 8 k16 steps:
 // a0 = (row r, pair (j,0)), a1 = (row r+8, pair (j,0)), a2 = (row r, pair (j,1)),
-// a3 = (row r+8, pair (j,1)); each register holds 2^(10-p) + q for its two codes.  Right shifts
-// are multiplications by powers of two (high word), left shifts plain multiplications, so they
-// run on the FMA pipe beside the mask-and-or operations.
+// a3 = (row r+8, pair (j,1)); each register holds 2^(10-p) + q for its two codes.  Shifts are
+// plain shifts: on GB300 a shift issues at the mask-and-or rate (two warp instructions per SM
+// cycle), a multiply-high only at one, and the legacy MMA leaves half of the integer work's
+// issue slots unhidden, so the record loop from shared memory costs 42.2 SM cycles per W3
+// record with shifts against 45.8 with multiply-high shifts.
 template <int BITS>
 __device__ __forceinline__ void extract(const uint32_t (&wd)[BITS == 4 ? 8 : 6],
                                         const Exps& x, uint32_t (&a)[8][4]) {
@@ -116,7 +118,7 @@ __device__ __forceinline__ void extract(const uint32_t (&wd)[BITS == 4 ? 8 : 6],
         const uint32_t e0 = x.e[0], e4 = x.e[1];
 #pragma unroll
         for (int j = 0; j < 8; ++j) {
-            const uint32_t w = wd[j], t = __umulhi(w, 1u << 24);  // w >> 8
+            const uint32_t w = wd[j], t = w >> 8;
             a[j][0] = (w & 0x000f000fu) | e0;  // pair (j, 0, r)      p = 0
             a[j][2] = (w & 0x00f000f0u) | e4;  // pair (j, 1, r)      p = 4
             a[j][1] = (t & 0x000f000fu) | e0;  // pair (j, 0, r + 8)  p = 0
@@ -127,7 +129,7 @@ __device__ __forceinline__ void extract(const uint32_t (&wd)[BITS == 4 ? 8 : 6],
         uint32_t rp[16][2];
 #pragma unroll
         for (int w = 0; w < 6; ++w) {
-            const uint32_t u = __umulhi(wd[w], 1u << 23);       // w >> 9
+            const uint32_t u = wd[w] >> 9;
             rp[w][0] = (wd[w] & 0x000e000eu) | e1;              // bits 1-3    p = 1
             rp[6 + w][0] = (wd[w] & 0x00700070u) | e4;          // bits 4-6    p = 4
             rp[w][1] = (u & 0x000e000eu) | e1;                  // bits 10-12  p = 1
@@ -139,10 +141,10 @@ __device__ __forceinline__ void extract(const uint32_t (&wd)[BITS == 4 ? 8 : 6],
             rp[12 + q][1] = (wd[2 * q + 1] & 0x03800380u) | e7;
         }
         // pair 15: bit 0 of words 0,1,2 (row r) / 3,4,5 (row r+8) -> code bits 0,1,2 at p = 4
-        rp[15][0] = ((wd[0] * 16u) & 0x00100010u) | ((wd[1] * 32u) & 0x00200020u) |
-                    ((wd[2] * 64u) & 0x00400040u) | e4;
-        rp[15][1] = ((wd[3] * 16u) & 0x00100010u) | ((wd[4] * 32u) & 0x00200020u) |
-                    ((wd[5] * 64u) & 0x00400040u) | e4;
+        rp[15][0] = ((wd[0] << 4) & 0x00100010u) | ((wd[1] << 5) & 0x00200020u) |
+                    ((wd[2] << 6) & 0x00400040u) | e4;
+        rp[15][1] = ((wd[3] << 4) & 0x00100010u) | ((wd[4] << 5) & 0x00200020u) |
+                    ((wd[5] << 6) & 0x00400040u) | e4;
 #pragma unroll
         for (int j = 0; j < 8; ++j) {
             a[j][0] = rp[2 * j][0];

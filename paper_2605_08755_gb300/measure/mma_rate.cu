@@ -1,0 +1,313 @@
+// mma_rate.cu -- the tensor-core rates behind the choice of mma.sync for the WbG128 record loop.
+//
+// A record (16 output columns x 128 rows of K) is 2048 weights.  At M <= 16 one GEMV record
+// needs, on the legacy path, 8 mma.sync.m16n8k16 (A = the record's dequantized codes in
+// registers, B = x), and on the 5th-generation path one tcgen05.mma.kind::f16 of M = 128 rows
+// (8 records' worth of output columns x 16 rows of K: 2048 weights) with N = 16 columns of x.
+// This program measures, one CTA per SM on every SM:
+//   1. mma.sync.m16n8k16 (f16 in, f32 accumulate): cycles per MMA per SM with 16 warps of 8
+//      independent chains, and the dependent latency of one chain;
+//   2. tcgen05.mma.cta_group::1.kind::f16, M = 128, K = 16, N = 16..256, A and B from shared
+//      memory (no swizzle, K-major), D in tensor memory: cycles per instruction, one thread
+//      issuing 512 back to back (the operand values are irrelevant to the rate);
+//   3. the W3 record loop of laq_gemm_wxg128 / laq_pass_run from shared memory: the
+//      mask-and-or extraction of one record's codes and its 8 MMAs, 16 warps, cycles per record
+//      per SM (the HBM rate of GB300, 6.78 TB/s over 152 SMs at 2.07 GHz, is one 816-byte W3
+//      record per 38 SM cycles), with the field shifts as plain shifts (the library's form) and
+//      as multiply-high instructions;
+//   4. the issue rates behind it: mask-and-or (LOP3), shift, multiply-high, add, and how much
+//      integer work hides behind mma.sync.
+// Every wait is bounded.
+//
+//   nvcc -gencode arch=compute_103a,code=sm_103a -O3 -Xptxas -v -o /tmp/mma_rate \
+//       paper_2605_08755_gb300/measure/mma_rate.cu && /tmp/mma_rate
+#include <cuda_runtime.h>
+#include <stdint.h>
+#include <stdio.h>
+
+#include <algorithm>
+#include <vector>
+
+namespace {
+
+__device__ __forceinline__ unsigned long long clk() {
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %%clock64;" : "=l"(t));
+    return t;
+}
+
+__device__ __forceinline__ void mma16816(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2,
+                                         uint32_t a3, uint32_t b0, uint32_t b1) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
+        "{%8,%9}, {%0,%1,%2,%3};\n"
+        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+        : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+// 1. mma.sync: `chains` independent accumulators per warp, `iters` rounds of one MMA each.
+template <int CHAINS>
+__global__ void __launch_bounds__(512, 1) mma_sync_rate(int iters, unsigned long long* out,
+                                                        float* sink) {
+    float d[CHAINS][4] = {};
+    const uint32_t a = 0x3c003c00u ^ threadIdx.x, b = 0x3c003c00u;
+    __syncthreads();
+    const unsigned long long t0 = clk();
+    for (int i = 0; i < iters; ++i) {
+#pragma unroll
+        for (int c = 0; c < CHAINS; ++c) mma16816(d[c], a, a + c, a ^ c, a, b, b + i);
+    }
+    __syncthreads();
+    const unsigned long long t1 = clk();
+    float s = 0.f;
+#pragma unroll
+    for (int c = 0; c < CHAINS; ++c) s += d[c][0] + d[c][1] + d[c][2] + d[c][3];
+    if (s == 12345.f) sink[0] = s;
+    if (threadIdx.x == 0) out[blockIdx.x] = t1 - t0;
+}
+
+// 2. tcgen05.mma kind::f16, M = 128, K = 16, N = n, operands in shared memory.
+__device__ __forceinline__ uint64_t smem_desc(uint32_t addr, uint32_t lbo, uint32_t sbo) {
+    // start address, leading (K) and stride (M/N) byte offsets in 16-byte units, descriptor
+    // version 1 (bits 46-47), no swizzle (layout type 0)
+    return (uint64_t)((addr >> 4) & 0x3fffu) | ((uint64_t)((lbo >> 4) & 0x3fffu) << 16) |
+           ((uint64_t)((sbo >> 4) & 0x3fffu) << 32) | ((uint64_t)1 << 46);
+}
+
+__global__ void __launch_bounds__(128, 1) tc_rate(int n, int iters, unsigned long long* out,
+                                                  int* status) {
+    extern __shared__ __align__(1024) uint8_t sm[];
+    __shared__ __align__(8) uint64_t bar;
+    __shared__ uint32_t tmem_slot;
+    const int warp = threadIdx.x >> 5;
+    const uint32_t bar_s = (uint32_t)__cvta_generic_to_shared(&bar);
+    if (threadIdx.x == 0) {
+        asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(bar_s));
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    if (warp == 0) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], 256;" ::"r"(
+                         (uint32_t)__cvta_generic_to_shared(&tmem_slot))
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    const uint32_t tmem = tmem_slot;
+    if (threadIdx.x == 0) {
+        const uint32_t base = (uint32_t)__cvta_generic_to_shared(sm);
+        // A: 128 rows x 16 fp16 as 8x8 core matrices, K-adjacent 128 B apart, row groups 256 B
+        // apart (4 KB); B: n rows x 16 fp16 the same way, at +16 KB (at most 8 KB)
+        const uint64_t adesc = smem_desc(base, 128, 256);
+        const uint64_t bdesc = smem_desc(base + 16384, 128, 256);
+        const uint32_t idesc = (1u << 4)               // D: f32
+                               | (0u << 7) | (0u << 10)  // A, B: f16
+                               | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(128 >> 4) << 24);
+        const unsigned long long t0 = clk();
+        for (int i = 0; i < iters; ++i) {
+            asm volatile(
+                "{\n.reg .pred p;\nsetp.ne.b32 p, %4, 0;\n"
+                "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem),
+                "l"(adesc), "l"(bdesc), "r"(idesc), "r"(i)
+                : "memory");
+        }
+        asm volatile(
+            "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+                bar_s)
+            : "memory");
+        uint32_t ok = 0;
+        for (int sp = 0; sp < (1 << 24) && !ok; ++sp)
+            asm volatile("{\n.reg .pred p;\nmbarrier.try_wait.parity.shared::cta.b64 p, [%1], 0;\n"
+                         "selp.u32 %0, 1, 0, p;\n}\n"
+                         : "=r"(ok) : "r"(bar_s) : "memory");
+        const unsigned long long t1 = clk();
+        out[blockIdx.x] = t1 - t0;
+        if (!ok) atomicExch(status, 1);
+    }
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    if (warp == 0)
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, 256;" ::"r"(tmem)
+                     : "memory");
+}
+
+// 3. The W3 record loop from shared memory: each warp walks records laid out as in the stream
+// (768 B of codes per record, lane l's 24 bytes at 16 l and 512 + 8 l), extracts its 32 A
+// registers (the library's mask-and-or scheme) and issues the 8 MMAs against a fixed B.
+template <bool MULHI>
+__device__ __forceinline__ void extract3(const uint32_t (&wd)[6], uint32_t (&a)[8][4]) {
+    const uint32_t e1 = 0x60006000u, e4 = 0x54005400u, e7 = 0x48004800u;
+    uint32_t rp[16][2];
+#pragma unroll
+    for (int w = 0; w < 6; ++w) {
+        const uint32_t u = MULHI ? __umulhi(wd[w], 1u << 23) : wd[w] >> 9;
+        rp[w][0] = (wd[w] & 0x000e000eu) | e1;
+        rp[6 + w][0] = (wd[w] & 0x00700070u) | e4;
+        rp[w][1] = (u & 0x000e000eu) | e1;
+        rp[6 + w][1] = (u & 0x00700070u) | e4;
+    }
+#pragma unroll
+    for (int q = 0; q < 3; ++q) {
+        rp[12 + q][0] = (wd[2 * q] & 0x03800380u) | e7;
+        rp[12 + q][1] = (wd[2 * q + 1] & 0x03800380u) | e7;
+    }
+    rp[15][0] = ((wd[0] << 4) & 0x00100010u) | ((wd[1] << 5) & 0x00200020u) |
+                ((wd[2] << 6) & 0x00400040u) | e4;
+    rp[15][1] = ((wd[3] << 4) & 0x00100010u) | ((wd[4] << 5) & 0x00200020u) |
+                ((wd[5] << 6) & 0x00400040u) | e4;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+        a[j][0] = rp[2 * j][0];
+        a[j][1] = rp[2 * j][1];
+        a[j][2] = rp[2 * j + 1][0];
+        a[j][3] = rp[2 * j + 1][1];
+    }
+}
+
+template <bool MULHI>
+__global__ void __launch_bounds__(512, 1) record_loop(int records, unsigned long long* out,
+                                                      float* sink) {
+    extern __shared__ __align__(1024) uint8_t sm[];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    constexpr int kRec = 768, kRing = 16;  // 16 records per warp in shared memory
+    for (int i = threadIdx.x; i < 16 * kRing * kRec / 4; i += blockDim.x)
+        reinterpret_cast<uint32_t*>(sm)[i] = 0x12345678u * (uint32_t)i;
+    __syncthreads();
+    const uint8_t* mine = sm + (size_t)warp * kRing * kRec;
+    float D[4][4] = {};
+    const uint32_t b0 = 0x3c003c00u, b1 = 0x3c003c00u ^ (uint32_t)lane;
+    const unsigned long long t0 = clk();
+    for (int r = 0; r < records; r += 8) {
+#pragma unroll
+        for (int g = 0; g < 8; ++g) {
+            const uint8_t* rec = mine + ((r + g) % kRing) * kRec;
+            const uint4 c0 = *reinterpret_cast<const uint4*>(rec + lane * 16);
+            const uint2 c1 = *reinterpret_cast<const uint2*>(rec + 512 + lane * 8);
+            const uint32_t wd[6] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y};
+            uint32_t a[8][4];
+            extract3<MULHI>(wd, a);
+#pragma unroll
+            for (int j = 0; j < 8; ++j) mma16816(D[j & 3], a[j][0], a[j][1], a[j][2], a[j][3], b0, b1);
+        }
+    }
+    __syncthreads();
+    const unsigned long long t1 = clk();
+    float s = 0.f;
+#pragma unroll
+    for (int c = 0; c < 4; ++c) s += D[c][0] + D[c][1] + D[c][2] + D[c][3];
+    if (s == 12345.f) sink[0] = s;
+    if (threadIdx.x == 0) out[blockIdx.x] = t1 - t0;
+}
+
+// 4. Issue rates: per warp-iteration, NL integer instructions of one kind (0: and-or LOP3,
+// 1: shift, 2: multiply-high, 3: add) and NM independent mma.sync, 32 warps per SM.
+template <int KIND, int NL, int NM>
+__global__ void __launch_bounds__(1024, 1) issue_mix(int iters, unsigned long long* out,
+                                                     uint32_t* sink) {
+    uint32_t v[8];
+    for (int i = 0; i < 8; ++i) v[i] = threadIdx.x * 2654435761u + i;
+    float d[4][4] = {};
+    const uint32_t m = 0x0e0e0e0eu ^ threadIdx.x, e = 0x60006000u, a = 0x3c003c00u ^ threadIdx.x;
+    __syncthreads();
+    const unsigned long long t0 = clk();
+    for (int it = 0; it < iters; ++it) {
+#pragma unroll
+        for (int i = 0; i < NL; ++i) {
+            if (KIND == 0)
+                asm volatile("lop3.b32 %0, %0, %1, %2, 0xEA;" : "+r"(v[i & 7]) : "r"(m), "r"(e));
+            if (KIND == 1)
+                asm volatile("shf.r.clamp.b32 %0, %0, %1, %2;" : "+r"(v[i & 7]) : "r"(m), "r"(e >> 28));
+            if (KIND == 2) asm volatile("mul.hi.u32 %0, %0, %1;" : "+r"(v[i & 7]) : "r"(m | 1u));
+            if (KIND == 3) asm volatile("add.u32 %0, %0, %1;" : "+r"(v[i & 7]) : "r"(m));
+        }
+#pragma unroll
+        for (int j = 0; j < NM; ++j) mma16816(d[j & 3], a, a + j, a ^ j, a, a, (uint32_t)it);
+    }
+    __syncthreads();
+    const unsigned long long t1 = clk();
+    uint32_t s = 0;
+    float f = 0.f;
+    for (int i = 0; i < 8; ++i) s ^= v[i];
+    for (int j = 0; j < 4; ++j) f += d[j][0] + d[j][1] + d[j][2] + d[j][3];
+    if (s == 0x12345u || f == 1234.5f) sink[0] = s;
+    if (threadIdx.x == 0) out[blockIdx.x] = t1 - t0;
+}
+
+unsigned long long median(std::vector<unsigned long long> v) {
+    std::sort(v.begin(), v.end());
+    return v[v.size() / 2];
+}
+
+}  // namespace
+
+int main() {
+    int dev = 0, P = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&P, cudaDevAttrMultiProcessorCount, dev);
+    unsigned long long* out = nullptr;
+    float* sink = nullptr;
+    int* status = nullptr;
+    if (cudaMalloc(&out, 8 * 1024) || cudaMalloc(&sink, 64) || cudaMalloc(&status, 4)) {
+        printf("allocation failed\n");
+        return 1;
+    }
+    cudaMemset(status, 0, 4);
+    std::vector<unsigned long long> h(P);
+    auto fetch = [&]() {
+        cudaMemcpy(h.data(), out, P * 8, cudaMemcpyDeviceToHost);
+        return median(h);
+    };
+
+    const int iters = 4096;
+    mma_sync_rate<8><<<P, 512>>>(iters, out, sink);
+    if (cudaDeviceSynchronize() != cudaSuccess) { printf("error 1\n"); return 1; }
+    printf("1. mma.sync.m16n8k16 f32.f16: %.2f cycles per MMA per SM (16 warps x 8 chains)\n",
+           (double)fetch() / (16.0 * 8 * iters));
+    mma_sync_rate<1><<<P, 32>>>(iters, out, sink);
+    if (cudaDeviceSynchronize() != cudaSuccess) { printf("error 2\n"); return 1; }
+    printf("   dependent latency of one chain: %.1f cycles\n", (double)fetch() / iters);
+
+    cudaFuncSetAttribute(tc_rate, cudaFuncAttributeMaxDynamicSharedMemorySize, 65536);
+    printf("2. tcgen05.mma.cta_group::1.kind::f16, M = 128, K = 16, A and B in shared memory:\n");
+    for (int n : {16, 32, 64, 128, 256}) {
+        tc_rate<<<P, 128, 65536>>>(n, 512, out, status);
+        if (cudaDeviceSynchronize() != cudaSuccess) { printf("error 3\n"); return 1; }
+        int st = 0;
+        cudaMemcpy(&st, status, 4, cudaMemcpyDeviceToHost);
+        const double cyc = (double)fetch() / 512;
+        printf("   N = %3d: %6.1f cycles per MMA (%5.0f MAC per cycle per SM)%s\n", n, cyc,
+               128.0 * n * 16 / cyc, st ? "  [a wait gave up]" : "");
+    }
+
+    const int smem = 16 * 16 * 768;
+    const int records = 2048;
+    for (int mulhi = 0; mulhi < 2; ++mulhi) {
+        if (mulhi) {
+            cudaFuncSetAttribute(record_loop<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+            record_loop<true><<<P, 512, smem>>>(records, out, sink);
+        } else {
+            cudaFuncSetAttribute(record_loop<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+            record_loop<false><<<P, 512, smem>>>(records, out, sink);
+        }
+        if (cudaDeviceSynchronize() != cudaSuccess) { printf("error 4\n"); return 1; }
+        printf("3. W3 record loop from shared memory, 16 warps, %s: %.1f cycles per record per SM\n",
+               mulhi ? "multiply-high shifts" : "plain shifts", (double)fetch() / (16.0 * records));
+    }
+
+    printf("4. cycles per warp-iteration per SM, 32 warps:\n");
+    struct Case { const char* name; void (*k)(int, unsigned long long*, uint32_t*); int n; };
+    const Case cases[] = {
+        {"8 and-or (lop3)", issue_mix<0, 8, 0>, 8}, {"8 shifts", issue_mix<1, 8, 0>, 8},
+        {"8 multiply-high", issue_mix<2, 8, 0>, 8}, {"8 adds", issue_mix<3, 8, 0>, 8},
+        {"4 mma.sync", issue_mix<0, 0, 4>, 4}, {"8 and-or + 4 mma.sync", issue_mix<0, 8, 4>, 4},
+        {"16 and-or + 4 mma.sync", issue_mix<0, 16, 4>, 4},
+        {"8 multiply-high + 4 mma.sync", issue_mix<2, 8, 4>, 4}};
+    for (const Case& c : cases) {
+        c.k<<<P, 1024>>>(2048, out, reinterpret_cast<uint32_t*>(sink));
+        if (cudaDeviceSynchronize() != cudaSuccess) { printf("error 5\n"); return 1; }
+        printf("   %-30s %6.2f\n", c.name, (double)fetch() / (32.0 * 2048));
+    }
+    return 0;
+}
