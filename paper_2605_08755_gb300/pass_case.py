@@ -1,16 +1,17 @@
 """One form of the decode-step weight pass, replayed a few times: the case for profiling a pass.
 
-    python -m paper_2605_08755_gb300.pass_case --variant graph_fused --bits 3 --M 1 --replays 3
+    python -m paper_2605_08755_gb300.pass_case --variant graph_fused --layers 2 --replays 1
 
-Builds the Qwen3-4B-shaped pass (36 layers, synthetic weights) in one of its forms
-(``graph_252``, ``graph_fused``, ``chain_252``, ``chain_fused``, and the planned pass over
-per-SM weight streams, ``planned_252`` and ``planned_fused``, M <= 4), captures it into a CUDA
-graph (the capture is preceded by one eager run of the pass), replays the graph ``replays``
-times and prints the mean device time per replay.  Under a profiler, the first replay's kernels
-follow the eager run's: for a graph form, ``-k regex:gemm_kernel -s L -c L`` with L = the
-printed ``launches`` selects exactly the first replay; for a chain form, ``-k
-regex:chain_kernel -s 1 -c 1`` does, and ``-k regex:pass_kernel -s 1 -c 1`` for a planned form.
-"""
+Builds the Qwen3-4B-shaped pass (synthetic weights; use a 1- or 2-layer pass under a profiler)
+in one of its forms (``graph_252``, ``graph_fused``, ``chain_252``, ``chain_fused``, and the
+planned pass over per-SM weight streams, ``planned_252`` and ``planned_fused``, M <= 4),
+captures it into a CUDA graph (the capture is preceded by one eager run of the pass), replays
+the graph ``replays`` times and prints the mean device time per replay.  Under a profiler, the
+first replay's kernels follow the eager run's: for a graph form with L launches per pass,
+``-k regex:gemm_kernel -s L -c 4`` selects one launch of each projection of the replay's first
+layer; for a chain form ``-k regex:chain_kernel -s 1 -c 1`` and for a planned form
+``-k regex:pass_kernel -s 1 -c 1`` select the replay's single launch.
+""""""
 import argparse
 import json
 
