@@ -22,6 +22,7 @@ def _lib():
     I = ctypes.c_int
     sigs = {
         "laqo_quantize_rtn": [P, I64, I64, I, I, P, P, P],
+        "laqo_quantize_rtn_threads": [P, I64, I64, I, I, P, P, P],
         "laqo_dequant": [P, P, P, I64, I64, P],
         "laqo_gemm": [P, I64, I64, I64, P, P, P, P],
         "laqo_gemm_columns": [P, I64, I64, I64, P, P, P, P, I64, P],
@@ -77,6 +78,19 @@ def quantize_rtn(W, bits, group=GROUP):
     z = np.zeros((G, N), np.uint8)
     _check(_lib().laqo_quantize_rtn(_ptr(Wb), K, N, bits, group, _ptr(codes), _ptr(s), _ptr(z)),
            "laqo_quantize_rtn")
+    return codes, s.view(np.float16), z
+
+
+def quantize_rtn_threads(W, bits, group=GROUP):
+    """``quantize_rtn`` with the columns split over the host's threads (bit-identical)."""
+    Wb = _bits16(W)
+    K, N = Wb.shape
+    G = K // GROUP if K % GROUP == 0 else 0
+    codes = np.zeros((K, N), np.uint8)
+    s = np.zeros((G, N), np.uint16)
+    z = np.zeros((G, N), np.uint8)
+    _check(_lib().laqo_quantize_rtn_threads(_ptr(Wb), K, N, bits, group, _ptr(codes), _ptr(s),
+                                            _ptr(z)), "laqo_quantize_rtn_threads")
     return codes, s.view(np.float16), z
 
 

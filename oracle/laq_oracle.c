@@ -73,6 +73,46 @@ static uint16_t half_round_up_positive(double v)
 
 /* ---------- Eq. (1): RTN group quantizer ---------- */
 
+/* Group g of column n (rows 128g .. 128g + 127): its scale, zero and codes. */
+static void quantize_group(const uint16_t *W, int64_t N, int64_t g, int64_t n, int qmax,
+                           uint8_t *codes, uint16_t *s, uint8_t *z)
+{
+    double lo = INFINITY, hi = -INFINITY;
+    for (int64_t k = g * LAQO_GROUP; k < (g + 1) * LAQO_GROUP; ++k) {
+        double w = laqo_half_to_double(W[k * N + n]);
+        if (w < lo) lo = w;
+        if (w > hi) hi = w;
+    }
+    uint16_t sh;
+    int zz;
+    if (lo == hi) {                       /* constant group: exact by construction */
+        if (lo != 0.0) {
+            sh = (uint16_t)(W[g * LAQO_GROUP * N + n] & 0x7fff);   /* |c| */
+            zz = lo < 0.0 ? 1 : 0;
+        } else {
+            sh = 0x3c00;                                           /* 1.0 */
+            zz = 0;
+        }
+    } else {
+        double lo0 = lo < 0.0 ? lo : 0.0;  /* zero-inclusive range */
+        double hi0 = hi > 0.0 ? hi : 0.0;
+        double sd = (hi0 - lo0) / (double)qmax;
+        sh = half_round_up_positive(sd);
+        if (sh < 0x0400) sh = 0x0400;       /* floor: smallest normal fp16 */
+        zz = (int)rint(-lo0 / laqo_half_to_double(sh));
+    }
+    double sv = laqo_half_to_double(sh);
+    s[g * N + n] = sh;
+    z[g * N + n] = (uint8_t)zz;
+    for (int64_t k = g * LAQO_GROUP; k < (g + 1) * LAQO_GROUP; ++k) {
+        double w = laqo_half_to_double(W[k * N + n]);
+        int q = (int)rint(w / sv) + zz;    /* round first, then add z (Eq. 1) */
+        if (q < 0) q = 0;
+        if (q > qmax) q = qmax;
+        codes[k * N + n] = (uint8_t)q;
+    }
+}
+
 int laqo_quantize_rtn(const uint16_t *W, int64_t K, int64_t N, int bits, int group,
                       uint8_t *codes, uint16_t *s, uint8_t *z)
 {
@@ -81,43 +121,29 @@ int laqo_quantize_rtn(const uint16_t *W, int64_t K, int64_t N, int bits, int gro
     if (K < 0 || N < 0 || K % LAQO_GROUP) return 4;
     const int qmax = (1 << bits) - 1;
     const int64_t G = K / LAQO_GROUP;
-    for (int64_t g = 0; g < G; ++g) {
-        for (int64_t n = 0; n < N; ++n) {
-            double lo = INFINITY, hi = -INFINITY;
-            for (int64_t k = g * LAQO_GROUP; k < (g + 1) * LAQO_GROUP; ++k) {
-                double w = laqo_half_to_double(W[k * N + n]);
-                if (w < lo) lo = w;
-                if (w > hi) hi = w;
-            }
-            uint16_t sh;
-            int zz;
-            if (lo == hi) {                       /* constant group: exact by construction */
-                if (lo != 0.0) {
-                    sh = (uint16_t)(W[g * LAQO_GROUP * N + n] & 0x7fff);   /* |c| */
-                    zz = lo < 0.0 ? 1 : 0;
-                } else {
-                    sh = 0x3c00;                                           /* 1.0 */
-                    zz = 0;
-                }
-            } else {
-                double lo0 = lo < 0.0 ? lo : 0.0;  /* zero-inclusive range */
-                double hi0 = hi > 0.0 ? hi : 0.0;
-                double sd = (hi0 - lo0) / (double)qmax;
-                sh = half_round_up_positive(sd);
-                if (sh < 0x0400) sh = 0x0400;       /* floor: smallest normal fp16 */
-                zz = (int)rint(-lo0 / laqo_half_to_double(sh));
-            }
-            double sv = laqo_half_to_double(sh);
-            s[g * N + n] = sh;
-            z[g * N + n] = (uint8_t)zz;
-            for (int64_t k = g * LAQO_GROUP; k < (g + 1) * LAQO_GROUP; ++k) {
-                double w = laqo_half_to_double(W[k * N + n]);
-                int q = (int)rint(w / sv) + zz;    /* round first, then add z (Eq. 1) */
-                if (q < 0) q = 0;
-                if (q > qmax) q = qmax;
-                codes[k * N + n] = (uint8_t)q;
-            }
-        }
+    for (int64_t g = 0; g < G; ++g)
+        for (int64_t n = 0; n < N; ++n) quantize_group(W, N, g, n, qmax, codes, s, z);
+    return 0;
+}
+
+/* laqo_quantize_rtn with the columns split over the host's threads (OpenMP, when the oracle is
+ * built with it): every (group, column) is quantized by the same quantize_group, so the codes,
+ * scales and zeros are laqo_quantize_rtn's bit for bit.  Used to check whole passes. */
+int laqo_quantize_rtn_threads(const uint16_t *W, int64_t K, int64_t N, int bits, int group,
+                              uint8_t *codes, uint16_t *s, uint8_t *z)
+{
+    if (bits != 3 && bits != 4) return 2;
+    if (group != LAQO_GROUP) return 3;
+    if (K < 0 || N < 0 || K % LAQO_GROUP) return 4;
+    const int qmax = (1 << bits) - 1;
+    const int64_t G = K / LAQO_GROUP;
+    const int64_t cb = 64; /* columns per task */
+    const int64_t ntask = (N + cb - 1) / cb;
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int64_t t = 0; t < ntask; ++t) {
+        const int64_t n1 = (t + 1) * cb < N ? (t + 1) * cb : N;
+        for (int64_t g = 0; g < G; ++g)
+            for (int64_t n = t * cb; n < n1; ++n) quantize_group(W, N, g, n, qmax, codes, s, z);
     }
     return 0;
 }

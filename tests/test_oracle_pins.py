@@ -298,3 +298,17 @@ def test_threaded_gemm_is_the_plain_gemm(bits):
     X = inputs.activations(3, 384, seed=bits)
     codes, s, z = co.quantize_rtn(W, bits)
     assert np.array_equal(co.gemm_threads(X, codes, s, z), co.gemm(X, codes, s, z))
+
+
+@pytest.mark.parametrize("bits", [3, 4])
+def test_threaded_quantizer_is_the_plain_quantizer(bits):
+    """The oracle's all-cores quantizer (columns split over threads, each (group, column) by the
+    same routine) gives the single-threaded codes, scales and zeros bit for bit, on a ragged N
+    with constant and one-signed groups planted."""
+    W = inputs.weights(512, 16 * 21 + 8, seed=bits + 10)
+    W[:128, 3] = np.float16(0.25)          # a constant group
+    W[128:256, 7] = np.abs(W[128:256, 7])  # a one-signed group
+    a = co.quantize_rtn(W, bits)
+    b = co.quantize_rtn_threads(W, bits)
+    for x, y in zip(a, b):
+        assert np.array_equal(np.asarray(x).view(np.uint8), np.asarray(y).view(np.uint8))
