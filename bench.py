@@ -239,7 +239,8 @@ class OracleSample:
     """A bounded sample of the same workload for the C oracle: the projections of layer 0 (same
     shapes, distributions and seeds recipe), quantized once by the oracle (untimed).  ``run``
     times the oracle's fp64 dequantize-and-multiply over whole projections (or a leading
-    column slice of one, when a short step is asked for)."""
+    column slice of one, when a short step is asked for); ``run_quantize`` times its quantizer
+    and packer, the offline step, separately."""
 
     def __init__(self, model, bits, M, seed=0):
         from oracle import c_oracle
@@ -248,12 +249,38 @@ class OracleSample:
         self.co = c_oracle
         self.bits, self.M = bits, M
         self.items = []
+        self.weights = []
         for pi, (name, K, N) in enumerate(shapes(model)):
             sd = inputs.proj_seed(seed, 0, pi)
             W = inputs.weights(K, N, sd, outliers=(model == "qwen3-8b"))
-            codes, s, z = c_oracle.quantize_rtn(W, bits)
+            codes, s, z = c_oracle.quantize_rtn_threads(W, bits)
             self.items.append((f"L0.{name}", codes, s, z, inputs.activations(M, K, sd)))
+            self.weights.append((f"L0.{name}", W))
         self.next = 0
+
+    def run_quantize(self, seconds, threaded=True):
+        """The oracle's RTN quantizer (``threaded``: over the host's threads) and its packer on
+        whole layer-0 projections, round-robin, for about ``seconds``; returns (weights,
+        quantize seconds, pack seconds, projections)."""
+        n = qs = ps = 0.0
+        names = []
+        i = 0
+        while True:
+            name, W = self.weights[i % len(self.weights)]
+            i += 1
+            t0 = time.perf_counter()
+            codes, _, _ = (self.co.quantize_rtn_threads if threaded else self.co.quantize_rtn)(
+                W, self.bits)
+            t1 = time.perf_counter()
+            self.co.pack(codes, self.bits)
+            t2 = time.perf_counter()
+            qs += t1 - t0
+            ps += t2 - t1
+            n += W.size
+            names.append(name)
+            if qs + ps >= seconds:
+                break
+        return n, qs, ps, names
 
     def nbytes(self, K, N):
         return K * N * self.bits // 8 + (K // 128) * N * 3 + 2 * self.M * K + 2 * self.M * N
@@ -753,8 +780,14 @@ def run_laq(a, world, rank, local):
                "sample": f"C oracle (fp64) dequantize-and-multiply, output columns split over "
                          f"{threads} threads, of {len(names)} whole projections of layer 0, "
                          f"round-robin over q,k,v,o,gate,up,down, {spent:.1f} s of wall time "
-                         f"(single-threaded: {len(n1)} projections in {s1:.1f} s); "
-                         f"quantization not timed"}
+                         f"(single-threaded: {len(n1)} projections in {s1:.1f} s); the "
+                         f"quantizer and packer timed separately (quantize_pack)"}
+        nw, qs, ps, qn = smp.run_quantize(min(4.0, a.cpu_seconds / 3))
+        cpu["quantize_pack"] = {
+            "quantize_weights_per_s": nw / qs, "pack_weights_per_s": nw / ps,
+            "sample": f"oracle RTN quantizer (fp64, columns split over {threads} threads) and "
+                      f"packer (one thread) on {len(qn)} whole layer-0 projections "
+                      f"({nw / 1e6:.0f} M weights): {qs:.2f} s quantizing, {ps:.2f} s packing"}
 
     if rank != 0:
         return
