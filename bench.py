@@ -310,6 +310,25 @@ class OracleSample:
         return done, spent, names
 
 
+def oracle_single_linear(bits, reps=20):
+    """The oracle, one thread, on a single 1024 x 1024 W{bits}G128 linear at M = 1 (the shapes
+    and distributions of the GPU's gemv_1024 sweep entry): median time of its
+    dequantize-and-multiply over ``reps`` calls."""
+    from oracle import c_oracle
+    from paper_2605_08755_gb300 import inputs
+    W = inputs.weights(1024, 1024, 0)
+    codes, s, z = c_oracle.quantize_rtn(W, bits)
+    X = inputs.activations(1, 1024, 0)
+    ts = []
+    for _ in range(reps):
+        t0 = time.perf_counter()
+        c_oracle.gemm(X, codes, s, z)
+        ts.append(time.perf_counter() - t0)
+    us = 1e6 * statistics.median(ts)
+    nbytes = 1024 * 1024 * bits // 8 + 8 * 1024 * 3 + 2 * 1024 + 2 * 1024
+    return {"us_per_gemv": us, "gbs": nbytes / us / 1e3, "threads": 1}
+
+
 # ------------------------------------------------------------------ reference arm
 
 
@@ -782,6 +801,7 @@ def run_laq(a, world, rank, local):
                          f"round-robin over q,k,v,o,gate,up,down, {spent:.1f} s of wall time "
                          f"(single-threaded: {len(n1)} projections in {s1:.1f} s); the "
                          f"quantizer and packer timed separately (quantize_pack)"}
+        cpu["single_linear_1024"] = oracle_single_linear(a.bits)
         nw, qs, ps, qn = smp.run_quantize(min(4.0, a.cpu_seconds / 3))
         cpu["quantize_pack"] = {
             "quantize_weights_per_s": nw / qs, "pack_weights_per_s": nw / ps,
