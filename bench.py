@@ -361,7 +361,7 @@ def run_reference(a, world, rank):
     threads = smp.co.threads()
     sample = (f"C oracle (fp64) dequantize-and-multiply, output columns split over {threads} "
               f"threads; each step = the first {cols} columns of one layer-0 projection, "
-              f"round-robin over q,k,v,o,gate,up,down; {tot_s:.1f} s of CPU work over "
+              f"round-robin over q,k,v,o,gate,up,down; {tot_s:.3g} s of CPU work over "
               f"{a.steps} steps; quantization not timed; host CPU {cpu_name}, {avail} cores "
               f"available")
     line = {"metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": a.gpus,
