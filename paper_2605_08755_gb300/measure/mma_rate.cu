@@ -16,7 +16,15 @@
 //      record per 38 SM cycles), with the field shifts as plain shifts (the library's form) and
 //      as multiply-high instructions;
 //   4. the issue rates behind it: mask-and-or (LOP3), shift, multiply-high, add, and how much
-//      integer work hides behind mma.sync.
+//      integer work hides behind mma.sync;
+//   5. mma.sync.m16n8k32 with e4m3 operands (f32 accumulate): the same 2048 weights per record
+//      in 4 instructions of K = 32 (a code q in the 3 mantissa bits of an e4m3 byte is the exact
+//      value 8 + q, four codes per 32-bit register), its rate and latency, and how integer work
+//      hides behind it;
+//   6. how precisely each form accumulates: every A and B element equal (so the fragment layout
+//      does not matter), the accumulator started at 2^20, and the 32 (e4m3) or 16 (f16)
+//      products 2^-e each; D - 2^20 is exact in fp32 for every e here, so any shortfall is the
+//      tensor core's own alignment of small addends.
 // Every wait is bounded.
 //
 //   nvcc -gencode arch=compute_103a,code=sm_103a -O3 -Xptxas -v -o /tmp/mma_rate \
@@ -56,6 +64,51 @@ __global__ void __launch_bounds__(512, 1) mma_sync_rate(int iters, unsigned long
     for (int i = 0; i < iters; ++i) {
 #pragma unroll
         for (int c = 0; c < CHAINS; ++c) mma16816(d[c], a, a + c, a ^ c, a, b, b + i);
+    }
+    __syncthreads();
+    const unsigned long long t1 = clk();
+    float s = 0.f;
+#pragma unroll
+    for (int c = 0; c < CHAINS; ++c) s += d[c][0] + d[c][1] + d[c][2] + d[c][3];
+    if (s == 12345.f) sink[0] = s;
+    if (threadIdx.x == 0) out[blockIdx.x] = t1 - t0;
+}
+
+// 5. mma.sync.m16n8k32 e4m3 x e4m3 -> f32, `chains` independent accumulators per warp.
+__device__ __forceinline__ void mma16832_e4m3(float (&d)[4], uint32_t a0, uint32_t a1,
+                                              uint32_t a2, uint32_t a3, uint32_t b0,
+                                              uint32_t b1) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k32.row.col.f32.e4m3.e4m3.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
+        "{%8,%9}, {%0,%1,%2,%3};\n"
+        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+        : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+// 6. One MMA with every A element a, every B element b and C = c; D[0] of lane 0 to out.
+__global__ void accum_probe(uint32_t a8, uint32_t b8, uint32_t a16, uint32_t b16, float c,
+                            float* out) {
+    float d[4] = {c, c, c, c};
+    mma16832_e4m3(d, a8, a8, a8, a8, b8, b8);
+    float h[4] = {c, c, c, c};
+    mma16816(h, a16, a16, a16, a16, b16, b16);
+    if (threadIdx.x == 0) {
+        out[0] = d[0];
+        out[1] = h[0];
+    }
+}
+
+template <int CHAINS>
+__global__ void __launch_bounds__(512, 1) mma_e4m3_rate(int iters, unsigned long long* out,
+                                                        float* sink) {
+    float d[CHAINS][4] = {};
+    // e4m3 bytes 0x38 = 1.0 and 0x50 | q = 8 + q: finite values whatever the lane
+    const uint32_t a = 0x50505050u | (threadIdx.x & 0x07070707u), b = 0x38383838u;
+    __syncthreads();
+    const unsigned long long t0 = clk();
+    for (int i = 0; i < iters; ++i) {
+#pragma unroll
+        for (int c = 0; c < CHAINS; ++c)
+            mma16832_e4m3(d[c], a, a, a, a, b, b);
     }
     __syncthreads();
     const unsigned long long t1 = clk();
@@ -202,14 +255,16 @@ __global__ void __launch_bounds__(512, 1) record_loop(int records, unsigned long
 }
 
 // 4. Issue rates: per warp-iteration, NL integer instructions of one kind (0: and-or LOP3,
-// 1: shift, 2: multiply-high, 3: add) and NM independent mma.sync, 32 warps per SM.
-template <int KIND, int NL, int NM>
+// 1: shift, 2: multiply-high, 3: add) and NM independent mma.sync (FP8: the e4m3 m16n8k32 form
+// of part 5 instead of f16 m16n8k16), 32 warps per SM.
+template <int KIND, int NL, int NM, bool FP8 = false>
 __global__ void __launch_bounds__(1024, 1) issue_mix(int iters, unsigned long long* out,
                                                      uint32_t* sink) {
     uint32_t v[8];
     for (int i = 0; i < 8; ++i) v[i] = threadIdx.x * 2654435761u + i;
     float d[4][4] = {};
     const uint32_t m = 0x0e0e0e0eu ^ threadIdx.x, e = 0x60006000u, a = 0x3c003c00u ^ threadIdx.x;
+    const uint32_t a8 = 0x50505050u | (a & 0x07070707u), b8 = 0x38383838u;  // e4m3 8 + q, 1.0
     __syncthreads();
     const unsigned long long t0 = clk();
     for (int it = 0; it < iters; ++it) {
@@ -223,7 +278,12 @@ __global__ void __launch_bounds__(1024, 1) issue_mix(int iters, unsigned long lo
             if (KIND == 3) asm volatile("add.u32 %0, %0, %1;" : "+r"(v[i & 7]) : "r"(m));
         }
 #pragma unroll
-        for (int j = 0; j < NM; ++j) mma16816(d[j & 3], a, a + j, a ^ j, a, a, (uint32_t)it);
+        for (int j = 0; j < NM; ++j) {
+            if (FP8)
+                mma16832_e4m3(d[j & 3], a8, a8, a8, a8, b8, b8);
+            else
+                mma16816(d[j & 3], a, a + j, a ^ j, a, a, (uint32_t)it);
+        }
     }
     __syncthreads();
     const unsigned long long t1 = clk();
@@ -303,11 +363,39 @@ int main() {
         {"8 multiply-high", issue_mix<2, 8, 0>, 8}, {"8 adds", issue_mix<3, 8, 0>, 8},
         {"4 mma.sync", issue_mix<0, 0, 4>, 4}, {"8 and-or + 4 mma.sync", issue_mix<0, 8, 4>, 4},
         {"16 and-or + 4 mma.sync", issue_mix<0, 16, 4>, 4},
-        {"8 multiply-high + 4 mma.sync", issue_mix<2, 8, 4>, 4}};
+        {"8 multiply-high + 4 mma.sync", issue_mix<2, 8, 4>, 4},
+        {"4 mma.sync e4m3", issue_mix<0, 0, 4, true>, 4},
+        {"8 and-or + 4 mma.sync e4m3", issue_mix<0, 8, 4, true>, 4},
+        {"16 and-or + 4 mma.sync e4m3", issue_mix<0, 16, 4, true>, 4}};
     for (const Case& c : cases) {
         c.k<<<P, 1024>>>(2048, out, reinterpret_cast<uint32_t*>(sink));
         if (cudaDeviceSynchronize() != cudaSuccess) { printf("error 5\n"); return 1; }
         printf("   %-30s %6.2f\n", c.name, (double)fetch() / (32.0 * 2048));
+    }
+
+    mma_e4m3_rate<8><<<P, 512>>>(iters, out, sink);
+    if (cudaDeviceSynchronize() != cudaSuccess) { printf("error 6\n"); return 1; }
+    printf("5. mma.sync.m16n8k32 f32.e4m3: %.2f cycles per MMA per SM (16 warps x 8 chains)\n",
+           (double)fetch() / (16.0 * 8 * iters));
+    mma_e4m3_rate<1><<<P, 32>>>(iters, out, sink);
+    if (cudaDeviceSynchronize() != cudaSuccess) { printf("error 7\n"); return 1; }
+    printf("   dependent latency of one chain: %.1f cycles\n", (double)fetch() / iters);
+
+    // e4m3 2^k (k = -6..8): exponent field k + 7, mantissa 0; f16 2^k: exponent field k + 15
+    printf("6. accumulation: C = 2^20, A = 1, B = 2^-e; D - 2^20 against the exact 32 (e4m3) or "
+           "16 (f16) x 2^-e:\n");
+    float* dv = reinterpret_cast<float*>(sink);
+    for (int e = 0; e <= 6; ++e) {
+        const uint32_t one8 = 0x38u, b8 = (uint32_t)(7 - e) << 3;
+        const uint32_t one16 = 0x3c00u, b16 = (uint32_t)(15 - e) << 10;
+        accum_probe<<<1, 32>>>(one8 * 0x01010101u, b8 * 0x01010101u, one16 * 0x00010001u,
+                               b16 * 0x00010001u, 1048576.f, dv);
+        if (cudaDeviceSynchronize() != cudaSuccess) { printf("error 8\n"); return 1; }
+        float hv[2];
+        cudaMemcpy(hv, dv, 8, cudaMemcpyDeviceToHost);
+        printf("   e = %d: e4m3 %.6f (exact %.6f), f16 %.6f (exact %.6f)\n", e,
+               (double)hv[0] - 1048576.0, 32.0 / (1 << e), (double)hv[1] - 1048576.0,
+               16.0 / (1 << e));
     }
     return 0;
 }
