@@ -101,14 +101,17 @@ laq_status check_config(const laq_gemm_config* c) {
 int ceil_div(int64_t a, int64_t b) { return (int)((a + b - 1) / b); }
 
 // Launch-shape plan: tiles per CTA (NT), K split over a cluster (C), warps and ring depth.
-//  * M = 1: the cheapest split by estimated SM time -- records per warp, x 1.3 when two CTAs
+//  * M = 1..4: the cheapest split by estimated SM time -- records per warp, x 1.3 when two CTAs
 //    share an SM (16 warps retire a record in ~0.65x the time of 8; measured on GB300), x 1.02
 //    for a cluster's reduction -- over NT, C in {1, 2, 4, 8} with at most two CTAs per SM.
-//  * M > 1: every CTA reads X for its whole K range, M rows of it -- at M = 16 with one tile
-//    per CTA that is 5x the CTA's weight bytes (b = 3).  So X is shared across 4 (M <= 4) or 8
-//    tiles per CTA and K is split over a cluster (which also splits X) until there is about one
-//    CTA per SM: 40-45% faster than the M = 1 rule on the Qwen3-4B pass at M = 4..16.
-//  * M = 1 with fewer than two tiles per SM (N < 32 x SMs) and a long K, where that plan
+//  * M > 4 (8 batch rows in the MMA's columns): every CTA reads X for its whole K range, M rows
+//    of it -- at M = 16 with one tile per CTA that is 5x the CTA's weight bytes (b = 3).  So X is
+//    shared across 8 tiles per CTA and K is split over a cluster (which also splits X) until
+//    there is about one CTA per SM.  Measured on GB300, fused Qwen3-4B pass, against the rule
+//    above: W3 M = 5 1160 vs 1235 us, M = 8 1183 vs 1586, M = 16 1791 vs 2574; at M = 2..4 the
+//    rule above is the faster one (W3 M = 2 809 vs 868 us, M = 4 915 vs 924; W4 M = 4 1088 vs
+//    1258).
+//  * M <= 4 with fewer than two tiles per SM (N < 32 x SMs) and a long K, where that plan
 //    leaves a warp more than 5 records (the 2560 x 9728 down projection: 160 tiles on 152 SMs,
 //    ~10 records per warp): 4-warp CTAs of 2 tiles instead, K split over a cluster that
 //    doubles until a warp holds at most 5 records and the grid covers every SM (down: 640
@@ -123,8 +126,8 @@ void plan(int64_t M, int64_t K, int64_t N, int bits, int sms, laq_gemm_config* o
     const int64_t rec = bits == 4 ? 1024 : 768;
     int best_nt = 8, best_cl = 1;
     int64_t warps_max = 8;
-    if (M > 1) {
-        int nt = M <= 4 ? 4 : 8;
+    if (M > 4) {
+        int nt = 8;
         while (nt > 1 && ceil_div(T, nt) < sms / 8) nt /= 2;
         int cl = 1;
         while (cl < 8 && cl * 2 <= G && (int64_t)ceil_div(T, nt) * cl < sms) cl *= 2;

@@ -215,12 +215,16 @@ def test_chain_static_argument_validation(L):
     assert L.laq_gemm_chain_static(bad, 1, None) == code["LAQ_ERR_SHAPE"]
 
 
-def test_plan_shares_x_across_tiles_at_m_above_one(L):
-    # M > 1: 4 (M <= 4) or 8 tiles per CTA, and a cluster K split towards one CTA per SM
-    c = laq.laq_gemm_plan(4, 9728, 2560, 3, 152)
-    assert (c.tiles_per_cta, c.cluster) == (4, 4)
-    c = laq.laq_gemm_plan(4, 2560, 19456, 3, 152)
-    assert (c.tiles_per_cta, c.warps, c.cluster) == (4, 8, 1)
+def test_plan_shares_x_across_tiles_above_m_four(L):
+    # M = 2..4: the M = 1 rule (the faster one there on GB300)
+    for M in (2, 3, 4):
+        for K, N in ((9728, 2560), (2560, 19456), (2560, 6144), (4096, 2560)):
+            for bits in (3, 4):
+                assert (laq.laq_gemm_plan(M, K, N, bits, 152).as_dict() ==
+                        laq.laq_gemm_plan(1, K, N, bits, 152).as_dict()), (M, K, N, bits)
+    # M > 4: 8 tiles per CTA, and a cluster K split towards one CTA per SM
+    c = laq.laq_gemm_plan(5, 9728, 2560, 3, 152)
+    assert (c.tiles_per_cta, c.cluster) == (8, 8)
     c = laq.laq_gemm_plan(8, 9728, 2560, 3, 152)
     assert (c.tiles_per_cta, c.warps, c.cluster) == (8, 8, 8)
     # M > 4 where that leaves one 8-warp CTA per SM: 16-warp CTAs (two warps per tile); the
