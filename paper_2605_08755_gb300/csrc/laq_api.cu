@@ -101,17 +101,16 @@ laq_status check_config(const laq_gemm_config* c) {
 int ceil_div(int64_t a, int64_t b) { return (int)((a + b - 1) / b); }
 
 // Launch-shape plan: tiles per CTA (NT), K split over a cluster (C), warps and ring depth.
-//  * M = 1..4: the cheapest split by estimated SM time -- records per warp, x 1.3 when two CTAs
+//  * M = 1, 2: the cheapest split by estimated SM time -- records per warp, x 1.3 when two CTAs
 //    share an SM (16 warps retire a record in ~0.65x the time of 8; measured on GB300), x 1.02
 //    for a cluster's reduction -- over NT, C in {1, 2, 4, 8} with at most two CTAs per SM.
-//  * M > 4 (8 batch rows in the MMA's columns): every CTA reads X for its whole K range, M rows
-//    of it -- at M = 16 with one tile per CTA that is 5x the CTA's weight bytes (b = 3).  So X is
-//    shared across 8 tiles per CTA and K is split over a cluster (which also splits X) until
-//    there is about one CTA per SM.  Measured on GB300, fused Qwen3-4B pass, against the rule
-//    above: W3 M = 5 1160 vs 1235 us, M = 8 1183 vs 1586, M = 16 1791 vs 2574; at M = 2..4 the
-//    rule above is the faster one (W3 M = 2 809 vs 868 us, M = 4 915 vs 924; W4 M = 4 1088 vs
-//    1258).
-//  * M <= 4 with fewer than two tiles per SM (N < 32 x SMs) and a long K, where that plan
+//  * M > 2: every CTA reads X for its whole K range, M rows of it -- at M = 16 with one tile per
+//    CTA that is 5x the CTA's weight bytes (b = 3).  So X is shared across 4 (M <= 4) or 8 tiles
+//    per CTA and K is split over a cluster (which also splits X) until there is about one CTA
+//    per SM.  Measured on GB300, fused Qwen3-4B pass, against the rule above: W3 M = 4 887 vs
+//    915 us, W4 M = 3 856 vs 889, M = 5 1160 vs 1235, M = 8 1183 vs 1586, M = 16 1791 vs 2574;
+//    at M = 2 the rule above is the faster one (W3 810 vs 868 us).
+//  * M <= 4 with fewer than two tiles per SM (N < 32 x SMs) and a long K, where the first plan
 //    leaves a warp more than 5 records (the 2560 x 9728 down projection: 160 tiles on 152 SMs,
 //    ~10 records per warp): 4-warp CTAs of 2 tiles instead, K split over a cluster that
 //    doubles until a warp holds at most 5 records and the grid covers every SM (down: 640
@@ -121,13 +120,51 @@ int ceil_div(int64_t a, int64_t b) { return (int)((a + b - 1) / b); }
 //    the long-K down projection at M > 8, with half the cluster).
 //  * Eight warps otherwise (fewer when a CTA owns fewer groups), and a cp.async ring deep
 //    enough to hold all of a warp's records (at most 16) within 100 KB.
+// Shared memory of one SM of sm_100 / sm_103 and what the hardware reserves per CTA.
+constexpr size_t kSmemPerSm = 228 * 1024, kSmemPerCta = 1024;
+
+void plan(int64_t M, int64_t K, int64_t N, int bits, int sms, laq_gemm_config* out);
+
+// M = 3, 4: X of 3-4 rows beside the ring can leave a CTA just too large for two to share an SM;
+// where the grid needs two per SM, the ring loses stages until two fit (measured on GB300, W4
+// M = 4 fused Qwen3-4B pass: gate|up 11 -> 10 stages, 1032 -> 940 us).
+void fit_two_ctas(int64_t M, int64_t K, int64_t N, int bits, int sms, laq_gemm_config* c) {
+    const int64_t ctas = (int64_t)ceil_div(N / 16, c->tiles_per_cta) * c->cluster;
+    if (ctas <= sms) return;
+    laq::GemmLaunch L;
+    L.M = (int)M;
+    L.K = (int)K;
+    L.N = (int)N;
+    L.bits = bits;
+    L.tiles_per_cta = c->tiles_per_cta;
+    L.warps = c->warps;
+    L.cluster = c->cluster;
+    L.pdl = 0;
+    for (; c->stages > 2; --c->stages) {
+        L.stages = c->stages;
+        if (2 * (laq::gemm_smem_bytes(L, nullptr) + kSmemPerCta) <= kSmemPerSm) break;
+    }
+}
+
 void plan(int64_t M, int64_t K, int64_t N, int bits, int sms, laq_gemm_config* out) {
     const int64_t T = N / 16, G = K / kGroup;
     const int64_t rec = bits == 4 ? 1024 : 768;
     int best_nt = 8, best_cl = 1;
     int64_t warps_max = 8;
-    if (M > 4) {
-        int nt = 8;
+    // M = 3, 4 take the first rule's down shape (below) where it applies, else the batch rule
+    bool batch = M > 4;
+    if (M > 2 && M <= 4) {
+        laq_gemm_config one;
+        plan(1, K, N, bits, sms, &one);
+        batch = !(one.warps == 4 && one.tiles_per_cta == 2 && one.cluster > 1);
+        if (!batch) {
+            *out = one;
+            fit_two_ctas(M, K, N, bits, sms, out);
+            return;
+        }
+    }
+    if (batch) {
+        int nt = M <= 4 ? 4 : 8;
         while (nt > 1 && ceil_div(T, nt) < sms / 8) nt /= 2;
         int cl = 1;
         while (cl < 8 && cl * 2 <= G && (int64_t)ceil_div(T, nt) * cl < sms) cl *= 2;
@@ -189,6 +226,7 @@ void plan(int64_t M, int64_t K, int64_t N, int bits, int sms, laq_gemm_config* o
     out->stages = st;
     out->pdl = 0;
     out->reserved[0] = out->reserved[1] = out->reserved[2] = 0;
+    if (M > 2 && M <= 4) fit_two_ctas(M, K, N, bits, sms, out);
 }
 
 laq_status run_gemm(const void* X, int64_t M, int64_t K, int64_t N, const void* packed,

@@ -215,13 +215,24 @@ def test_chain_static_argument_validation(L):
     assert L.laq_gemm_chain_static(bad, 1, None) == code["LAQ_ERR_SHAPE"]
 
 
-def test_plan_shares_x_across_tiles_above_m_four(L):
-    # M = 2..4: the M = 1 rule (the faster one there on GB300)
-    for M in (2, 3, 4):
+def test_plan_shares_x_across_tiles_above_m_two(L):
+    one = lambda K, N, bits: laq.laq_gemm_plan(1, K, N, bits, 152).as_dict()
+    shape = lambda c: (c.tiles_per_cta, c.warps, c.cluster, c.stages)
+    for bits in (3, 4):
         for K, N in ((9728, 2560), (2560, 19456), (2560, 6144), (4096, 2560)):
-            for bits in (3, 4):
-                assert (laq.laq_gemm_plan(M, K, N, bits, 152).as_dict() ==
-                        laq.laq_gemm_plan(1, K, N, bits, 152).as_dict()), (M, K, N, bits)
+            # M = 2: the M = 1 rule (the faster one there on GB300)
+            assert laq.laq_gemm_plan(2, K, N, bits, 152).as_dict() == one(K, N, bits)
+        for M in (3, 4):
+            # the long-K down projection keeps the M = 1 shape (4-warp CTAs of 2 tiles, cluster 8)
+            assert laq.laq_gemm_plan(M, 9728, 2560, bits, 152).as_dict() == one(9728, 2560, bits)
+            # otherwise X shared by 4 tiles per CTA, K split until about one CTA per SM
+            assert shape(laq.laq_gemm_plan(M, 2560, 6144, bits, 152))[:3] == (4, 8, 2)
+            assert shape(laq.laq_gemm_plan(M, 4096, 2560, bits, 152))[:3] == (4, 8, 4)
+            assert shape(laq.laq_gemm_plan(M, 2560, 19456, bits, 152))[:3] == (4, 8, 1)
+    # gate|up at W4 M = 4: one ring stage less, so that two CTAs share an SM's 228 KB
+    assert laq.laq_gemm_plan(4, 2560, 19456, 4, 152).stages == 10
+    assert laq.laq_gemm_plan(3, 2560, 19456, 4, 152).stages == 11
+    assert laq.laq_gemm_plan(4, 2560, 19456, 3, 152).stages == 11
     # M > 4: 8 tiles per CTA, and a cluster K split towards one CTA per SM
     c = laq.laq_gemm_plan(5, 9728, 2560, 3, 152)
     assert (c.tiles_per_cta, c.cluster) == (8, 8)
