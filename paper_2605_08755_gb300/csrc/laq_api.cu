@@ -101,16 +101,20 @@ laq_status check_config(const laq_gemm_config* c) {
 int ceil_div(int64_t a, int64_t b) { return (int)((a + b - 1) / b); }
 
 // Launch-shape plan: tiles per CTA (NT), K split over a cluster (C), warps and ring depth.
-//  * M = 1, 2: the cheapest split by estimated SM time -- records per warp, x 1.3 when two CTAs
-//    share an SM (16 warps retire a record in ~0.65x the time of 8; measured on GB300), x 1.02
-//    for a cluster's reduction -- over NT, C in {1, 2, 4, 8} with at most two CTAs per SM.
+//  * M = 1, 2: the cheapest split by estimated SM time -- records per warp plus a start cost of
+//    two records' time per wave of CTAs, x the waves (two 8-warp CTAs per SM at a time), x 1.3
+//    when two CTAs share an SM (16 warps retire a record in ~0.65x the time of 8; measured on
+//    GB300), x 1.02 for a cluster's reduction -- over NT, C in {1, 2, 4, 8}.  Several waves win
+//    for wide outputs: a single wave of 8-tile CTAs leaves the Qwen3-8B gate|up (1536 tiles)
+//    with 1.26 CTAs per SM, the SMs holding two doing twice the work (measured on GB300, fused
+//    Qwen3-8B pass: 1624 -> 1262 us with 2-tile CTAs in three waves).
 //  * M > 2: every CTA reads X for its whole K range, M rows of it -- at M = 16 with one tile per
 //    CTA that is 5x the CTA's weight bytes (b = 3).  So X is shared across 4 (M <= 4) or 8 tiles
 //    per CTA and K is split over a cluster (which also splits X) until there is about one CTA
 //    per SM.  Measured on GB300, fused Qwen3-4B pass, against the rule above: W3 M = 4 887 vs
 //    915 us, W4 M = 3 856 vs 889, M = 5 1160 vs 1235, M = 8 1183 vs 1586, M = 16 1791 vs 2574;
 //    at M = 2 the rule above is the faster one (W3 810 vs 868 us).
-//  * M <= 4 with fewer than two tiles per SM (N < 32 x SMs) and a long K, where the first plan
+//  * M <= 4 with fewer than 1.5 tiles per SM (N < 24 x SMs) and a long K, where the first plan
 //    leaves a warp more than 5 records (the 2560 x 9728 down projection: 160 tiles on 152 SMs,
 //    ~10 records per warp): 4-warp CTAs of 2 tiles instead, K split over a cluster that
 //    doubles until a warp holds at most 5 records and the grid covers every SM (down: 640
@@ -125,9 +129,9 @@ constexpr size_t kSmemPerSm = 228 * 1024, kSmemPerCta = 1024;
 
 void plan(int64_t M, int64_t K, int64_t N, int bits, int sms, laq_gemm_config* out);
 
-// M = 3, 4: X of 3-4 rows beside the ring can leave a CTA just too large for two to share an SM;
-// where the grid needs two per SM, the ring loses stages until two fit (measured on GB300, W4
-// M = 4 fused Qwen3-4B pass: gate|up 11 -> 10 stages, 1032 -> 940 us).
+// X of a long K, or of 3-4 rows, beside the ring can leave a CTA just too large for two to share
+// an SM; where the grid needs two per SM, the ring loses stages until two fit (measured on
+// GB300, W4 M = 4 fused Qwen3-4B pass: gate|up 11 -> 10 stages, 1032 -> 940 us).
 void fit_two_ctas(int64_t M, int64_t K, int64_t N, int bits, int sms, laq_gemm_config* c) {
     const int64_t ctas = (int64_t)ceil_div(N / 16, c->tiles_per_cta) * c->cluster;
     if (ctas <= sms) return;
@@ -188,11 +192,12 @@ void plan(int64_t M, int64_t K, int64_t N, int bits, int sms, laq_gemm_config* o
             if (cl > 1 && cl > G) break;
             for (int nt = 1; nt <= 8; nt *= 2) {
                 const int64_t ctas = (int64_t)ceil_div(T, nt) * cl;
-                if (ctas > 2 * (int64_t)sms) continue;
+                if (ctas > 16 * (int64_t)sms) continue;
                 const int64_t gc = (G + cl - 1) / cl;
                 const int64_t per_warp = (gc + (8 / nt) - 1) / (8 / nt);
-                const double cost =
-                    (double)per_warp * (ctas > sms ? 1.3 : 1.0) * (cl > 1 ? 1.02 : 1.0);
+                const int64_t waves = (ctas + 2 * sms - 1) / (2 * sms);
+                const double cost = (double)(per_warp + 2) * (double)waves *
+                                    (ctas > sms ? 1.3 : 1.0) * (cl > 1 ? 1.02 : 1.0);
                 if (cost < best_cost - 1e-9 || (cost < best_cost + 1e-9 && ctas < best_ctas)) {
                     best_cost = cost;
                     best_ctas = ctas;
@@ -203,7 +208,7 @@ void plan(int64_t M, int64_t K, int64_t N, int bits, int sms, laq_gemm_config* o
         }
         const int64_t gc8 = (G + best_cl - 1) / best_cl;
         const int64_t wt8 = gc8 < 8 / best_nt ? gc8 : 8 / best_nt;
-        if (T >= 2 && T < 2 * (int64_t)sms && (gc8 + wt8 - 1) / wt8 > 5) {
+        if (T >= 2 && 2 * T < 3 * (int64_t)sms && (gc8 + wt8 - 1) / wt8 > 5) {
             best_nt = 2;
             best_cl = 1;
             warps_max = 4;
@@ -226,7 +231,7 @@ void plan(int64_t M, int64_t K, int64_t N, int bits, int sms, laq_gemm_config* o
     out->stages = st;
     out->pdl = 0;
     out->reserved[0] = out->reserved[1] = out->reserved[2] = 0;
-    if (M > 2 && M <= 4) fit_two_ctas(M, K, N, bits, sms, out);
+    if (M <= 4) fit_two_ctas(M, K, N, bits, sms, out);
 }
 
 laq_status run_gemm(const void* X, int64_t M, int64_t K, int64_t N, const void* packed,

@@ -255,12 +255,33 @@ def test_plan_shares_x_across_tiles_above_m_two(L):
     assert laq.laq_gemm_plan(1, 2560, 6144, 3, 152).tiles_per_cta == 2
 
 
+def test_plan_of_the_decode_pass_projections(L):
+    """The launch shapes (tiles per CTA, warps, cluster, ring stages) of the fused Qwen3-4B and
+    Qwen3-8B projections at M = 1 on 152 SMs, each the best or within 1 % of the best of a
+    sweep of every shape inside the pass on GB300."""
+    shape = lambda M, K, N, b: tuple(laq.laq_gemm_plan(M, K, N, b, 152).as_dict()[k]
+                                     for k in ("tiles_per_cta", "warps", "cluster", "stages"))
+    for bits in (3, 4):
+        for M in (1, 2):
+            assert shape(M, 2560, 6144, bits) == (2, 8, 1, 6)      # q|k|v
+            assert shape(M, 4096, 2560, bits) == (1, 8, 1, 5)      # o
+            assert shape(M, 2560, 19456, bits) == (4, 8, 1, 11)    # gate|up
+            assert shape(M, 9728, 2560, bits) == (2, 4, 8, 6)      # down
+        assert shape(1, 4096, 6144, bits) == (2, 8, 1, 9)
+        assert shape(1, 4096, 4096, bits) == (1, 8, 1, 5)
+        # 1536 tiles: 2-tile CTAs in three waves, not one wave of 8-tile CTAs
+        assert shape(1, 4096, 24576, bits) == (2, 8, 1, 9)
+        # 256 tiles (1.7 per SM): no cluster; at W4 the ring gives up stages so that two CTAs
+        # share an SM
+        assert shape(1, 12288, 4096, bits) == (1, 8, 1, 13 if bits == 3 else 10)
+
+
 @pytest.mark.parametrize("bits", [3, 4])
 def test_plan_splits_k_of_narrow_outputs_at_m_one(L, bits):
-    # Fewer than two 16-column tiles per SM and a K long enough that 8-warp CTAs would leave a
+    # Fewer than 1.5 16-column tiles per SM and a K long enough that 8-warp CTAs would leave a
     # warp more than 5 records: 4-warp CTAs of 2 tiles, K split over a cluster until a warp
     # holds at most 5 records and the grid covers every SM.
-    for K, N, cl in ((9728, 2560, 8), (12288, 4096, 8)):
+    for K, N, cl in ((9728, 2560, 8),):
         c = laq.laq_gemm_plan(1, K, N, bits, 152)
         assert (c.tiles_per_cta, c.warps, c.cluster) == (2, 4, cl), (K, N, c.as_dict())
         per_warp = c.tiles_per_cta * -(-(K // 128) // c.cluster) / c.warps
