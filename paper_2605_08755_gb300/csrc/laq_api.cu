@@ -182,8 +182,24 @@ void plan(int64_t M, int64_t K, int64_t N, int bits, int sms, laq_gemm_config* o
         if (M > 8 && G >= 64 && best_cl >= 2) {
             warps_max = 16;
             best_cl /= 2;
+        } else if (M > 4 && M <= 8 && G >= 64 && 2 * T < 3 * (int64_t)sms &&
+                   (bits == 4 || M >= 7)) {
+            // M = 5..8 (W3: 7, 8), a long K and fewer than 1.5 tiles per SM (the down
+            // projection): 4-tile CTAs of 4 warps, one per tile, K over a cluster of 8 -- small
+            // CTAs, two or more per SM.  Measured on GB300, fused Qwen3-4B pass, against 8-tile
+            // 8-warp CTAs with a cluster of 8: W4 M = 5 1135 -> 1104 us, M = 8 1350 -> 1130 (one
+            // such CTA per SM fits there; with a shallower ring, 1202), W3 M = 8 1186 -> 1166;
+            // but W3 M = 5, 6 1162 -> 1184, 1173 -> 1195, so W3 keeps the 8-warp shape there.
+            best_nt = 4;
+            best_cl = 8;
+            warps_max = 4;
         } else if (M > 4 && best_cl == 1 && (int64_t)ceil_div(T, best_nt) >= sms) {
             warps_max = 16;
+            // one 16-warp CTA per SM at a time: a grid between one and two CTAs per SM leaves
+            // some SMs two in turn, so K goes over a cluster of 2 (measured on GB300, Qwen3-8B
+            // W3 M = 16 gate|up, 192 -> 384 CTAs: pass 3183 -> 3099 us)
+            const int64_t ctas = ceil_div(T, best_nt);
+            if (ctas > sms && ctas < 2 * (int64_t)sms && G >= 2) best_cl = 2;
         }
     } else {
         double best_cost = 1e300;
@@ -231,7 +247,7 @@ void plan(int64_t M, int64_t K, int64_t N, int bits, int sms, laq_gemm_config* o
     out->stages = st;
     out->pdl = 0;
     out->reserved[0] = out->reserved[1] = out->reserved[2] = 0;
-    if (M <= 4) fit_two_ctas(M, K, N, bits, sms, out);
+    if (M <= 4 || out->warps <= 8) fit_two_ctas(M, K, N, bits, sms, out);
 }
 
 laq_status run_gemm(const void* X, int64_t M, int64_t K, int64_t N, const void* packed,

@@ -234,10 +234,19 @@ def test_plan_shares_x_across_tiles_above_m_two(L):
     assert laq.laq_gemm_plan(3, 2560, 19456, 4, 152).stages == 11
     assert laq.laq_gemm_plan(4, 2560, 19456, 3, 152).stages == 11
     # M > 4: 8 tiles per CTA, and a cluster K split towards one CTA per SM
-    c = laq.laq_gemm_plan(5, 9728, 2560, 3, 152)
-    assert (c.tiles_per_cta, c.cluster) == (8, 8)
-    c = laq.laq_gemm_plan(8, 9728, 2560, 3, 152)
-    assert (c.tiles_per_cta, c.warps, c.cluster) == (8, 8, 8)
+    c = laq.laq_gemm_plan(8, 2560, 6144, 3, 152)
+    assert (c.tiles_per_cta, c.warps, c.cluster) == (8, 8, 4)
+    # M = 5..8, long K and fewer than 1.5 tiles per SM (down): 4-tile CTAs of 4 warps, cluster 8
+    # (at W3 from M = 7; W3 M = 5, 6 keep 8-tile 8-warp CTAs)
+    for M, bits in ((5, 4), (6, 4), (7, 3), (8, 3), (8, 4)):
+        c = laq.laq_gemm_plan(M, 9728, 2560, bits, 152)
+        assert (c.tiles_per_cta, c.warps, c.cluster) == (4, 4, 8), (M, bits)
+    for M in (5, 6):
+        c = laq.laq_gemm_plan(M, 9728, 2560, 3, 152)
+        assert (c.tiles_per_cta, c.warps, c.cluster, c.stages) == (8, 8, 8, 11)
+    # 16-warp CTAs (one per SM at a time) whose grid falls between one and two per SM: cluster 2
+    c = laq.laq_gemm_plan(16, 4096, 24576, 3, 152)
+    assert (c.tiles_per_cta, c.warps, c.cluster) == (8, 16, 2)
     # M > 4 where that leaves one 8-warp CTA per SM: 16-warp CTAs (two warps per tile); the
     # long-K down projection at M > 8 with half the cluster
     c = laq.laq_gemm_plan(8, 2560, 19456, 3, 152)
