@@ -24,7 +24,12 @@
 //   6. how precisely each form accumulates: every A and B element equal (so the fragment layout
 //      does not matter), the accumulator started at 2^20, and the 32 (e4m3) or 16 (f16)
 //      products 2^-e each; D - 2^20 is exact in fp32 for every e here, so any shortfall is the
-//      tensor core's own alignment of small addends.
+//      tensor core's own alignment of small addends;
+//   7. the W3 record loop with an 8-bit A operand (part 3's loop, measured the same way): a
+//      lane's six words hold its 64 codes as two 3-bit fields per byte (48 codes) and, in bits
+//      6-7 of every byte, the other 16; the extraction makes 16 e4m3 registers of 8 + q (34
+//      integer instructions) and 12 mma.sync.m16n8k32 contract them with x as three e4m3
+//      terms.
 // Every wait is bounded.
 //
 //   nvcc -gencode arch=compute_103a,code=sm_103a -O3 -Xptxas -v -o /tmp/mma_rate \
@@ -84,6 +89,78 @@ __device__ __forceinline__ void mma16832_e4m3(float (&d)[4], uint32_t a0, uint32
         : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
         : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
 }
+// 7. One record's 64 codes of a lane into 16 e4m3 A registers (four k32 steps x a0..a3) of
+// 8 + q: words 0-5 hold two codes per byte (bits 0-2, 3-5); bits 6-7 of the bytes of words 0-3
+// give bits 0-1 of the last 16 codes, bits 6 and 7 of words 4 and 5 their bit 2.
+__device__ __forceinline__ void extract3_e4m3(const uint32_t (&wd)[6], uint32_t (&a)[4][4]) {
+    const uint32_t E = 0x50505050u, m3 = 0x07070707u, m2 = 0x03030303u, m1 = 0x04040404u;
+    uint32_t r[16];
+#pragma unroll
+    for (int w = 0; w < 6; ++w) {
+        r[2 * w] = (wd[w] & m3) | E;
+        r[2 * w + 1] = ((wd[w] >> 3) & m3) | E;
+    }
+    r[12] = ((wd[0] >> 6) & m2) | ((wd[4] >> 4) & m1) | E;
+    r[13] = ((wd[1] >> 6) & m2) | ((wd[4] >> 5) & m1) | E;
+    r[14] = ((wd[2] >> 6) & m2) | ((wd[5] >> 4) & m1) | E;
+    r[15] = ((wd[3] >> 6) & m2) | ((wd[5] >> 5) & m1) | E;
+#pragma unroll
+    for (int t = 0; t < 4; ++t)
+#pragma unroll
+        for (int i = 0; i < 4; ++i) a[t][i] = r[4 * t + i];
+}
+
+// FULL: the extraction above; else each A register is one record word or'ed with the exponent
+// (the 12 MMAs and the loads alone).
+template <bool FULL>
+__global__ void __launch_bounds__(512, 1) record_loop_e4m3(int records, unsigned long long* out,
+                                                           float* sink) {
+    extern __shared__ __align__(1024) uint8_t sm[];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    constexpr int kRec = 768, kRing = 16;
+    for (int i = threadIdx.x; i < 16 * kRing * kRec / 4; i += blockDim.x)
+        reinterpret_cast<uint32_t*>(sm)[i] = 0x12345678u * (uint32_t)i;
+    __syncthreads();
+    const uint8_t* mine = sm + (size_t)warp * kRing * kRec;
+    float D[4][4] = {};
+    // x as three e4m3 terms (1.0, 2^-4, 2^-8 per byte), a fixed B as in part 3
+    const uint32_t b[3][2] = {{0x38383838u, 0x38383838u ^ (uint32_t)(lane & 7)},
+                              {0x18181818u, 0x18181818u},
+                              {0x08080808u, 0x08080808u}};
+    const unsigned long long t0 = clk();
+    for (int r = 0; r < records; r += 8) {
+#pragma unroll 1
+        for (int g = 0; g < 8; ++g) {
+            const uint8_t* rec = mine + ((r + g) % kRing) * kRec;
+            const uint4 c0 = *reinterpret_cast<const uint4*>(rec + lane * 16);
+            const uint2 c1 = *reinterpret_cast<const uint2*>(rec + 512 + lane * 8);
+            const uint32_t wd[6] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y};
+            uint32_t a[4][4];
+            if (FULL) {
+                extract3_e4m3(wd, a);
+            } else {
+#pragma unroll
+                for (int t = 0; t < 4; ++t)
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) a[t][i] = wd[(4 * t + i) % 6] | 0x50505050u;
+            }
+#pragma unroll
+            for (int t = 0; t < 4; ++t)
+#pragma unroll
+                for (int term = 0; term < 3; ++term)
+                    mma16832_e4m3(D[(3 * t + term) & 3], a[t][0], a[t][1], a[t][2], a[t][3],
+                                  b[term][0], b[term][1]);
+        }
+    }
+    __syncthreads();
+    const unsigned long long t1 = clk();
+    float s = 0.f;
+#pragma unroll
+    for (int c = 0; c < 4; ++c) s += D[c][0] + D[c][1] + D[c][2] + D[c][3];
+    if (s == 12345.f) sink[0] = s;
+    if (threadIdx.x == 0) out[blockIdx.x] = t1 - t0;
+}
+
 // 6. One MMA with every A element a, every B element b and C = c; D[0] of lane 0 to out.
 __global__ void accum_probe(uint32_t a8, uint32_t b8, uint32_t a16, uint32_t b16, float c,
                             float* out) {
@@ -397,5 +474,17 @@ int main() {
                (double)hv[0] - 1048576.0, 32.0 / (1 << e), (double)hv[1] - 1048576.0,
                16.0 / (1 << e));
     }
+
+    cudaFuncSetAttribute(record_loop_e4m3<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    record_loop_e4m3<true><<<P, 512, smem>>>(records, out, sink);
+    if (cudaDeviceSynchronize() != cudaSuccess) { printf("error 9\n"); return 1; }
+    printf("7. W3 record loop from shared memory, 16 warps, e4m3 A (34 integer instructions, "
+           "12 mma.sync.m16n8k32): %.1f cycles per record per SM\n",
+           (double)fetch() / (16.0 * records));
+    cudaFuncSetAttribute(record_loop_e4m3<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    record_loop_e4m3<false><<<P, 512, smem>>>(records, out, sink);
+    if (cudaDeviceSynchronize() != cudaSuccess) { printf("error 10\n"); return 1; }
+    printf("   the same with one or per A register instead of the extraction: %.1f cycles per "
+           "record per SM\n", (double)fetch() / (16.0 * records));
     return 0;
 }
