@@ -154,7 +154,9 @@ typedef struct {
 } laq_gemm_config;
 
 /* The configuration laq_gemm_wxg128 uses for this shape on a GPU with `num_sms` SMs (host-only
- * computation; no device access).  Returns the same argument statuses as laq_gemm_wxg128. */
+ * computation; no device access; the shared memory of an SM is taken as sm_100 / sm_103's
+ * 228 KB, so that two CTAs fit one SM where the grid needs it).  Returns the same argument
+ * statuses as laq_gemm_wxg128. */
 laq_status laq_gemm_plan(int64_t M, int64_t K, int64_t N, int bits, int num_sms,
                          laq_gemm_config *out);
 
