@@ -7,8 +7,9 @@ projection's fp16 weights (regenerated from their seeds) and multiplies every ou
 routines split over the host's cores (bit-identical to the single-threaded definitions, pinned
 in tests/test_oracle_pins.py).  Scales and zeros must match bit for bit, every Y within the
 stated tolerance.  Cases: the Qwen3-4B W3 M = 1 pass in both forms, W4, the batch paths at
-M = 4 and M = 16 (two MMAs per k16 step), a planned W4 M = 2 pass, and the Qwen3-8B pass with
-1 % outlier weights in its faster, planned form.
+M = 4, 8 (W4: the down projection in 4-warp CTAs with a cluster of 8) and 16 (two MMAs per k16
+step), a planned W4 M = 2 pass, and the Qwen3-8B pass with 1 % outlier weights in both forms
+(the graph's gate|up in three waves of 2-tile CTAs, its down unclustered).
 """
 import numpy as np
 import pytest
@@ -34,7 +35,9 @@ CASES = [
     ("qwen3-4b", 3, 4, False),
     ("qwen3-4b", 3, 16, False),
     ("qwen3-4b", 4, 2, True),
+    ("qwen3-4b", 4, 8, False),
     ("qwen3-8b", 3, 1, True),
+    ("qwen3-8b", 3, 1, False),
 ]
 
 
